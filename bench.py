@@ -1,0 +1,376 @@
+#!/usr/bin/env python3
+"""Benchmark of the certified cache lookup on GB300.
+
+A step is one batch of the online lookup (Algorithm 2: certified screen,
+recheck and nearest-hit selection) against a cache built beforehand with the
+certified insertion of Algorithm 1. Default workload: the scale stress case,
+a 4,000,000-entry cache of d = 128 FP32 GuardNet-like features (C = 200
+classes, Lipschitz-constrained head) probed in batches of 4,096 queries, 25%
+of them near-duplicates of cached rows. Inputs are seeded synthetic data
+(synth.py); the key table (2.06 GB) is larger than L2, so no L2 flush is
+needed between steps.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
+  python bench.py --impl reference ...   # FP64 CPU oracle on host cores
+
+Prints one JSON line (rank 0). Under torchrun each rank runs an independent
+replica on its own GPU ("replicas only"; the lookup never exchanges data),
+and the line reports the units of all ranks over the slowest rank's time.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import synth  # noqa: E402
+
+METRIC = "certified probe queries/s and query-key pairs/s at N=4M; % of HBM/TC roofline"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+TF32_OVER_BF16 = 1.1 / 2.25  # nominal dense TF32 / BF16 tensor rates of GB300
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=200)
+    p.add_argument("--warmup", type=int, default=5)
+    p.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    p.add_argument("--workload", default="scale", choices=sorted(synth.WORKLOADS))
+    p.add_argument("--path", default="auto", choices=["auto", "tensor", "exact"])
+    p.add_argument("--cpu-seconds", type=float, default=15.0, help="budget of the oracle CPU baseline")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    return p.parse_args()
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            return json.load(f), "measured"
+    return dict(FALLBACK_PEAKS), "fallback"
+
+
+# ---------------------------------------------------------------- distributed plumbing
+class Dist:
+    def __init__(self):
+        self.world = int(os.environ.get("WORLD_SIZE", "1"))
+        self.rank = int(os.environ.get("RANK", "0"))
+        self.local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+        self.pg = None
+        if self.world > 1:
+            import torch.distributed as dist
+            os.environ.setdefault("MASTER_ADDR", "127.0.0.1")
+            dist.init_process_group("gloo", rank=self.rank, world_size=self.world)
+            self.pg = dist
+
+    def barrier(self):
+        if self.pg:
+            self.pg.barrier()
+
+    def max(self, x: float) -> float:
+        if not self.pg:
+            return x
+        import torch
+        t = torch.tensor([x], dtype=torch.float64)
+        self.pg.all_reduce(t, op=self.pg.ReduceOp.MAX)
+        return float(t.item())
+
+    def sum(self, x: float) -> float:
+        if not self.pg:
+            return x
+        import torch
+        t = torch.tensor([x], dtype=torch.float64)
+        self.pg.all_reduce(t, op=self.pg.ReduceOp.SUM)
+        return float(t.item())
+
+    def close(self):
+        if self.pg:
+            self.pg.destroy_process_group()
+
+
+def aggregate(dist: Dist, units: float, seconds: float) -> tuple[float, float]:
+    """Whole-job throughput: units of all ranks over the slowest rank's time."""
+    total = dist.sum(units)
+    tmax = dist.max(seconds)
+    return total / tmax, tmax
+
+
+# ---------------------------------------------------------------- clocks
+class Clocks:
+    FIELDS = ["index", "clocks.sm", "clocks.max.sm", "power.draw", "clocks_event_reasons.active",
+              "clocks_event_reasons.hw_slowdown", "clocks_event_reasons.hw_thermal_slowdown",
+              "clocks_event_reasons.sw_thermal_slowdown", "clocks_event_reasons.sw_power_cap"]
+
+    def __init__(self, gpu_index: int):
+        self.f = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+        try:
+            self.p = subprocess.Popen(["nvidia-smi", "--query-gpu=" + ",".join(self.FIELDS),
+                                       "--format=csv,noheader,nounits", "-i", str(gpu_index), "-lms", "100"],
+                                      stdout=self.f, stderr=subprocess.DEVNULL)
+        except OSError:
+            self.p = None
+        self.t0 = self.t1 = None
+
+    def mark_start(self):
+        self.t0 = time.time()
+
+    def mark_end(self):
+        self.t1 = time.time()
+
+    def stop(self) -> dict:
+        if self.p is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        time.sleep(0.15)
+        self.p.terminate()
+        self.p.wait()
+        self.f.seek(0)
+        rows = [r.split(",") for r in self.f.read().strip().splitlines() if r.strip()]
+        os.unlink(self.f.name)
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for r in rows:
+            r = [x.strip() for x in r]
+            if len(r) < 9:
+                continue
+            try:
+                sm.append(float(r[1]))
+                smax.append(float(r[2]))
+            except ValueError:
+                continue
+            for name, v in zip(names, r[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(name)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(smax) if smax else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ---------------------------------------------------------------- workload
+def workload_data(w: synth.Workload):
+    W, b = synth.head(w)
+    rows = synth.cache_rows(w)
+    Q, _ = synth.queries(w, rows)
+    return W, b, rows, Q
+
+
+def roofline(w: synth.Workload, N: int, B: int, kernel_ms: float, pk: dict, pk_kind: str) -> dict:
+    flops = 2.0 * B * N * w.d
+    bytes_ = N * (4.0 * w.d + 4.0) + 4.0 * B * w.d + 16.0 * B
+    tf32_peak = pk["bf16_tflops"] * TF32_OVER_BF16
+    hbm_peak = pk["hbm_gbs"]
+    t_tc = flops / (tf32_peak * 1e12)
+    t_hbm = bytes_ / (hbm_peak * 1e9)
+    s = kernel_ms * 1e-3
+    if t_tc >= t_hbm:
+        ach = flops / s / 1e12
+        return {"bound": "tensor", "achieved": ach, "peak": tf32_peak, "unit": "TFLOP/s", "frac": ach / tf32_peak,
+                "traffic": None, "algorithmic_flops": flops, "algorithmic_bytes": bytes_,
+                "peak_source": f"{pk_kind} bf16 burst x nominal tf32/bf16 ratio {TF32_OVER_BF16:.4f}",
+                "kernel": "k_probe_tc", "kernel_ms": kernel_ms,
+                "hbm_frac": bytes_ / s / 1e9 / hbm_peak}
+    ach = bytes_ / s / 1e9
+    return {"bound": "hbm", "achieved": ach, "peak": hbm_peak, "unit": "GB/s", "frac": ach / hbm_peak,
+            "traffic": None, "algorithmic_flops": flops, "algorithmic_bytes": bytes_,
+            "peak_source": f"{pk_kind} copy bandwidth", "kernel": "k_probe_tc", "kernel_ms": kernel_ms}
+
+
+def cpu_baseline(w, W, b, rows, Q, budget_s: float) -> dict:
+    """The FP64 oracle as it stands, on the host cores, on a bounded sample:
+    the first n queries against the whole cache (n sized to the budget)."""
+    import oracle
+    t0 = time.perf_counter()
+    sigma = oracle.sigma_max(W)
+    cache = oracle.build_cache(W, b, sigma, rows)
+    t_build = time.perf_counter() - t0
+    n = max(1, oracle.threads())
+    t0 = time.perf_counter()
+    oracle.probe(cache["keys"], cache["radius"], cache["label"], Q[:n])
+    t1 = time.perf_counter() - t0
+    total_q, total_t = n, t1
+    if t1 < budget_s:
+        m = int(min(len(Q) - n, max(0, (budget_s - t1) / t1 * n)))
+        if m > 0:
+            t0 = time.perf_counter()
+            oracle.probe(cache["keys"], cache["radius"], cache["label"], Q[n:n + m])
+            total_t += time.perf_counter() - t0
+            total_q += m
+    N = len(cache["keys"])
+    return {"value": total_q / total_t, "unit": "queries/s", "cores": oracle.threads(), "kind": "oracle",
+            "pairs_per_s": total_q * N / total_t,
+            "sample": f"{total_q} queries of the '{w.name}' workload against the full {N}-entry cache "
+                      f"(FP64 brute force, {total_t:.1f} s; oracle cache build {t_build:.1f} s untimed)"}
+
+
+# ---------------------------------------------------------------- our arm
+def run_ours(args, dist: Dist):
+    import torch
+
+    from paper_2608_13144_gb300.lipcache import LipCache
+
+    w = synth.WORKLOADS[args.workload]
+    dev = torch.device("cuda", dist.local_rank)
+    torch.cuda.set_device(dev)
+    pk, pk_kind = peaks()
+    W, b, rows, Q = workload_data(w)
+    stream = torch.cuda.current_stream(dev)
+
+    cache = LipCache(w.d, w.C, w.N, device=dev)
+    sigma = cache.set_head(torch.from_numpy(W).to(dev), torch.from_numpy(b).to(dev))
+    # certified insertion (Algorithm 1), timed separately
+    rows_d = torch.from_numpy(rows).to(dev)
+    torch.cuda.synchronize(dev)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    n_acc = 0
+    for s, e in synth.batches(w.N, w.insert_batch):
+        n_acc += cache.insert(rows_d[s:e])[2]
+    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    insert_ms = e0.elapsed_time(e1)
+    del rows_d
+    cache.set_probe_path(args.path)
+    cache.reserve(w.batch)
+    N = cache.size
+
+    # query batches resident in HBM
+    nb = max(1, len(Q) // w.batch)
+    Qd = torch.from_numpy(Q[: nb * w.batch]).to(dev).view(nb, w.batch, w.d)
+    B = w.batch
+    outs = [(torch.empty(B, dtype=torch.int64, device=dev), torch.empty(B, dtype=torch.int32, device=dev),
+             torch.empty(B, dtype=torch.float32, device=dev)) for _ in range(nb)]
+    for i in range(args.warmup):
+        cache.probe(Qd[i % nb], out=outs[i % nb])
+    torch.cuda.synchronize(dev)
+    cache.reset_stats()
+    cache.enable_timing(True)
+
+    clk = Clocks(dist.local_rank)
+    dist.barrier()
+    torch.cuda.synchronize(dev)
+    clk.mark_start()
+    e0.record(stream)
+    for i in range(args.steps):
+        cache.probe(Qd[i % nb], out=outs[i % nb])
+    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    clk.mark_end()
+    dist.barrier()
+    step_s = e0.elapsed_time(e1) * 1e-3
+    clocks = clk.stop()
+    info = cache.info()
+    cache.enable_timing(False)
+    kernel_ms = info["kernel_ms_total"] / max(1, info["kernel_launches"])
+    hits = sum(int((o[0] >= 0).sum()) for o in outs[: min(nb, args.steps)])
+    hit_rate = hits / (min(nb, args.steps) * B)
+
+    value, tmax = aggregate(dist, args.steps * B, step_s)
+
+    # end to end through the host-buffer entry point: H2D of the queries,
+    # probe, D2H of index/label/distance, every step
+    hq = [torch.from_numpy(np.ascontiguousarray(Q[i * B:(i + 1) * B])).pin_memory() for i in range(nb)]
+    ho = [(torch.empty(B, dtype=torch.int64).pin_memory(), torch.empty(B, dtype=torch.int32).pin_memory(),
+           torch.empty(B, dtype=torch.float32).pin_memory()) for _ in range(nb)]
+    for i in range(min(3, args.warmup + 1)):
+        cache.probe_host(hq[i % nb], out=ho[i % nb])
+    e2e_steps = max(1, min(args.steps, 50))
+    dist.barrier()
+    t0 = time.perf_counter()
+    for i in range(e2e_steps):
+        cache.probe_host(hq[i % nb], out=ho[i % nb])
+    e2e_s = time.perf_counter() - t0
+    e2e_value, _ = aggregate(dist, e2e_steps * B, e2e_s)
+
+    cpu = None
+    if dist.rank == 0 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(w, W, b, rows, Q, args.cpu_seconds)
+    cache.close()
+
+    rf = roofline(w, N, B, kernel_ms, pk, pk_kind)
+    line = {
+        "metric": METRIC, "value": value, "unit": "queries/s", "n_gpus": dist.world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": tmax / args.steps * 1e3, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "tf32" if info["last_probe_path"] == 1 else "fp32",
+        "data": "synthetic (seeded Gaussian-mixture GuardNet features; no datasets or trained weights)",
+        "config": {"workload": w.name, "N": N, "d": w.d, "C": w.C, "batch": B, "radius": "conservative",
+                   "probe_path": {1: "tensor", 2: "exact"}[info["last_probe_path"]],
+                   "parallelism": f"replicas{dist.world}" if dist.world > 1 else "single",
+                   "l2": f"inputs larger than L2 ({N * (4 * info['d_pad'] + 16) / 1e9:.2f} GB key table)"},
+        "pairs_per_s": value * N,
+        "roofline": rf,
+        "cpu_baseline": cpu,
+        "e2e": {"value": e2e_value, "unit": "queries/s", "h2d_bytes_per_step": B * w.d * 4,
+                "d2h_bytes_per_step": B * (8 + 4 + 4)},
+        "gpu_launches": 3 * args.steps,
+        "clocks": clocks,
+        "insert": {"rows": w.N, "accepted": n_acc, "ms": insert_ms, "rows_per_s": w.N / (insert_ms * 1e-3),
+                   "batch": w.insert_batch},
+        "stats": {"sigma": sigma, "hit_rate": hit_rate,
+                  "candidates_per_query": info["candidates"] / max(1, args.steps * B),
+                  "device_errors": info["device_errors"], "kernel_ms": kernel_ms},
+    }
+    return line
+
+
+# ---------------------------------------------------------------- reference arm (the oracle)
+def run_reference(args, dist: Dist):
+    """The FP64 CPU oracle, as it stands, timed on the host cores on the same
+    workload: each step probes a bounded sample of queries (one per core)
+    against the whole cache."""
+    import oracle
+    w = synth.WORKLOADS[args.workload]
+    W, b, rows, Q = workload_data(w)
+    sigma = oracle.sigma_max(W)
+    cache = oracle.build_cache(W, b, sigma, rows)
+    N = len(cache["keys"])
+    n = max(1, oracle.threads())
+    for i in range(args.warmup):
+        s = (i * n) % max(1, len(Q) - n)
+        oracle.probe(cache["keys"], cache["radius"], cache["label"], Q[s:s + n])
+    t0 = time.perf_counter()
+    for i in range(args.steps):
+        s = ((args.warmup + i) * n) % max(1, len(Q) - n)
+        oracle.probe(cache["keys"], cache["radius"], cache["label"], Q[s:s + n])
+    t = time.perf_counter() - t0
+    value = args.steps * n / t
+    sample = f"{n} queries per step of the '{w.name}' workload against the full {N}-entry cache (FP64 brute force)"
+    return {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "queries/s", "n_gpus": dist.world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": t / args.steps * 1e3, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": w.name, "N": N, "d": w.d, "C": w.C, "batch": w.batch, "radius": "conservative"},
+        "pairs_per_s": value * N,
+        "cpu_baseline": {"value": value, "unit": "queries/s", "cores": oracle.threads(), "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": value, "unit": "queries/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+
+
+def main():
+    args = parse()
+    dist = Dist()
+    try:
+        if args.impl == "reference":
+            if dist.rank != 0:
+                return
+            line = run_reference(args, dist)
+        else:
+            line = run_ours(args, dist)
+        if dist.rank == 0:
+            print(json.dumps(line), flush=True)
+    finally:
+        if args.impl != "reference":
+            dist.close()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,219 @@
+/*
+ * lipcache.h — C ABI of the GB300-native certified cache lookup.
+ *
+ * The library implements the data-parallel hot path of LipCache
+ * (arxiv 2608.13144): certified insertion of GuardNet features into a
+ * feature cache (Sec. 3.3, Algorithm 1; Eqs. 17-21, 29) and batched online
+ * lookup with MainNet fallback (Sec. 3.4, Algorithm 2; Eqs. 13-15).
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ *  - Every function returns a lipcache_status. On failure nothing the caller
+ *    owns has been written unless stated, and lipcache_last_error() returns
+ *    a thread-local, human-readable message. No C++ exception crosses the ABI.
+ *  - Pointers are DEVICE pointers (CUDA global memory of the device the cache
+ *    was created on) unless marked "host". The caller owns every input and
+ *    output buffer; the library owns the cache table, its copies of W and b,
+ *    sigma_max(W) and all scratch memory.
+ *  - Work is enqueued on the caller's stream (a cudaStream_t; NULL = legacy
+ *    default stream). Functions that return a host scalar synchronise that
+ *    stream before returning; lipcache_probe does not and returns as soon as
+ *    its kernels are enqueued.
+ *  - Feature vectors are FP32, row-major, d contiguous floats per row, any
+ *    4-byte alignment. Indices are int64 in cache insertion order.
+ *  - A cache handle is not thread-safe: calls on one handle must be
+ *    serialised by the caller. Distinct handles are independent.
+ *  - Inputs are not validated element by element: a NaN logit margin fails
+ *    r > 0 (the row is rejected); a NaN query fails the strict hit test
+ *    (it misses and falls back to MainNet).
+ */
+#ifndef LIPCACHE_H
+#define LIPCACHE_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Opaque cache handle. */
+typedef struct lipcache lipcache_t;
+
+/* Binary-compatible with cudaStream_t / CUstream. */
+typedef struct CUstream_st* lipcache_stream_t;
+
+typedef enum lipcache_status {
+  LIPCACHE_OK = 0,
+  LIPCACHE_E_INVALID = 1,         /* bad argument (size, pointer, mode) */
+  LIPCACHE_E_STATE = 2,           /* call not allowed now (e.g. probe before set_head) */
+  LIPCACHE_E_DEGENERATE_HEAD = 3, /* sigma_max(W) <= 0: Algorithm 1 stops construction */
+  LIPCACHE_E_FULL = 4,            /* insert would exceed the capacity; nothing inserted */
+  LIPCACHE_E_NOT_CONVERGED = 5,   /* spectral power iteration hit its iteration limit */
+  LIPCACHE_E_CUDA = 6,            /* a CUDA runtime call failed (message has the detail) */
+  LIPCACHE_E_NOMEM = 7,           /* device or host allocation failed */
+  LIPCACHE_E_DEVICE = 8           /* a kernel reported an error (a bounded wait expired) */
+} lipcache_status;
+
+/* Radius modes rho (policy tuple, Sec. 3.4). */
+#define LIPCACHE_RADIUS_CONSERVATIVE 0 /* r  = m / (sigma_max(W) sqrt 2), Eq. 21 */
+#define LIPCACHE_RADIUS_TIGHT 1        /* r* = min_j (s_y - s_j) / ||W_y - W_j||, Eq. 29 */
+
+/* Probe kernels. Both return identical results; they differ in speed. */
+#define LIPCACHE_PROBE_AUTO 0   /* tensor path when supported (d <= 256), else exact */
+#define LIPCACHE_PROBE_TENSOR 1 /* tcgen05 TF32 screen, then exact FP32 recheck of candidates */
+#define LIPCACHE_PROBE_EXACT 2  /* exact FP32 distance of every pair on CUDA cores */
+
+/* Limits checked by lipcache_create. */
+#define LIPCACHE_MAX_DIM 1024
+#define LIPCACHE_MAX_CLASSES 1024
+#define LIPCACHE_MAX_CAPACITY 2147483647LL /* indices are packed in 31 bits */
+
+typedef struct lipcache_info {
+  int32_t d;                /* feature dimension */
+  int32_t C;                /* classes */
+  int32_t d_pad;            /* row stride of the key table: d rounded up to 32 */
+  int32_t radius_mode;      /* LIPCACHE_RADIUS_* */
+  int64_t capacity;         /* maximum number of cache entries */
+  int64_t size;             /* current number of cache entries */
+  int32_t head_set;         /* 1 after a successful lipcache_set_head */
+  int32_t sigma_iterations; /* power iterations used by the last set_head */
+  double sigma;             /* sigma_max(W) of the current head (0 before set_head) */
+  double sigma_residual;    /* ||W^T W v - theta v|| / theta at exit */
+  double radius_scale;      /* kappa in (0, 1]: radius tightening factor (Sec. 5.4) */
+  double eps_recheck;       /* relative deflation of r^2 covering the FP32 recheck error */
+  double c_screen;          /* relative slack of the tensor-core screen */
+  int64_t candidates;       /* screen candidates rechecked since the last reset */
+  int64_t device_errors;    /* kernel-reported errors since the last reset */
+  int32_t probe_path;       /* LIPCACHE_PROBE_* configured for lipcache_probe */
+  int32_t last_probe_path;  /* path that served the last probe */
+  float last_probe_ms;      /* main-kernel time of the last probe (timing enabled) */
+  int32_t num_sms;          /* SMs of the device */
+  double kernel_ms_total;   /* summed main-kernel time of timed probes since the last reset */
+  int64_t kernel_launches;  /* number of timed probes in kernel_ms_total */
+} lipcache_info;
+
+/*
+ * Create an empty cache for d-dimensional GuardNet features and a C-class
+ * head (Sec. 3.1 notation: z in R^d, W in R^{C x d}). Allocates the key table
+ * for `capacity` entries on the current CUDA device.
+ *   d           1 .. LIPCACHE_MAX_DIM
+ *   C           2 .. LIPCACHE_MAX_CLASSES
+ *   capacity    1 .. LIPCACHE_MAX_CAPACITY
+ *   radius_mode LIPCACHE_RADIUS_CONSERVATIVE or LIPCACHE_RADIUS_TIGHT
+ *   out         host; receives the handle (NULL on failure)
+ * Errors: E_INVALID, E_NOMEM, E_CUDA (e.g. no device).
+ */
+lipcache_status lipcache_create(int32_t d, int32_t C, int64_t capacity, int32_t radius_mode, lipcache_t** out);
+
+/*
+ * Install the GuardNet affine head f(z) = W z + b (Eq. 5) and compute its
+ * Lipschitz constant sigma_max(W) (Eqs. 17-19; Algorithm 1, first step) by
+ * power iteration on W^T W in FP64, accelerated by repeated squaring, until
+ * successive Rayleigh quotients agree to 1e-13 and the eigen-residual is
+ * below 1e-10 theta.
+ *   W         C x d row-major FP32 (device); copied, the caller may free it after return
+ *   b         C FP32 (device); copied
+ *   sigma_out host, nullable; receives sigma_max(W)
+ * Synchronises `stream`. Allowed only while the cache is empty (radii depend
+ * on W). Errors: E_STATE (cache not empty), E_DEGENERATE_HEAD (sigma <= 0;
+ * Algorithm 1 stops construction), E_NOT_CONVERGED, E_INVALID (NULL W or b),
+ * E_CUDA.
+ */
+lipcache_status lipcache_set_head(lipcache_t* h, const float* W, const float* b, double* sigma_out,
+                                  lipcache_stream_t stream);
+
+/*
+ * Certify n candidate rows and append the accepted ones (Algorithm 1 with
+ * every accepted candidate selected). For each row z: logits s = W z + b,
+ * y^G = argmax s (lowest class on ties), margin m = s_y - max_{j!=y} s_j
+ * (Eq. 20), radius r = kappa * m / (sigma sqrt 2) (Eq. 21) or the tight r*
+ * (Eq. 29); payload = payload[i] if given else y^G (proxy label). A row is
+ * skipped if require_consistency != 0 and payload != y^G, else if r <= 0.
+ * Accepted rows get consecutive indices in input order.
+ *   H           n x d FP32 (device)
+ *   n           >= 0; n == 0 is a no-op
+ *   payload     n int32 (device), nullable -> proxy labels y^G
+ *   out_index   n int64 (device), nullable; cache index or -1 if skipped
+ *   out_radius  n FP32 (device), nullable; r of every row rounded toward zero
+ *               (also for skipped rows)
+ *   n_accepted  host, nullable; number of rows appended
+ * Synchronises `stream`. All or nothing: if size + n > capacity nothing is
+ * written and E_FULL is returned. Errors: E_STATE (no head), E_FULL,
+ * E_INVALID, E_CUDA.
+ */
+lipcache_status lipcache_insert(lipcache_t* h, const float* H, int64_t n, const int32_t* payload,
+                                int32_t require_consistency, int64_t* out_index, float* out_radius,
+                                int64_t* n_accepted, lipcache_stream_t stream);
+
+/*
+ * Batched certified lookup (Algorithm 2, Eqs. 13-15): for every query q the
+ * hit set H(q) = { i : ||q - z_i|| < r_i } (strict) and the nearest hit
+ * i* = argmin_{i in H(q)} ||q - z_i||, ties to the lowest index. A miss
+ * means "fall back to MainNet".
+ * The GPU accepts an entry only if its FP32 distance is below r_i deflated by
+ * a proven error bound, so it never accepts a pair whose exact distance is
+ * not below r_i; pairs within ~2e-6 relative of the boundary may be missed.
+ *   Q          B x d FP32 (device)
+ *   B          >= 0; B == 0 is a no-op
+ *   out_index  B int64 (device): i*, or -1 on a miss
+ *   out_label  B int32 (device), nullable: payload of i*, or -1
+ *   out_dist   B FP32 (device), nullable: ||q - z_i*|| (FP32), or +inf
+ * Asynchronous on `stream`. Errors: E_STATE (no head), E_INVALID, E_NOMEM
+ * (scratch growth), E_CUDA. A device-side failure (bounded wait expired)
+ * turns the affected queries into misses and is counted in
+ * lipcache_info.device_errors.
+ */
+lipcache_status lipcache_probe(lipcache_t* h, const float* Q, int64_t B, int64_t* out_index, int32_t* out_label,
+                               float* out_dist, lipcache_stream_t stream);
+
+/*
+ * lipcache_probe for callers holding HOST buffers: copies Q to the device,
+ * probes, copies the results back and synchronises `stream`.
+ *   Q_host     B x d FP32 (host; pinned memory gives asynchronous copies)
+ *   out_*_host host, same meaning as lipcache_probe (out_label/out_dist nullable)
+ */
+lipcache_status lipcache_probe_host(lipcache_t* h, const float* Q_host, int64_t B, int64_t* out_index_host,
+                                    int32_t* out_label_host, float* out_dist_host, lipcache_stream_t stream);
+
+/* Select the probe kernel (LIPCACHE_PROBE_*). E_INVALID for an unknown path
+ * or TENSOR when d > 256. */
+lipcache_status lipcache_set_probe_path(lipcache_t* h, int32_t path);
+
+/* Radius tightening kappa in (0, 1] (Sec. 5.4): radii of rows inserted
+ * afterwards are multiplied by kappa. Only while the cache is empty. */
+lipcache_status lipcache_set_radius_scale(lipcache_t* h, double kappa);
+
+/* Spectral-norm options: `squarings` (0..60) normalised squarings of W^T W
+ * before the power iteration and `max_iter` (>= 1) power iterations. */
+lipcache_status lipcache_set_spectral_options(lipcache_t* h, int32_t squarings, int32_t max_iter);
+
+/* Pre-size the probe scratch for batches of up to max_batch queries so that
+ * later probes allocate nothing. */
+lipcache_status lipcache_reserve(lipcache_t* h, int64_t max_batch);
+
+/* When on, each probe times its main kernel (the screen/recheck kernel, not
+ * the prologue and finalize) with a pair of CUDA events recorded on `stream`.
+ * lipcache_get_info returns the last duration and the sum and count since the
+ * last lipcache_reset_stats. */
+lipcache_status lipcache_enable_timing(lipcache_t* h, int32_t on);
+
+/* Fill *info (host). Synchronises the device work of this handle. */
+lipcache_status lipcache_get_info(lipcache_t* h, lipcache_info* info);
+
+/* Zero the candidate / device-error counters and the kernel-time sum. */
+lipcache_status lipcache_reset_stats(lipcache_t* h);
+
+/* Number of cache entries (0 for NULL). */
+int64_t lipcache_size(const lipcache_t* h);
+
+/* Free the cache and its device memory. NULL-safe. */
+void lipcache_destroy(lipcache_t* h);
+
+/* Message of the last failed call on this thread ("" if none). */
+const char* lipcache_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* LIPCACHE_H */

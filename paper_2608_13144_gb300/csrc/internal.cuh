@@ -1,0 +1,196 @@
+// Internal declarations of the lipcache library (not part of the C ABI).
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <cmath>
+#include <stdexcept>
+#include <string>
+
+#include "../../include/lipcache.h"
+
+namespace lc {
+
+// ---------------------------------------------------------------- errors
+struct Error : std::runtime_error {
+  lipcache_status status;
+  Error(lipcache_status s, const std::string& m) : std::runtime_error(m), status(s) {}
+};
+
+#define LC_CUDA(call)                                                                          \
+  do {                                                                                         \
+    cudaError_t e_ = (call);                                                                   \
+    if (e_ != cudaSuccess)                                                                     \
+      throw ::lc::Error(e_ == cudaErrorMemoryAllocation ? LIPCACHE_E_NOMEM : LIPCACHE_E_CUDA, \
+                        std::string(#call) + ": " + cudaGetErrorString(e_));                 \
+  } while (0)
+
+#define LC_LAUNCH_CHECK(name)                                                                      \
+  do {                                                                                             \
+    cudaError_t e_ = cudaGetLastError();                                                           \
+    if (e_ != cudaSuccess)                                                                         \
+      throw ::lc::Error(LIPCACHE_E_CUDA, std::string("launch of ") + (name) + ": " + cudaGetErrorString(e_)); \
+  } while (0)
+
+#define LC_REQUIRE(cond, status, msg) \
+  do {                                \
+    if (!(cond)) throw ::lc::Error((status), (msg)); \
+  } while (0)
+
+// ---------------------------------------------------------------- numerics
+// Unit roundoff of FP32 and FP64 (round to nearest).
+constexpr double kU32 = 5.9604644775390625e-08;   // 2^-24
+constexpr double kU64 = 1.1102230246251565e-16;   // 2^-53
+
+inline double gamma32(int n) { return n * kU32 / (1.0 - n * kU32); }
+inline double gamma64(int n) { return n * kU64 / (1.0 - n * kU64); }
+
+// Relative error bound of the canonical FP32 squared distance (see
+// dist2_canonical): every term e_j^2 passes one subtraction rounding (which
+// at most doubles in the square), at most 32 roundings inside its 32-wide
+// chunk and at most d_pad/32 - 1 roundings while the chunk sums are added, so
+// |S~ - S| <= gamma_{d_pad/32 + 33} S (all terms are non-negative). A small
+// slack covers the FP64 arithmetic that forms the threshold.
+inline double eps_recheck(int dpad) { return gamma32(dpad / 32 + 33) * (1.0 + 1.0 / 1024); }
+
+// Relative slack of the tensor-core screen. With TF32 operands (10 explicit
+// mantissa bits, error <= 2^-10 relative whether truncated or rounded) a
+// product is within (2^-9 + 2^-20)|q_j k_j|; FP32-or-better accumulation of
+// d_pad products adds at most d_pad 2^-22 sum|q_j k_j|. The sum |q_j k_j| is
+// at most ||q|| ||k|| <= (||q||^2 + ||k||^2)/2. The bound is doubled for
+// safety, and the FP32 norms (error gamma_{d_pad}) plus one final rounding
+// are added on top.
+inline double c_screen(int dpad) {
+  return 2.0 * (std::ldexp(1.0, -9) + std::ldexp(1.0, -20) + dpad * std::ldexp(1.0, -22)) + 2.0 * gamma32(dpad) +
+         std::ldexp(1.0, -20);
+}
+
+// sigma from the power iteration is a Rayleigh-quotient estimate (from
+// below); radii used for acceptance divide by sigma * (1 + kSigmaSlack).
+constexpr double kSigmaSlack = 1e-9;
+
+// ---------------------------------------------------------------- state
+struct SpecResult {
+  double sigma;
+  double theta;
+  double residual_rel;
+  int iterations;
+  int converged;
+  int degenerate;
+  int pad;
+};
+
+struct DevStats {
+  unsigned long long candidates;
+  unsigned long long errors;
+  int abort_flag;  // set by a kernel whose bounded wait expired; cleared per probe
+  int pad;
+};
+
+// Per-entry table of the cache (structure of arrays, capacity entries).
+struct Table {
+  float* keys = nullptr;     // capacity x dpad, zero padded
+  float* kn = nullptr;       // FP32 ||k||^2
+  float* tau = nullptr;      // screen threshold term
+  float* rr = nullptr;       // acceptance threshold on the FP32 squared distance
+  float* radius = nullptr;   // reported radius r (rounded toward zero)
+  int32_t* label = nullptr;  // payload
+  int32_t* yG = nullptr;     // GuardNet label of the cached feature
+};
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+}  // namespace lc
+
+struct lipcache {
+  int device = 0;
+  int num_sms = 0;
+  int d = 0, C = 0, dpad = 0;
+  int64_t capacity = 0, size = 0;
+  int64_t table_rows = 0;  // capacity rounded up to 256 (whole key tiles)
+  int radius_mode = 0;
+  double radius_scale = 1.0;
+  int probe_path = LIPCACHE_PROBE_AUTO;
+  int last_probe_path = 0;
+  int squarings = 40, max_iter = 1000;
+  bool head_set = false;
+  double sigma = 0.0, sigma_residual = 0.0;
+  int sigma_iterations = 0;
+
+  // head
+  float* W = nullptr;        // C x d
+  float* b = nullptr;        // C
+  double* Wnorm = nullptr;   // C
+  double* pairnorm = nullptr;  // C x C (tight mode)
+  double* gram[2] = {nullptr, nullptr};  // d x d FP64
+  lc::SpecResult* spec = nullptr;        // device
+  lc::SpecResult* spec_host = nullptr;   // pinned
+
+  lc::Table table;
+
+  // insert scratch (grows)
+  int64_t ins_cap = 0;
+  uint8_t* ins_accept = nullptr;
+  int32_t* ins_yG = nullptr;
+  int32_t* ins_label = nullptr;
+  float* ins_radius = nullptr;
+  float* ins_rr = nullptr;
+  float* ins_kn = nullptr;
+  float* ins_tau = nullptr;
+  int32_t* ins_rank = nullptr;
+  int32_t* ins_bcount = nullptr;
+  int32_t* ins_boffset = nullptr;
+  int64_t* ins_total = nullptr;       // device
+  int64_t* ins_total_host = nullptr;  // pinned
+
+  // probe scratch (grows)
+  int64_t q_cap = 0;  // rows (multiple of 128)
+  float* qpad = nullptr;
+  float* kappa = nullptr;
+  unsigned long long* best = nullptr;
+  // host-buffer probe staging
+  int64_t hq_cap = 0;
+  float* hq = nullptr;
+  int64_t* hidx = nullptr;
+  int32_t* hlabel = nullptr;
+  float* hdist = nullptr;
+
+  lc::DevStats* stats = nullptr;
+  lc::DevStats* stats_host = nullptr;
+
+  // main-kernel timing: a ring of event pairs harvested lazily
+  static constexpr int kTimingRing = 64;
+  bool timing = false;
+  cudaEvent_t tev0[kTimingRing] = {}, tev1[kTimingRing] = {};
+  int64_t t_issued = 0, t_harvested = 0;
+  double t_ms_total = 0.0;
+  int64_t t_count = 0;
+  float last_ms = 0.f;
+
+  double eps_rc = 0.0, c_scr = 0.0;
+  lc::EncodeTiledFn encode = nullptr;
+};
+
+namespace lc {
+
+// ---------------------------------------------------------------- launchers
+// spectral.cu
+void spectral_norm(lipcache* h, cudaStream_t s);
+// certify.cu
+void certify_insert(lipcache* h, const float* H, int64_t n, const int32_t* payload, int require_consistency,
+                    int64_t* out_index, float* out_radius, cudaStream_t s);
+// probe.cu
+void probe(lipcache* h, const float* Q, int64_t B, int64_t* out_index, int32_t* out_label, float* out_dist,
+           cudaStream_t s);
+bool tensor_path_supported(int dpad);
+// probe_tc.cu
+void launch_probe_tc(lipcache* h, int64_t B, cudaStream_t s);
+// api.cu: harvest completed timing events (blocking on the oldest if `all`
+// or if the ring is full).
+void harvest_timing(lipcache* h, bool all);
+
+}  // namespace lc

@@ -1,0 +1,149 @@
+"""Python binding of the certified cache lookup (argument marshalling only).
+
+Every step of the lookup runs in the CUDA kernels of liblipcache.so, called
+through the C ABI of include/lipcache.h. PyTorch provides device memory and
+the current stream; tensors are passed by pointer.
+"""
+from __future__ import annotations
+
+import ctypes as C
+
+import torch
+
+from . import _lib
+from ._lib import Info, check
+
+RADIUS_MODES = {"conservative": _lib.RADIUS_CONSERVATIVE, "tight": _lib.RADIUS_TIGHT}
+PROBE_PATHS = {"auto": _lib.PROBE_AUTO, "tensor": _lib.PROBE_TENSOR, "exact": _lib.PROBE_EXACT}
+
+
+def _stream(device: torch.device):
+    return C.c_void_p(torch.cuda.current_stream(device).cuda_stream)
+
+
+def _ptr(t):
+    return C.c_void_p(t.data_ptr()) if t is not None else None
+
+
+class LipCache:
+    """Feature cache C = {(z_i, y~_i, r_i)} on one GPU (Sec. 3.3-3.4)."""
+
+    def __init__(self, d: int, C_classes: int, capacity: int, radius_mode: str = "conservative",
+                 device: int | torch.device | None = None):
+        self.L = _lib.load()
+        self.device = torch.device("cuda", torch.cuda.current_device() if device is None else
+                                   torch.device("cuda", device).index if isinstance(device, int) else device.index)
+        self.d, self.C = int(d), int(C_classes)
+        h = C.c_void_p()
+        with torch.cuda.device(self.device):
+            check(self.L.lipcache_create(self.d, self.C, int(capacity), RADIUS_MODES[radius_mode], C.byref(h)))
+        self._h = h
+
+    # -- lifecycle
+    def close(self):
+        if getattr(self, "_h", None):
+            self.L.lipcache_destroy(self._h)
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def __enter__(self):
+        return self
+
+    def __exit__(self, *exc):
+        self.close()
+
+    def _dev(self, t: torch.Tensor, dtype: torch.dtype, name: str) -> torch.Tensor:
+        if t.device != self.device or t.dtype != dtype:
+            raise ValueError(f"{name} must be a {dtype} tensor on {self.device}")
+        return t.contiguous()
+
+    # -- Algorithm 1
+    def set_head(self, W: torch.Tensor, b: torch.Tensor) -> float:
+        W = self._dev(W, torch.float32, "W")
+        b = self._dev(b, torch.float32, "b")
+        if tuple(W.shape) != (self.C, self.d) or tuple(b.shape) != (self.C,):
+            raise ValueError("W must be C x d and b must have C entries")
+        sigma = C.c_double()
+        check(self.L.lipcache_set_head(self._h, _ptr(W), _ptr(b), C.byref(sigma), _stream(self.device)))
+        return sigma.value
+
+    def insert(self, H: torch.Tensor, payload: torch.Tensor | None = None, require_consistency: bool = False):
+        """Certify and append rows of H. Returns (index, radius, n_accepted):
+        index[i] is the cache index of row i or -1 if it was skipped."""
+        H = self._dev(H, torch.float32, "H")
+        n = H.shape[0]
+        if H.dim() != 2 or (n and H.shape[1] != self.d):
+            raise ValueError("H must be n x d")
+        if payload is not None:
+            payload = self._dev(payload, torch.int32, "payload")
+        index = torch.empty(n, dtype=torch.int64, device=self.device)
+        radius = torch.empty(n, dtype=torch.float32, device=self.device)
+        acc = C.c_int64()
+        check(self.L.lipcache_insert(self._h, _ptr(H), n, _ptr(payload), int(bool(require_consistency)),
+                                     _ptr(index), _ptr(radius), C.byref(acc), _stream(self.device)))
+        return index, radius, acc.value
+
+    # -- Algorithm 2
+    def probe(self, Q: torch.Tensor, out=None):
+        """Nearest certified hit per query: (index, label, dist); -1/-1/inf on a miss."""
+        Q = self._dev(Q, torch.float32, "Q")
+        B = Q.shape[0]
+        if Q.dim() != 2 or (B and Q.shape[1] != self.d):
+            raise ValueError("Q must be B x d")
+        if out is None:
+            out = (torch.empty(B, dtype=torch.int64, device=self.device),
+                   torch.empty(B, dtype=torch.int32, device=self.device),
+                   torch.empty(B, dtype=torch.float32, device=self.device))
+        idx, lab, dist = out
+        check(self.L.lipcache_probe(self._h, _ptr(Q), B, _ptr(idx), _ptr(lab), _ptr(dist), _stream(self.device)))
+        return idx, lab, dist
+
+    def probe_host(self, Q, out=None):
+        """Probe from host memory (pinned tensors give asynchronous copies)."""
+        Q = Q.contiguous()
+        if Q.device.type != "cpu" or Q.dtype != torch.float32:
+            raise ValueError("Q must be a float32 CPU tensor")
+        B = Q.shape[0]
+        if out is None:
+            out = (torch.empty(B, dtype=torch.int64), torch.empty(B, dtype=torch.int32),
+                   torch.empty(B, dtype=torch.float32))
+        idx, lab, dist = out
+        check(self.L.lipcache_probe_host(self._h, _ptr(Q), B, _ptr(idx), _ptr(lab), _ptr(dist),
+                                         _stream(self.device)))
+        return idx, lab, dist
+
+    # -- options / introspection
+    def set_probe_path(self, path: str):
+        check(self.L.lipcache_set_probe_path(self._h, PROBE_PATHS[path]))
+
+    def set_radius_scale(self, kappa: float):
+        check(self.L.lipcache_set_radius_scale(self._h, float(kappa)))
+
+    def set_spectral_options(self, squarings: int, max_iter: int):
+        check(self.L.lipcache_set_spectral_options(self._h, int(squarings), int(max_iter)))
+
+    def reserve(self, max_batch: int):
+        check(self.L.lipcache_reserve(self._h, int(max_batch)))
+
+    def enable_timing(self, on: bool = True):
+        check(self.L.lipcache_enable_timing(self._h, int(bool(on))))
+
+    def reset_stats(self):
+        check(self.L.lipcache_reset_stats(self._h))
+
+    def info(self) -> dict:
+        inf = Info()
+        check(self.L.lipcache_get_info(self._h, C.byref(inf)))
+        return {name: getattr(inf, name) for name, _ in Info._fields_}
+
+    @property
+    def size(self) -> int:
+        return int(self.L.lipcache_size(self._h))
+
+    def __len__(self):
+        return self.size

@@ -1,0 +1,46 @@
+"""Comparison rules between the CUDA path and the FP64 oracle.
+
+Bit-exact: acceptance of inserted rows, cache indices, hit/miss decisions,
+selected indices and labels. Within 1e-5 relative: radii and distances.
+The only tolerated disagreements are queries in the oracle's 1e-5 band:
+some entry has |D - r| <= 1e-5 r (decision band) or the two nearest hits
+are within 1e-5 of each other (selection band). A GPU hit the oracle
+rejects (an unsafe accept) is never tolerated.
+"""
+import numpy as np
+
+import oracle
+
+RTOL = 1e-5
+
+
+def check_insert(g_index, g_radius, n_acc, ref):
+    cert = ref["cert"]
+    assert n_acc == int(cert["accept"].sum())
+    bad = np.nonzero(g_index != ref["index"])[0]
+    assert bad.size == 0, f"{bad.size} rows differ in acceptance/index, first {bad[:5]}"
+    r = cert["radius"]
+    m = np.isfinite(r) & (r > 0)
+    np.testing.assert_allclose(g_radius[m], r[m], rtol=RTOL)
+    # reported radii are rounded toward zero, never above the FP64 value
+    assert np.all(g_radius[m].astype(np.float64) <= r[m] * (1 + 1e-12))
+
+
+def check_probe(gi, gl, gd, ref, Q, orc):
+    keys, radius, labels = ref["keys"], ref["radius"], ref["label"]
+    hits = gi >= 0
+    if hits.any():
+        qi = np.nonzero(hits)[0]
+        D = oracle.pair_dist(Q, keys, qi, gi[hits])
+        unsafe = ~(D < radius[gi[hits]])
+        assert not unsafe.any(), f"{unsafe.sum()} unsafe accepts, e.g. query {qi[unsafe][:3]}"
+        assert np.array_equal(gl[hits], labels[gi[hits]])
+        np.testing.assert_allclose(gd[hits].astype(np.float64), D, rtol=RTOL)
+    assert np.all(gl[~hits] == -1) and np.all(np.isinf(gd[~hits]))
+    band = (orc["decision_band"] | orc["selection_band"]).astype(bool)
+    mism = gi != orc["index"]
+    out = mism & ~band
+    assert not out.any(), (f"{out.sum()} queries differ outside the 1e-5 band: "
+                           f"gpu {gi[out][:5]} oracle {orc['index'][out][:5]}")
+    return {"queries": len(gi), "hits": int(hits.sum()), "oracle_hits": int((orc["index"] >= 0).sum()),
+            "band": int(band.sum()), "band_mismatch": int((mism & band).sum())}

@@ -1,0 +1,82 @@
+"""Host-side checks of the C ABI that need no GPU: the library loads, exports
+every symbol include/lipcache.h declares, and rejects bad arguments before
+touching a device."""
+import ctypes as C
+import os
+import re
+import subprocess
+
+import pytest
+
+from conftest import ROOT
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2608_13144_gb300.build import build
+    build()
+    from paper_2608_13144_gb300 import _lib
+    return _lib.load()
+
+
+def _declared_functions():
+    text = open(os.path.join(ROOT, "include", "lipcache.h")).read()
+    return sorted(set(re.findall(r"^\s*(?:lipcache_status|void|int64_t|const char\*)\s+(lipcache_\w+)\s*\(", text,
+                                 re.M)))
+
+
+def test_exports_every_declared_symbol(lib):
+    from paper_2608_13144_gb300 import _lib
+    declared = _declared_functions()
+    assert declared, "no declarations parsed"
+    assert sorted(_lib.EXPORTS) == declared
+    out = subprocess.run(["nm", "-D", "--defined-only", _lib.LIB_PATH], capture_output=True, text=True).stdout
+    exported = sorted(set(re.findall(r" T (lipcache_\w+)", out)))
+    assert exported == declared
+    for name in declared:
+        assert hasattr(lib, name)
+
+
+def test_no_gpu_runtime_dependency(lib):
+    from paper_2608_13144_gb300 import _lib
+    out = subprocess.run(["ldd", _lib.LIB_PATH], capture_output=True, text=True).stdout
+    assert "libcuda.so" not in out and "libcudart" not in out
+
+
+@pytest.mark.parametrize("args", [(0, 10, 100, 0), (16, 1, 100, 0), (16, 10, 0, 0), (16, 10, 100, 7),
+                                  (2000, 10, 100, 0), (16, 5000, 100, 0), (16, 10, 1 << 40, 0)])
+def test_create_rejects_bad_arguments(lib, args):
+    h = C.c_void_p()
+    st = lib.lipcache_create(*args, C.byref(h))
+    assert st == 1  # E_INVALID, decided before any CUDA call
+    assert not h.value
+    assert lib.lipcache_last_error()
+
+
+def test_null_handle_calls(lib):
+    assert lib.lipcache_size(None) == 0
+    lib.lipcache_destroy(None)
+    assert lib.lipcache_set_head(None, None, None, None, None) == 1
+    assert lib.lipcache_probe(None, None, 0, None, None, None, None) == 1
+    assert lib.lipcache_insert(None, None, 0, None, 0, None, None, None, None) == 1
+
+
+def test_create_without_gpu_fails_cleanly(lib):
+    import torch
+    if torch.cuda.is_available():
+        pytest.skip("a GPU is present")
+    h = C.c_void_p()
+    st = lib.lipcache_create(16, 10, 100, 0, C.byref(h))
+    assert st in (6, 7)  # E_CUDA / E_NOMEM from the runtime
+    assert not h.value
+
+
+def test_numerics_constants():
+    """The slack constants are bounded as the design states: the recheck
+    deflation is far inside the 1e-5 decision band, and the screen slack is
+    of order 2^-8 for the feature sizes of the workloads."""
+    u = 2.0 ** -24
+    for dpad in (32, 64, 128, 256, 1024):
+        g = (dpad / 32 + 33) * u / (1 - (dpad / 32 + 33) * u)
+        assert g < 5e-6
+    assert abs((2 * (2 ** -9 + 2 ** -20 + 128 * 2 ** -22)) - 0.00397) < 1e-4
