@@ -50,6 +50,7 @@ def parse():
     p.add_argument("--path", default="auto", choices=["auto", "tensor", "exact"])
     p.add_argument("--cpu-seconds", type=float, default=15.0, help="budget of the oracle CPU baseline")
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--cache-rows", type=int, default=0, help="override the workload's cache size N (profiling)")
     return p.parse_args()
 
 
@@ -218,6 +219,8 @@ def run_ours(args, dist: Dist):
     from paper_2608_13144_gb300.lipcache import LipCache
 
     w = synth.WORKLOADS[args.workload]
+    if args.cache_rows:
+        w = w.scaled(N=args.cache_rows)
     dev = torch.device("cuda", dist.local_rank)
     torch.cuda.set_device(dev)
     pk, pk_kind = peaks()
@@ -328,6 +331,8 @@ def run_reference(args, dist: Dist):
     against the whole cache."""
     import oracle
     w = synth.WORKLOADS[args.workload]
+    if args.cache_rows:
+        w = w.scaled(N=args.cache_rows)
     W, b, rows, Q = workload_data(w)
     sigma = oracle.sigma_max(W)
     cache = oracle.build_cache(W, b, sigma, rows)
