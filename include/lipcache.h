@@ -175,6 +175,28 @@ lipcache_status lipcache_probe(lipcache_t* h, const float* Q, int64_t B, int64_t
 lipcache_status lipcache_probe_host(lipcache_t* h, const float* Q_host, int64_t B, int64_t* out_index_host,
                                     int32_t* out_label_host, float* out_dist_host, lipcache_stream_t stream);
 
+/*
+ * lipcache_probe for callers that cannot allocate device memory while they
+ * run — e.g. a serving loop whose device memory belongs entirely to another
+ * allocator, or whose latency budget cannot absorb cudaMalloc/cudaFree, which
+ * may block and synchronise the device. The paper has no counterpart: this is
+ * an interface choice of this library, not part of the method.
+ * Same arguments, results and errors as lipcache_probe, but the probe's
+ * scratch lives in one fixed array compiled into the library
+ * (LIPCACHE_NOALLOC_SCRATCH_BYTES per device, held by every GPU that loads
+ * the library until the process exits) and nothing is allocated.
+ * Limit: ceil(B/128)*128 * (4*d_pad + 12) bytes, plus alignment, must fit the
+ * array (e.g. 4,096 queries at d <= 256); larger batches get E_INVALID with
+ * the sizes in the message. The first call on a device resolves the array's
+ * device address (cudaGetSymbolAddress); make that first call before any
+ * stream capture. All calls on a device share the array: calls whose GPU work
+ * overlaps (other streams, handles or threads on the same device) race on it
+ * and must be serialised by the caller.
+ */
+#define LIPCACHE_NOALLOC_SCRATCH_BYTES 4259840
+lipcache_status lipcache_probe_noalloc(lipcache_t* h, const float* Q, int64_t B, int64_t* out_index,
+                                       int32_t* out_label, float* out_dist, lipcache_stream_t stream);
+
 /* Select the probe kernel (LIPCACHE_PROBE_*). E_INVALID for an unknown path
  * or TENSOR when d > 256. */
 lipcache_status lipcache_set_probe_path(lipcache_t* h, int32_t path);

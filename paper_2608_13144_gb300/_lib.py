@@ -15,10 +15,12 @@ OK, E_INVALID, E_STATE, E_DEGENERATE_HEAD, E_FULL, E_NOT_CONVERGED, E_CUDA, E_NO
 STATUS_NAMES = {0: "OK", 1: "E_INVALID", 2: "E_STATE", 3: "E_DEGENERATE_HEAD", 4: "E_FULL", 5: "E_NOT_CONVERGED",
                 6: "E_CUDA", 7: "E_NOMEM", 8: "E_DEVICE"}
 RADIUS_CONSERVATIVE, RADIUS_TIGHT = 0, 1
+NOALLOC_SCRATCH_BYTES = 4259840  # LIPCACHE_NOALLOC_SCRATCH_BYTES
 PROBE_AUTO, PROBE_TENSOR, PROBE_EXACT = 0, 1, 2
 
 # Every symbol the header declares; tests check the library exports them all.
 EXPORTS = ["lipcache_create", "lipcache_set_head", "lipcache_insert", "lipcache_probe", "lipcache_probe_host",
+           "lipcache_probe_noalloc",
            "lipcache_set_probe_path", "lipcache_set_radius_scale", "lipcache_set_spectral_options",
            "lipcache_reserve", "lipcache_enable_timing", "lipcache_get_info", "lipcache_reset_stats",
            "lipcache_size", "lipcache_destroy", "lipcache_last_error"]
@@ -58,6 +60,7 @@ def load(path: str = LIB_PATH):
         "lipcache_insert": ([vp, vp, i64, vp, i32, vp, vp, C.POINTER(i64), vp], C.c_int),
         "lipcache_probe": ([vp, vp, i64, vp, vp, vp, vp], C.c_int),
         "lipcache_probe_host": ([vp, vp, i64, vp, vp, vp, vp], C.c_int),
+        "lipcache_probe_noalloc": ([vp, vp, i64, vp, vp, vp, vp], C.c_int),
         "lipcache_set_probe_path": ([vp, i32], C.c_int),
         "lipcache_set_radius_scale": ([vp, f64], C.c_int),
         "lipcache_set_spectral_options": ([vp, i32, i32], C.c_int),

@@ -109,6 +109,11 @@ void resolve_encoder(lipcache* h) {
 
 }  // namespace
 
+// Runs fn(ctx) under the same error handling as every other entry point.
+lipcache_status lc::run_guarded(void (*fn)(void*), void* ctx) {
+  return guarded([&] { fn(ctx); });
+}
+
 void lc::harvest_timing(lipcache* h, bool all) {
   while (h->t_harvested < h->t_issued) {
     const int slot = (int)(h->t_harvested % lipcache::kTimingRing);

@@ -189,6 +189,13 @@ void probe(lipcache* h, const float* Q, int64_t B, int64_t* out_index, int32_t* 
 bool tensor_path_supported(int dpad);
 // probe_tc.cu
 void launch_probe_tc(lipcache* h, int64_t B, cudaStream_t s);
+// probe.cu / probe_tc.cu: the probe on caller-provided scratch memory
+void probe_external_scratch(lipcache* h, const float* Q, int64_t B, int64_t* out_index, int32_t* out_label,
+                            float* out_dist, float* qpad, float* kappa, unsigned long long* best, cudaStream_t s);
+void launch_probe_tc_external(lipcache* h, int64_t B, const float* qpad, const float* kappa, unsigned long long* best,
+                              cudaStream_t s);
+// api.cu: run fn(ctx) with the C ABI's error handling (status + message)
+lipcache_status run_guarded(void (*fn)(void*), void* ctx);
 // api.cu: harvest completed timing events (blocking on the oldest if `all`
 // or if the ring is full).
 void harvest_timing(lipcache* h, bool all);

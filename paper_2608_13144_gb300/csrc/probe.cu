@@ -205,4 +205,30 @@ void probe(lipcache* h, const float* Q, int64_t B, int64_t* out_index, int32_t* 
   LC_LAUNCH_CHECK("k_finalize");
 }
 
+// The same launch sequence as probe(), on scratch memory the caller
+// provides (qpad: Bpad x d_pad floats, kappa: Bpad floats, best: Bpad words,
+// Bpad = B rounded up to 128). Allocates nothing.
+void probe_external_scratch(lipcache* h, const float* Q, int64_t B, int64_t* out_index, int32_t* out_label,
+                            float* out_dist, float* qpad, float* kappa, unsigned long long* best, cudaStream_t s) {
+  const int64_t Bpad = (B + 127) / 128 * 128;
+  k_prologue<<<(unsigned)((Bpad + 7) / 8), 256, 0, s>>>(Q, B, h->d, h->dpad, Bpad, qpad, kappa, best,
+                                                      1.0 - h->c_scr, h->stats);
+  LC_LAUNCH_CHECK("k_prologue");
+  int path = h->probe_path;
+  if (path == LIPCACHE_PROBE_AUTO) path = tensor_path_supported(h->dpad) ? LIPCACHE_PROBE_TENSOR : LIPCACHE_PROBE_EXACT;
+  h->last_probe_path = path;
+  if (h->size > 0) {
+    if (path == LIPCACHE_PROBE_TENSOR) {
+      launch_probe_tc_external(h, B, qpad, kappa, best, s);
+    } else {
+      dim3 grid((unsigned)((h->size + kEK - 1) / kEK), (unsigned)((B + kEQ - 1) / kEQ));
+      k_probe_exact<<<grid, 256, 0, s>>>(qpad, B, h->table.keys, h->table.rr, h->size, h->dpad, best);
+      LC_LAUNCH_CHECK("k_probe_exact");
+    }
+  }
+  k_finalize<<<(unsigned)((B + 255) / 256), 256, 0, s>>>(best, B, h->table.label, out_index, out_label, out_dist,
+                                                       h->stats);
+  LC_LAUNCH_CHECK("k_finalize");
+}
+
 }  // namespace lc

@@ -30,6 +30,7 @@
 #include "tc_ptx.cuh"
 
 namespace lc {
+int tc_key_tile(int dpad);
 namespace {
 
 constexpr int kBM = 128;              // queries per tile (MMA M)
@@ -349,7 +350,52 @@ void launch(lipcache* h, int64_t B, cudaStream_t s) {
   LC_LAUNCH_CHECK("k_probe_tc");
 }
 
+template <int BN>
+void launch_external(lipcache* h, int64_t B, const float* qpad, const float* kappa, unsigned long long* best,
+                     cudaStream_t s) {
+  const int64_t Bpad = (B + kBM - 1) / kBM * kBM;
+  CUtensorMap tmQ, tmK;
+  encode_2d(h, &tmQ, qpad, (uint64_t)Bpad, kBM);
+  encode_2d(h, &tmK, h->table.keys, (uint64_t)h->table_rows, BN);
+  TcArgs a;
+  a.nch = h->dpad / kChunkF;
+  a.dpad = h->dpad;
+  a.nq = (int)(Bpad / kBM);
+  const int64_t n_kt = (h->size + BN - 1) / BN;
+  const int64_t target = 2LL * h->num_sms;
+  int n_qg = (int)((target + n_kt - 1) / n_kt);
+  if (n_qg < 1) n_qg = 1;
+  if (n_qg > a.nq) n_qg = a.nq;
+  a.qpg = (a.nq + n_qg - 1) / n_qg;
+  a.n_qg = (a.nq + a.qpg - 1) / a.qpg;
+  const int64_t n_units = n_kt * a.n_qg;
+  LC_REQUIRE(n_units < (1LL << 31), LIPCACHE_E_INVALID, "too many work units");
+  a.n_units = (int)n_units;
+  a.kappa = kappa;
+  a.qpad = qpad;
+  a.keys = h->table.keys;
+  a.tau = h->table.tau;
+  a.rr = h->table.rr;
+  a.best = best;
+  a.stats = h->stats;
+  const Layout<BN> L{a.nch};
+  const int smem = L.total() + 1024;
+  LC_CUDA(cudaFuncSetAttribute(k_probe_tc<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
+  const int grid = (int)(n_units < h->num_sms ? n_units : h->num_sms);
+  k_probe_tc<BN><<<grid, kThreads, smem, s>>>(tmQ, tmK, a);
+  LC_LAUNCH_CHECK("k_probe_tc");
+}
+
 }  // namespace
+
+void launch_probe_tc_external(lipcache* h, int64_t B, const float* qpad, const float* kappa, unsigned long long* best,
+                              cudaStream_t s) {
+  LC_REQUIRE(tensor_path_supported(h->dpad), LIPCACHE_E_INVALID, "the tensor probe supports d <= 256");
+  if (tc_key_tile(h->dpad) == 256)
+    launch_external<256>(h, B, qpad, kappa, best, s);
+  else
+    launch_external<128>(h, B, qpad, kappa, best, s);
+}
 
 int tc_key_tile(int dpad) { return dpad <= 128 ? 256 : 128; }
 

@@ -103,6 +103,17 @@ class LipCache:
         check(self.L.lipcache_probe(self._h, _ptr(Q), B, _ptr(idx), _ptr(lab), _ptr(dist), _stream(self.device)))
         return idx, lab, dist
 
+    def probe_noalloc(self, Q: torch.Tensor, out):
+        """probe() without any device allocation, for callers that cannot
+        allocate while they run: the scratch is a fixed array inside the
+        library (see lipcache_probe_noalloc). `out` must be preallocated;
+        overlapping calls on one device race on the shared array."""
+        Q = self._dev(Q, torch.float32, "Q")
+        idx, lab, dist = out
+        check(self.L.lipcache_probe_noalloc(self._h, _ptr(Q), Q.shape[0], _ptr(idx), _ptr(lab), _ptr(dist),
+                                            _stream(self.device)))
+        return idx, lab, dist
+
     def probe_host(self, Q, out=None):
         """Probe from host memory (pinned tensors give asynchronous copies)."""
         Q = Q.contiguous()
