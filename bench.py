@@ -319,7 +319,8 @@ def run_ours(args, dist: Dist):
                    "batch": w.insert_batch},
         "stats": {"sigma": sigma, "hit_rate": hit_rate,
                   "candidates_per_query": info["candidates"] / max(1, args.steps * B),
-                  "device_errors": info["device_errors"], "kernel_ms": kernel_ms},
+                  "device_errors": info["device_errors"], "kernel_ms": kernel_ms,
+                  "grid": info["last_grid"], "cluster": info["last_cluster"]},
     }
     return line
 

@@ -90,6 +90,8 @@ typedef struct lipcache_info {
   int32_t num_sms;          /* SMs of the device */
   double kernel_ms_total;   /* summed main-kernel time of timed probes since the last reset */
   int64_t kernel_launches;  /* number of timed probes in kernel_ms_total */
+  int32_t last_grid;        /* CTAs launched by the last probe's main kernel */
+  int32_t last_cluster;     /* CTAs per cluster of that launch (1 = no cluster) */
 } lipcache_info;
 
 /*

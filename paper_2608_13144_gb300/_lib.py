@@ -33,7 +33,8 @@ class Info(C.Structure):
                 ("radius_scale", C.c_double), ("eps_recheck", C.c_double), ("c_screen", C.c_double),
                 ("candidates", C.c_int64), ("device_errors", C.c_int64), ("probe_path", C.c_int32),
                 ("last_probe_path", C.c_int32), ("last_probe_ms", C.c_float), ("num_sms", C.c_int32),
-                ("kernel_ms_total", C.c_double), ("kernel_launches", C.c_int64)]
+                ("kernel_ms_total", C.c_double), ("kernel_launches", C.c_int64), ("last_grid", C.c_int32),
+                ("last_cluster", C.c_int32)]
 
 
 class LipCacheError(RuntimeError):

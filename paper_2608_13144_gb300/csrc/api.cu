@@ -388,5 +388,7 @@ LC_API lipcache_status lipcache_get_info(lipcache_t* h, lipcache_info* info) {
     info->num_sms = h->num_sms;
     info->kernel_ms_total = h->t_ms_total;
     info->kernel_launches = h->t_count;
+    info->last_grid = h->last_grid;
+    info->last_cluster = h->last_cluster;
   });
 }

@@ -9,7 +9,7 @@
 #include <stdexcept>
 #include <string>
 
-#include "../../include/lipcache.h"
+#include "lipcache.h"
 
 namespace lc {
 
@@ -116,6 +116,7 @@ struct lipcache {
   double radius_scale = 1.0;
   int probe_path = LIPCACHE_PROBE_AUTO;
   int last_probe_path = 0;
+  int last_grid = 0, last_cluster = 0;
   int squarings = 40, max_iter = 1000;
   bool head_set = false;
   double sigma = 0.0, sigma_residual = 0.0;

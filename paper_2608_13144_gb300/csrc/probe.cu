@@ -192,6 +192,8 @@ void probe(lipcache* h, const float* Q, int64_t B, int64_t* out_index, int32_t* 
       launch_probe_tc(h, B, s);
     } else {
       dim3 grid((unsigned)((h->size + kEK - 1) / kEK), (unsigned)((B + kEQ - 1) / kEQ));
+      h->last_grid = (int)(grid.x * grid.y);
+      h->last_cluster = 1;
       k_probe_exact<<<grid, 256, 0, s>>>(h->qpad, B, h->table.keys, h->table.rr, h->size, h->dpad, h->best);
       LC_LAUNCH_CHECK("k_probe_exact");
     }

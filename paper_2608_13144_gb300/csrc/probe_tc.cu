@@ -12,19 +12,27 @@
 // fl(a - tau_k) >= kappa_q, which therefore never drops an acceptable pair;
 // the separable form costs one subtraction and one max per pair.
 //
-// Schedule (one persistent CTA per SM, 320 threads):
+// Schedule. Persistent CTAs, one per SM, launched as clusters of two. The two
+// CTAs of a cluster own two adjacent key tiles and stream the SAME sequence of
+// query tiles: each CTA TMA-loads one half of every query stage with
+// .multicast::cluster into both CTAs' shared memory, so the L2 delivers each
+// query byte once per pair of SMs (the query stream from L2 is what limits a
+// single CTA). Per CTA (320 threads):
 //   warp 0     TMA producer: the CTA's key tile (BN keys x d_pad, resident,
 //              one barrier pair per 32-float chunk so the next tile streams in
-//              while the last query tile still runs) and the query tiles
-//              (128 queries x 32 floats per stage, 4-stage ring);
+//              while the last query tile still runs) and its half of each
+//              query stage (128 queries x 32 floats per stage, multi-stage ring);
 //   warp 1     allocates TMEM, issues tcgen05.mma kind::tf32 (M=128 queries,
 //              N=BN keys, K=8) from one thread into one of two TMEM
-//              accumulators;
+//              accumulators; releases each query stage in BOTH CTAs;
 //   warps 2-9  epilogue: tcgen05.ld of the accumulator (warp w reads TMEM
 //              lane quarter w % 4, column half (w - 2) / 4), screen, recheck,
 //              atomicMin of the packed (distance, index) word.
-// A work unit is one key tile against a group of query tiles; units are
-// dealt round-robin over the persistent CTAs.
+// A work unit is one key-tile pair against a group of query tiles; units are
+// dealt round-robin over the clusters. When the number of key tiles is odd the
+// last pair's second tile lies past the table: that CTA multiplies the TMA's
+// zero fill and its epilogue skips the unit, so both CTAs still consume every
+// query stage.
 #include "internal.cuh"
 #include "probe_common.cuh"
 #include "tc_ptx.cuh"
@@ -35,19 +43,29 @@ namespace {
 
 constexpr int kBM = 128;              // queries per tile (MMA M)
 constexpr int kChunkF = 32;           // floats per K chunk (one 128-byte swizzle row)
-constexpr int kStages = 4;            // query ring depth
+constexpr int kMaxStages = 8;         // query ring depth limit (runtime count fills shared memory)
+constexpr int kMaxChunks = 8;         // d_pad <= 256
 constexpr int kQStageBytes = kBM * 128;
-constexpr int kThreads = 320;
-constexpr int kEpiWarps = 8;
-constexpr long long kWaitLimit = 1LL << 31;  // ~1 s at GB300 clocks
+constexpr int kQHalfBytes = kQStageBytes / 2;
+#ifndef LC_EPI_WARPS
+#define LC_EPI_WARPS 8
+#endif
+constexpr int kEpiWarps = LC_EPI_WARPS;  // 4 or 8: one or two per SM sub-partition
+constexpr int kThreads = 32 * (2 + kEpiWarps);
+constexpr int kCluster = 2;
+constexpr uint16_t kClusterMask = 0x3;
+constexpr int kSmemBudget = 227 * 1024 - 1024;  // opt-in limit minus the alignment slack
+constexpr long long kWaitLimit = 1LL << 31;     // ~1 s at GB300 clocks
 
 struct TcArgs {
+  int nst;       // query ring stages
   int nch;       // d_pad / 32
   int dpad;
   int nq;        // query tiles
   int qpg;       // query tiles per unit
   int n_qg;      // query groups
-  int n_units;   // key tiles x query groups
+  int n_units;   // key-tile pairs x query groups
+  int n_kt;      // key tiles holding cache entries
   const float* kappa;
   const float* qpad;
   const float* keys;
@@ -61,22 +79,33 @@ template <int BN>
 struct Layout {
   static constexpr int kKChunkBytes = BN * 128;
   static constexpr int kTmemCols = 2 * BN;
-  int nch;
+  static constexpr int kTauBytes = 4 * BN * 4;  // one private tau slice per epilogue warp (kEpiWarps x 4BN/kEpiWarps)
+  int nch, nst;
   __device__ __host__ int kbytes() const { return nch * kKChunkBytes; }
   __device__ __host__ int qoff() const { return kbytes(); }
-  __device__ __host__ int baroff() const { return qoff() + kStages * kQStageBytes; }
-  // barriers: full_k[nch], empty_k[nch], full_q[S], empty_q[S], acc_full[2], acc_empty[2], drain
-  __device__ __host__ int nbar() const { return 2 * nch + 2 * kStages + 5; }
+  __device__ __host__ int tauoff() const { return qoff() + nst * kQStageBytes; }
+  __device__ __host__ int baroff() const { return tauoff() + kTauBytes; }
+  // barriers: full_k[nch], empty_k[nch], full_q[nst], empty_q[nst], acc_full[2], acc_empty[2], drain
+  __device__ __host__ int nbar() const { return 2 * nch + 2 * nst + 5; }
   __device__ __host__ int miscoff() const { return baroff() + 8 * nbar(); }
   __device__ __host__ int total() const { return miscoff() + 16; }
+  // deepest ring that fits the shared-memory budget
+  static __host__ int stages_for(int nch) {
+    for (int n = kMaxStages; n >= 2; --n) {
+      Layout<BN> L{nch, n};
+      if (L.total() <= kSmemBudget) return n;
+    }
+    return 0;
+  }
 };
 
-__device__ __forceinline__ void unit_range(const TcArgs& a, int u, int BN, int& kt, int& qt0, int& qt1) {
-  kt = u / a.n_qg;
-  const int g = u - kt * a.n_qg;
+// Unit u of this cluster -> this CTA's key tile and the query-tile range.
+__device__ __forceinline__ void unit_range(const TcArgs& a, int u, uint32_t rank, int& kt, int& qt0, int& qt1) {
+  const int pair = u / a.n_qg;
+  const int g = u - pair * a.n_qg;
+  kt = pair * kCluster + (int)rank;
   qt0 = g * a.qpg;
   qt1 = min(a.nq, qt0 + a.qpg);
-  (void)BN;
 }
 
 template <int BN>
@@ -84,30 +113,32 @@ __global__ void __launch_bounds__(kThreads, 1)
     k_probe_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK, const TcArgs a) {
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   // 1024-byte alignment of the swizzled tiles
-  unsigned char* smem = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
-  const Layout<BN> L{a.nch};
+  unsigned char* smem =
+      reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+  const Layout<BN> L{a.nch, a.nst};
   const uint32_t s_base = ptx::smem_u32(smem);
   const uint32_t s_k = s_base;
   const uint32_t s_q = s_base + L.qoff();
   const uint32_t s_bar = s_base + L.baroff();
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + L.baroff());
-  (void)bars;
   const uint32_t full_k = s_bar, empty_k = s_bar + 8 * a.nch;
-  const uint32_t full_q = s_bar + 16 * a.nch, empty_q = full_q + 8 * kStages;
-  const uint32_t acc_full = empty_q + 8 * kStages, acc_empty = acc_full + 16, drain = acc_empty + 16;
+  const uint32_t full_q = s_bar + 16 * a.nch, empty_q = full_q + 8 * a.nst;
+  const uint32_t acc_full = empty_q + 8 * a.nst, acc_empty = acc_full + 16, drain = acc_empty + 16;
+  float* tau_s = reinterpret_cast<float*>(smem + L.tauoff());
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L.miscoff());
   volatile int* abort_s = reinterpret_cast<volatile int*>(smem + L.miscoff() + 4);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t rank = ptx::cluster_ctarank();
+  const int cluster_id = blockIdx.x / kCluster, n_clusters = gridDim.x / kCluster;
 
   if (threadIdx.x == 0) {
     for (int c = 0; c < a.nch; ++c) {
       ptx::mbar_init(full_k + 8 * c, 1);
       ptx::mbar_init(empty_k + 8 * c, 1);
     }
-    for (int s = 0; s < kStages; ++s) {
-      ptx::mbar_init(full_q + 8 * s, 1);
-      ptx::mbar_init(empty_q + 8 * s, 1);
+    for (int s = 0; s < a.nst; ++s) {
+      ptx::mbar_init(full_q + 8 * s, 1);         // own arrival; bytes from both CTAs
+      ptx::mbar_init(empty_q + 8 * s, kCluster); // released by the MMA of both CTAs
     }
     for (int b = 0; b < 2; ++b) {
       ptx::mbar_init(acc_full + 8 * b, 1);
@@ -126,6 +157,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   ptx::tc_fence_before();
   __syncthreads();
   ptx::tc_fence_after();
+  ptx::cluster_sync();  // the peer's barriers exist before any multicast reaches them
   const uint32_t tmem = *tmem_slot;
 
   if (warp == 0) {
@@ -134,80 +166,123 @@ __global__ void __launch_bounds__(kThreads, 1)
       int qs = 0;
       uint32_t qph = 0;
       int i = 0;
-      int last_unit_par = -1;
-      uint32_t last_q_par[kStages];
-      bool q_used[kStages];
-      for (int s = 0; s < kStages; ++s) {
+      int last_k_par[kMaxChunks];
+      uint32_t last_q_par[kMaxStages];
+      bool q_used[kMaxStages];
+      for (int c = 0; c < kMaxChunks; ++c) last_k_par[c] = -1;
+      for (int s = 0; s < kMaxStages; ++s) {
         q_used[s] = false;
         last_q_par[s] = 0;
       }
       bool ok = true;
-      for (int u = blockIdx.x; u < a.n_units && ok; u += gridDim.x, ++i) {
+      for (int u = cluster_id; u < a.n_units && ok; u += n_clusters, ++i) {
         int kt, qt0, qt1;
-        unit_range(a, u, BN, kt, qt0, qt1);
-        for (int c = 0; c < a.nch && ok; ++c) {
-          ok = ptx::mbar_wait(empty_k + 8 * c, (uint32_t)(i & 1) ^ 1u, abort_s, kWaitLimit);
-          if (!ok) break;
-          ptx::mbar_expect_tx(full_k + 8 * c, (uint32_t)Layout<BN>::kKChunkBytes);
-          ptx::tma_load_2d(s_k + c * Layout<BN>::kKChunkBytes, &tmK, c * kChunkF, kt * BN, full_k + 8 * c);
-        }
-        if (ok) last_unit_par = i & 1;
+        unit_range(a, u, rank, kt, qt0, qt1);
         for (int qt = qt0; qt < qt1 && ok; ++qt) {
           for (int c = 0; c < a.nch && ok; ++c) {
+            if (qt == qt0) {
+              // key chunk c of this unit, as soon as the previous unit's last
+              // query tile has finished with it (past the table: zero fill)
+              ok = ptx::mbar_wait(empty_k + 8 * c, (uint32_t)(i & 1) ^ 1u, abort_s, kWaitLimit);
+              if (!ok) break;
+              ptx::mbar_expect_tx(full_k + 8 * c, (uint32_t)Layout<BN>::kKChunkBytes);
+              ptx::tma_load_2d(s_k + c * Layout<BN>::kKChunkBytes, &tmK, c * kChunkF, kt * BN, full_k + 8 * c);
+              last_k_par[c] = i & 1;
+            }
+            // stage qs is free in both CTAs; fetch this CTA's half for both
             ok = ptx::mbar_wait(empty_q + 8 * qs, qph ^ 1u, abort_s, kWaitLimit);
             if (!ok) break;
             ptx::mbar_expect_tx(full_q + 8 * qs, (uint32_t)kQStageBytes);
-            ptx::tma_load_2d(s_q + qs * kQStageBytes, &tmQ, c * kChunkF, qt * kBM, full_q + 8 * qs);
+            ptx::tma_load_2d_multicast(s_q + qs * kQStageBytes + rank * kQHalfBytes, &tmQ, c * kChunkF,
+                                       qt * kBM + (int)rank * (kBM / 2), full_q + 8 * qs, kClusterMask);
             q_used[qs] = true;
             last_q_par[qs] = qph;
-            if (++qs == kStages) {
+            if (++qs == a.nst) {
               qs = 0;
               qph ^= 1u;
             }
           }
         }
       }
-      // Let every copy this thread issued land before the CTA can exit.
-      // (Bounded; a phase that already completed returns at once.)
+      // Let every copy into this CTA land before it can exit. (Bounded; a
+      // phase that already completed returns at once.)
       volatile int never = 0;
-      for (int s = 0; s < kStages; ++s)
+      for (int s = 0; s < a.nst; ++s)
         if (q_used[s]) ptx::mbar_wait(full_q + 8 * s, last_q_par[s], &never, kWaitLimit);
-      if (last_unit_par >= 0)
-        for (int c = 0; c < a.nch; ++c) ptx::mbar_wait(full_k + 8 * c, (uint32_t)last_unit_par, &never, kWaitLimit);
+      for (int c = 0; c < a.nch; ++c)
+        if (last_k_par[c] >= 0) ptx::mbar_wait(full_k + 8 * c, (uint32_t)last_k_par[c], &never, kWaitLimit);
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
+    // The tensor pipe queues about one MMA ahead, so this loop keeps the work
+    // between MMA issues minimal: shared-memory descriptors are built once and
+    // advanced by adding encoded offsets (the start-address field holds
+    // address >> 4, so +32 bytes is +2 and never carries out of the field).
     if (lane == 0) {
       constexpr uint32_t idesc = ptx::idesc_tf32(kBM, BN);
+      const uint64_t qdesc0 = ptx::sw128_kmajor_desc(s_q);
+      const uint64_t kdesc0 = ptx::sw128_kmajor_desc(s_k);
+      constexpr uint64_t kQStride = kQStageBytes >> 4;
+      constexpr uint64_t kKStride = Layout<BN>::kKChunkBytes >> 4;
+      const int nst = a.nst, nch = a.nch;
       int qs = 0;
       uint32_t qph = 0;
       int t = 0, i = 0;
       bool ok = true;
-      for (int u = blockIdx.x; u < a.n_units && ok; u += gridDim.x, ++i) {
+      for (int u = cluster_id; u < a.n_units && ok; u += n_clusters, ++i) {
         int kt, qt0, qt1;
-        unit_range(a, u, BN, kt, qt0, qt1);
+        unit_range(a, u, rank, kt, qt0, qt1);
         for (int qt = qt0; qt < qt1 && ok; ++qt, ++t) {
           const int buf = t & 1;
           ok = ptx::mbar_wait(acc_empty + 8 * buf, (uint32_t)((t >> 1) & 1) ^ 1u, abort_s, kWaitLimit);
           if (!ok) break;
           ptx::tc_fence_after();
           const uint32_t d_tmem = tmem + (uint32_t)(buf * BN);
-          for (int c = 0; c < a.nch && ok; ++c) {
-            ok = ptx::mbar_wait(full_k + 8 * c, (uint32_t)(i & 1), abort_s, kWaitLimit);
-            if (ok) ok = ptx::mbar_wait(full_q + 8 * qs, qph, abort_s, kWaitLimit);
-            if (!ok) break;
-            ptx::tc_fence_after();
-            const uint32_t qa = s_q + qs * kQStageBytes;
-            const uint32_t kb = s_k + c * Layout<BN>::kKChunkBytes;
-#pragma unroll
-            for (int kk = 0; kk < 4; ++kk)
-              ptx::mma_tf32(d_tmem, ptx::sw128_kmajor_desc(qa + kk * 32), ptx::sw128_kmajor_desc(kb + kk * 32), idesc,
-                            (c | kk) != 0);
-            ptx::mma_commit(empty_q + 8 * qs);
-            if (qt == qt1 - 1) ptx::mma_commit(empty_k + 8 * c);
-            if (++qs == kStages) {
-              qs = 0;
-              qph ^= 1u;
+          const bool first = qt == qt0, last = qt == qt1 - 1;
+          uint64_t kd = kdesc0;
+          if (first || last) {
+            // Unit edges: the key chunk arrives once per unit (TMA completion on
+            // the mbarrier already orders the copies before the MMA's reads),
+            // and the last query tile hands each chunk back to the producer.
+            for (int c = 0; c < nch; ++c, kd += kKStride) {
+              if (first && !ptx::mbar_wait(full_k + 8 * c, (uint32_t)(i & 1), abort_s, kWaitLimit)) {
+                ok = false;
+                break;
+              }
+              if (!ptx::mbar_wait(full_q + 8 * qs, qph, abort_s, kWaitLimit)) {
+                ok = false;
+                break;
+              }
+              const uint64_t qd = qdesc0 + (uint64_t)qs * kQStride;
+              ptx::mma_tf32(d_tmem, qd, kd, idesc, c != 0);
+              ptx::mma_tf32(d_tmem, qd + 2, kd + 2, idesc, 1u);
+              ptx::mma_tf32(d_tmem, qd + 4, kd + 4, idesc, 1u);
+              ptx::mma_tf32(d_tmem, qd + 6, kd + 6, idesc, 1u);
+              ptx::mma_commit_multicast(empty_q + 8 * qs, kClusterMask);
+              if (last) ptx::mma_commit(empty_k + 8 * c);
+              if (++qs == nst) {
+                qs = 0;
+                qph ^= 1u;
+              }
+            }
+          } else {
+            // Steady state: nothing but the stage wait, four MMAs and the
+            // stage release (no predicated tensor-pipe instructions).
+            for (int c = 0; c < nch; ++c, kd += kKStride) {
+              if (!ptx::mbar_wait(full_q + 8 * qs, qph, abort_s, kWaitLimit)) {
+                ok = false;
+                break;
+              }
+              const uint64_t qd = qdesc0 + (uint64_t)qs * kQStride;
+              ptx::mma_tf32(d_tmem, qd, kd, idesc, c != 0);
+              ptx::mma_tf32(d_tmem, qd + 2, kd + 2, idesc, 1u);
+              ptx::mma_tf32(d_tmem, qd + 4, kd + 4, idesc, 1u);
+              ptx::mma_tf32(d_tmem, qd + 6, kd + 6, idesc, 1u);
+              ptx::mma_commit_multicast(empty_q + 8 * qs, kClusterMask);
+              if (++qs == nst) {
+                qs = 0;
+                qph ^= 1u;
+              }
             }
           }
           if (ok) ptx::mma_commit(acc_full + 8 * buf);
@@ -223,66 +298,79 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ------------------------------------------------------------ epilogue
     const int ew = warp - 2;
     const int quarter = warp & 3;         // TMEM lane quarter this warp may access
-    const int half = ew >> 2;             // column half
-    constexpr int kColsPerWarp = BN / 2;
+    const int half = ew >> 2;             // column slice
+    constexpr int kColsPerWarp = BN * 4 / kEpiWarps;
     constexpr int kChunks = kColsPerWarp / 32;
     const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
+    float* my_tau = tau_s + ew * kColsPerWarp;  // private to this warp
     int t = 0;
     bool ok = true;
     unsigned long long ncand = 0;
-    for (int u = blockIdx.x; u < a.n_units && ok; u += gridDim.x) {
+    for (int u = cluster_id; u < a.n_units && ok; u += n_clusters) {
       int kt, qt0, qt1;
-      unit_range(a, u, BN, kt, qt0, qt1);
+      unit_range(a, u, rank, kt, qt0, qt1);
+      const bool live = kt < a.n_kt;
       const int key0 = kt * BN + half * kColsPerWarp;
-      const float4* tau4 = reinterpret_cast<const float4*>(a.tau + key0);
+      // this warp's screen terms for the unit's key tile, staged once per unit
+      __syncwarp();
+      if (live)
+        for (int v4 = lane; v4 < kColsPerWarp / 4; v4 += 32)
+          reinterpret_cast<float4*>(my_tau)[v4] = __ldg(reinterpret_cast<const float4*>(a.tau + key0) + v4);
+      __syncwarp();
+      float kap = __ldg(a.kappa + qt0 * kBM + quarter * 32 + lane);
       for (int qt = qt0; qt < qt1; ++qt, ++t) {
         const int buf = t & 1;
+        const int row = qt * kBM + quarter * 32 + lane;
+        // next tile's screen constant, fetched while this accumulator is produced
+        const float kap_next = (qt + 1 < qt1) ? __ldg(a.kappa + row + kBM) : 0.f;
         ok = ptx::mbar_wait(acc_full + 8 * buf, (uint32_t)((t >> 1) & 1), abort_s, kWaitLimit);
         ok = __all_sync(0xffffffffu, ok);  // warp-uniform before the aligned TMEM loads
         if (!ok) break;
         ptx::tc_fence_after();
-        const int row = qt * kBM + quarter * 32 + lane;
-        const float kap = __ldg(a.kappa + row);
-        const uint32_t tbase = tmem + lane_base + (uint32_t)(buf * BN + half * kColsPerWarp);
-        uint32_t r[2][32];
-        ptx::tmem_ld32(tbase, r[0]);
-        ptx::tmem_wait_ld();
+        if (live) {
+          const uint32_t tbase = tmem + lane_base + (uint32_t)(buf * BN + half * kColsPerWarp);
+          uint32_t r[2][32];
+          ptx::tmem_ld32(tbase, r[0]);
+          ptx::tmem_wait_ld();
 #pragma unroll
-        for (int ch = 0; ch < kChunks; ++ch) {
-          if (ch + 1 < kChunks) ptx::tmem_ld32(tbase + (uint32_t)((ch + 1) * 32), r[(ch + 1) & 1]);
-          const uint32_t* v = r[ch & 1];
-          float m = -INFINITY;
-          float tv[32];
+          for (int ch = 0; ch < kChunks; ++ch) {
+            if (ch + 1 < kChunks) ptx::tmem_ld32(tbase + (uint32_t)((ch + 1) * 32), r[(ch + 1) & 1]);
+            const uint32_t* v = r[ch & 1];
+            // fl(a - tau) for two columns per instruction, folded into two
+            // independent three-input max chains
+            const uint4* t4 = reinterpret_cast<const uint4*>(my_tau + ch * 32);
+            float m0 = -INFINITY, m1 = -INFINITY;
 #pragma unroll
-          for (int j4 = 0; j4 < 8; ++j4) {
-            const float4 t4 = __ldg(tau4 + ch * 8 + j4);
-            tv[4 * j4 + 0] = t4.x;
-            tv[4 * j4 + 1] = t4.y;
-            tv[4 * j4 + 2] = t4.z;
-            tv[4 * j4 + 3] = t4.w;
-          }
-#pragma unroll
-          for (int j = 0; j < 32; ++j) m = fmaxf(m, __uint_as_float(v[j]) - tv[j]);
-          if (m >= kap) {
-            uint32_t mask = 0;
-#pragma unroll
-            for (int j = 0; j < 32; ++j) mask |= (uint32_t)(__uint_as_float(v[j]) - tv[j] >= kap) << j;
-            const float* qrow = a.qpad + (size_t)row * a.dpad;
-            while (mask) {
-              const int j = __ffs(mask) - 1;
-              mask &= mask - 1;
-              const int key = key0 + ch * 32 + j;
-              const float d2 = dist2_canonical(qrow, a.keys + (size_t)key * a.dpad, a.dpad);
-              ++ncand;
-              if (d2 < __ldg(a.rr + key)) atomicMin(a.best + row, pack_hit(d2, key));
+            for (int j4 = 0; j4 < 8; ++j4) {
+              const uint4 tv = t4[j4];
+              const uint64_t d0 = ptx::sub_f32x2(ptx::pack_f32x2(v[4 * j4 + 0], v[4 * j4 + 1]), ptx::pack_f32x2(tv.x, tv.y));
+              const uint64_t d1 = ptx::sub_f32x2(ptx::pack_f32x2(v[4 * j4 + 2], v[4 * j4 + 3]), ptx::pack_f32x2(tv.z, tv.w));
+              m0 = ptx::max3_f32(m0, __uint_as_float((uint32_t)d0), __uint_as_float((uint32_t)(d0 >> 32)));
+              m1 = ptx::max3_f32(m1, __uint_as_float((uint32_t)d1), __uint_as_float((uint32_t)(d1 >> 32)));
             }
+            if (fmaxf(m0, m1) >= kap) {
+              uint32_t mask = 0;
+#pragma unroll
+              for (int j = 0; j < 32; ++j)
+                mask |= (uint32_t)(__uint_as_float(v[j]) - my_tau[ch * 32 + j] >= kap) << j;
+              const float* qrow = a.qpad + (size_t)row * a.dpad;
+              while (mask) {
+                const int j = __ffs(mask) - 1;
+                mask &= mask - 1;
+                const int key = key0 + ch * 32 + j;
+                const float d2 = dist2_canonical(qrow, a.keys + (size_t)key * a.dpad, a.dpad);
+                ++ncand;
+                if (d2 < __ldg(a.rr + key)) atomicMin(a.best + row, pack_hit(d2, key));
+              }
+            }
+            __syncwarp();
+            if (ch + 1 < kChunks) ptx::tmem_wait_ld();
           }
-          __syncwarp();
-          if (ch + 1 < kChunks) ptx::tmem_wait_ld();
         }
         ptx::tc_fence_before();
         __syncwarp();
         if (lane == 0) ptx::mbar_arrive(acc_empty + 8 * buf);
+        kap = kap_next;
       }
     }
     // candidate count: one atomic per warp
@@ -293,10 +381,16 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   ptx::tc_fence_before();
   __syncthreads();
-  if (threadIdx.x == 0 && *abort_s) {
-    atomicAdd(&a.stats->errors, 1ull);
-    atomicExch(&a.stats->abort_flag, 1);
+  if (*abort_s) {
+    // A role gave up: leave time for copies the peer may still be
+    // multicasting into this CTA before the cluster retires.
+    if (threadIdx.x == 0) {
+      atomicAdd(&a.stats->errors, 1ull);
+      atomicExch(&a.stats->abort_flag, 1);
+    }
+    __nanosleep(50000);
   }
+  ptx::cluster_sync();  // no remote arrival or copy can target an exited CTA
   if (warp == 1) {
     ptx::tc_fence_after();
     ptx::tmem_dealloc(tmem, (uint32_t)Layout<BN>::kTmemCols);
@@ -316,61 +410,31 @@ void encode_2d(lipcache* h, CUtensorMap* map, const float* base, uint64_t rows, 
 }
 
 template <int BN>
-void launch(lipcache* h, int64_t B, cudaStream_t s) {
+void launch(lipcache* h, int64_t B, const float* qpad, const float* kappa, unsigned long long* best, cudaStream_t s) {
   const int64_t Bpad = (B + kBM - 1) / kBM * kBM;
   CUtensorMap tmQ, tmK;
-  encode_2d(h, &tmQ, h->qpad, (uint64_t)Bpad, kBM);
+  encode_2d(h, &tmQ, qpad, (uint64_t)Bpad, kBM / 2);  // half a query tile per CTA of the pair
   encode_2d(h, &tmK, h->table.keys, (uint64_t)h->table_rows, BN);
   TcArgs a;
   a.nch = h->dpad / kChunkF;
+  a.nst = Layout<BN>::stages_for(a.nch);
+  LC_REQUIRE(a.nst >= 2, LIPCACHE_E_INVALID, "key tile does not fit shared memory");
   a.dpad = h->dpad;
   a.nq = (int)(Bpad / kBM);
   const int64_t n_kt = (h->size + BN - 1) / BN;
-  const int64_t target = 2LL * h->num_sms;
-  int n_qg = (int)((target + n_kt - 1) / n_kt);
+  const int64_t n_pairs = (n_kt + kCluster - 1) / kCluster;
+  const int max_clusters = h->num_sms / kCluster;
+  LC_REQUIRE(max_clusters >= 1, LIPCACHE_E_CUDA, "device has fewer than two SMs");
+  // enough units to keep every cluster busy when the cache is small
+  int n_qg = (int)((2LL * max_clusters + n_pairs - 1) / n_pairs);
   if (n_qg < 1) n_qg = 1;
   if (n_qg > a.nq) n_qg = a.nq;
   a.qpg = (a.nq + n_qg - 1) / n_qg;
   a.n_qg = (a.nq + a.qpg - 1) / a.qpg;
-  const int64_t n_units = n_kt * a.n_qg;
+  const int64_t n_units = n_pairs * a.n_qg;
   LC_REQUIRE(n_units < (1LL << 31), LIPCACHE_E_INVALID, "too many work units");
   a.n_units = (int)n_units;
-  a.kappa = h->kappa;
-  a.qpad = h->qpad;
-  a.keys = h->table.keys;
-  a.tau = h->table.tau;
-  a.rr = h->table.rr;
-  a.best = h->best;
-  a.stats = h->stats;
-  const Layout<BN> L{a.nch};
-  const int smem = L.total() + 1024;
-  LC_CUDA(cudaFuncSetAttribute(k_probe_tc<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
-  const int grid = (int)(n_units < h->num_sms ? n_units : h->num_sms);
-  k_probe_tc<BN><<<grid, kThreads, smem, s>>>(tmQ, tmK, a);
-  LC_LAUNCH_CHECK("k_probe_tc");
-}
-
-template <int BN>
-void launch_external(lipcache* h, int64_t B, const float* qpad, const float* kappa, unsigned long long* best,
-                     cudaStream_t s) {
-  const int64_t Bpad = (B + kBM - 1) / kBM * kBM;
-  CUtensorMap tmQ, tmK;
-  encode_2d(h, &tmQ, qpad, (uint64_t)Bpad, kBM);
-  encode_2d(h, &tmK, h->table.keys, (uint64_t)h->table_rows, BN);
-  TcArgs a;
-  a.nch = h->dpad / kChunkF;
-  a.dpad = h->dpad;
-  a.nq = (int)(Bpad / kBM);
-  const int64_t n_kt = (h->size + BN - 1) / BN;
-  const int64_t target = 2LL * h->num_sms;
-  int n_qg = (int)((target + n_kt - 1) / n_kt);
-  if (n_qg < 1) n_qg = 1;
-  if (n_qg > a.nq) n_qg = a.nq;
-  a.qpg = (a.nq + n_qg - 1) / n_qg;
-  a.n_qg = (a.nq + a.qpg - 1) / a.qpg;
-  const int64_t n_units = n_kt * a.n_qg;
-  LC_REQUIRE(n_units < (1LL << 31), LIPCACHE_E_INVALID, "too many work units");
-  a.n_units = (int)n_units;
+  a.n_kt = (int)n_kt;
   a.kappa = kappa;
   a.qpad = qpad;
   a.keys = h->table.keys;
@@ -378,33 +442,49 @@ void launch_external(lipcache* h, int64_t B, const float* qpad, const float* kap
   a.rr = h->table.rr;
   a.best = best;
   a.stats = h->stats;
-  const Layout<BN> L{a.nch};
+  const Layout<BN> L{a.nch, a.nst};
   const int smem = L.total() + 1024;
   LC_CUDA(cudaFuncSetAttribute(k_probe_tc<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
-  const int grid = (int)(n_units < h->num_sms ? n_units : h->num_sms);
-  k_probe_tc<BN><<<grid, kThreads, smem, s>>>(tmQ, tmK, a);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)(max_clusters * kCluster));
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = (size_t)smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = kCluster;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  // persistent grid: no more clusters than can be resident at once
+  int resident = 0;
+  LC_CUDA(cudaOccupancyMaxActiveClusters(&resident, k_probe_tc<BN>, &cfg));
+  LC_REQUIRE(resident >= 1, LIPCACHE_E_CUDA, "no CTA pair of the probe kernel fits on this device");
+  int clusters = max_clusters < resident ? max_clusters : resident;
+  if (n_units < clusters) clusters = (int)n_units;
+  cfg.gridDim = dim3((unsigned)(clusters * kCluster));
+  h->last_grid = clusters * kCluster;
+  h->last_cluster = kCluster;
+  LC_CUDA(cudaLaunchKernelEx(&cfg, k_probe_tc<BN>, tmQ, tmK, a));
   LC_LAUNCH_CHECK("k_probe_tc");
 }
 
 }  // namespace
 
+int tc_key_tile(int dpad) { return dpad <= 128 ? 256 : 128; }
+
 void launch_probe_tc_external(lipcache* h, int64_t B, const float* qpad, const float* kappa, unsigned long long* best,
                               cudaStream_t s) {
   LC_REQUIRE(tensor_path_supported(h->dpad), LIPCACHE_E_INVALID, "the tensor probe supports d <= 256");
   if (tc_key_tile(h->dpad) == 256)
-    launch_external<256>(h, B, qpad, kappa, best, s);
+    launch<256>(h, B, qpad, kappa, best, s);
   else
-    launch_external<128>(h, B, qpad, kappa, best, s);
+    launch<128>(h, B, qpad, kappa, best, s);
 }
 
-int tc_key_tile(int dpad) { return dpad <= 128 ? 256 : 128; }
-
 void launch_probe_tc(lipcache* h, int64_t B, cudaStream_t s) {
-  LC_REQUIRE(tensor_path_supported(h->dpad), LIPCACHE_E_INVALID, "the tensor probe supports d <= 256");
-  if (tc_key_tile(h->dpad) == 256)
-    launch<256>(h, B, s);
-  else
-    launch<128>(h, B, s);
+  launch_probe_tc_external(h, B, h->qpad, h->kappa, h->best, s);
 }
 
 }  // namespace lc
