@@ -185,6 +185,28 @@ def roofline(w: synth.Workload, N: int, B: int, kernel_ms: float, pk: dict, pk_k
             "peak_source": f"{pk_kind} copy bandwidth", "kernel": "k_probe_tc", "kernel_ms": kernel_ms}
 
 
+def recorded_traffic(workload: str):
+    """DRAM bytes per probe launch recorded in profiles/k_probe_tc_scale.md
+    from an ncu capture, or None when the kernel sources changed since."""
+    import hashlib
+    path = os.path.join(ROOT, "profiles", "k_probe_tc_scale.md")
+    if not os.path.exists(path):
+        return None
+    rec = {}
+    for line in open(path):
+        line = line.strip()
+        for key in ("traffic_bytes_per_launch", "traffic_workload", "sources_sha256_16"):
+            if line.startswith(key + ":"):
+                rec[key] = line.split(":", 1)[1].strip()
+    h = hashlib.sha256()
+    for f in ("probe_tc.cu", "tc_ptx.cuh", "probe_common.cuh"):
+        with open(os.path.join(ROOT, "paper_2608_13144_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    if rec.get("sources_sha256_16") != h.hexdigest()[:16] or rec.get("traffic_workload") != workload:
+        return None
+    return float(rec["traffic_bytes_per_launch"])
+
+
 def cpu_baseline(w, W, b, rows, Q, budget_s: float) -> dict:
     """The FP64 oracle as it stands, on the host cores, on a bounded sample:
     the first n queries against the whole cache (n sized to the budget)."""
@@ -299,6 +321,8 @@ def run_ours(args, dist: Dist):
     cache.close()
 
     rf = roofline(w, N, B, kernel_ms, pk, pk_kind)
+    if info["last_probe_path"] == 1 and w.N == synth.WORKLOADS[w.name].N:
+        rf["traffic"] = recorded_traffic(w.name)
     line = {
         "metric": METRIC, "value": value, "unit": "queries/s", "n_gpus": dist.world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": tmax / args.steps * 1e3, "higher_is_better": True,

@@ -1,0 +1,55 @@
+"""The N > 1 path of bench.py on CPU: each rank is an independent replica;
+a gloo process group carries only the barrier and the timing reduction
+(queries of all ranks over the slowest rank's time)."""
+import os
+import socket
+
+import pytest
+
+torch = pytest.importorskip("torch")
+import torch.multiprocessing as mp  # noqa: E402
+
+
+def _free_port():
+    s = socket.socket()
+    s.bind(("127.0.0.1", 0))
+    p = s.getsockname()[1]
+    s.close()
+    return p
+
+
+def _worker(rank, world, port, out):
+    os.environ.update({"RANK": str(rank), "LOCAL_RANK": str(rank), "WORLD_SIZE": str(world),
+                       "MASTER_ADDR": "127.0.0.1", "MASTER_PORT": str(port)})
+    import bench
+    d = bench.Dist()
+    d.barrier()
+    # rank r processed (r + 1) * 1000 queries in (r + 1) seconds
+    value, tmax = bench.aggregate(d, (rank + 1) * 1000.0, rank + 1.0)
+    out[rank] = (value, tmax)
+    d.close()
+
+
+def test_replica_aggregation_two_ranks():
+    world = 2
+    port = _free_port()
+    ctx = mp.get_context("spawn")
+    out = ctx.Manager().dict()
+    procs = [ctx.Process(target=_worker, args=(r, world, port, out)) for r in range(world)]
+    for p in procs:
+        p.start()
+    for p in procs:
+        p.join(120)
+        assert p.exitcode == 0
+    for r in range(world):
+        value, tmax = out[r]
+        assert tmax == 2.0                  # max over ranks
+        assert value == pytest.approx(1500.0)  # (1000 + 2000) queries / 2 s
+
+
+def test_single_rank_aggregation_is_identity():
+    import bench
+    d = bench.Dist()
+    assert d.world == int(os.environ.get("WORLD_SIZE", "1"))
+    if d.world == 1:
+        assert bench.aggregate(d, 500.0, 2.0) == (250.0, 2.0)
