@@ -58,7 +58,9 @@ void release(lipcache* h) {
   dev_free(h->W);
   dev_free(h->b);
   dev_free(h->Wnorm);
+  dev_free(h->Wnorm32);
   dev_free(h->pairnorm);
+  dev_free(h->inv_pairnorm);
   dev_free(h->gram[0]);
   dev_free(h->gram[1]);
   dev_free(h->spec);
@@ -158,7 +160,11 @@ LC_API lipcache_status lipcache_create(int32_t d, int32_t C, int64_t capacity, i
     dev_alloc(h->W, (size_t)C * d);
     dev_alloc(h->b, (size_t)C);
     dev_alloc(h->Wnorm, (size_t)C);
-    if (radius_mode == LIPCACHE_RADIUS_TIGHT) dev_alloc(h->pairnorm, (size_t)C * C);
+    dev_alloc(h->Wnorm32, (size_t)C);
+    if (radius_mode == LIPCACHE_RADIUS_TIGHT) {
+      dev_alloc(h->pairnorm, (size_t)C * C);
+      dev_alloc(h->inv_pairnorm, (size_t)C * C);
+    }
     dev_alloc(h->gram[0], (size_t)d * d);
     dev_alloc(h->gram[1], (size_t)d * d);
     dev_alloc(h->spec, 1);

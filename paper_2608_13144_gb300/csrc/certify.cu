@@ -12,16 +12,24 @@
 // a decision boundary, where m is a small difference of large logits. The
 // kernel therefore computes all logits in FP32 with a proven error bound
 // E_c = gamma_{d+2} (||W_c|| ||z|| + |b_c|), keeps every class whose FP32
-// interval can reach the true top two, and recomputes those classes in FP64
-// (products of FP32 values are exact in FP64). The true top-1 and runner-up
-// are always among them, so m equals the FP64 margin of the full logit
-// vector. The tight radius needs every class and refines all of them.
+// interval can reach the true top two, and recomputes those classes with a
+// compensated FP32 dot product (Dot2, Ogita, Rump and Oishi 2005) kept as an
+// unevaluated pair hi + lo, accurate to 2 gamma_{d+40}^2 (||W_c|| ||z|| +
+// |b_c|). The true top-1 and runner-up are always among them, so m is the
+// margin of the full logit vector to ~1e-10 relative of the logit scale.
+// FP64 runs at a small fraction of the FP32 rate on this GPU, so only the
+// per-row margin and radius use it. The tight radius needs every class and
+// refines all of them in FP64 (products of FP32 values are exact there).
 //
 // Besides the reported radius r, the kernel derives a certified lower bound
-// r_safe (FP64 error bounds of the two logits, sigma inflated by 1e-9) and
-// from it the probe's acceptance threshold rr = RZ(r_safe^2 (1 - eps_rc)) on
-// the canonical FP32 squared distance, and the screen term tau.
+// r_safe of the exact radius (the refined logits' error bounds, sigma
+// inflated by 1e-9, every step rounded downwards) and from it the probe's
+// acceptance threshold rr <= r_safe^2 (1 - eps_rc) on the canonical FP32
+// squared distance, and the screen term tau.
 //
+// Two kernels compute the FP32 logits: when C <= 256 and the head fits in
+// shared memory, persistent CTAs keep W^T resident and form a register-tiled
+// product (k_certify_wres); otherwise each CTA streams W from L2 (k_certify).
 // Insertion order is kept by a block-count scan and a scatter.
 #include "internal.cuh"
 
@@ -43,6 +51,16 @@ struct CertArgs {
   const double* pairnorm;
   const int32_t* payload;
   double sigma, kappa, eps_rc, gamma_rc, c_scr, g32, g64;
+  const float* Wnorm32;  // ||W_c|| rounded up
+  float g32f;            // gamma_{d+2} with FP32 rounding slack
+  float g2f;             // error factor of the compensated dot product
+  double inv_denom;      // kappa / (sigma sqrt 2)
+  double inv_denom_safe; // kappa (1 - 8u) / (sigma (1 + slack) sqrt 2)
+  float om_eps_rd;       // 1 - eps_rc, rounded down
+  float inv_omg_ru;      // 1 / (1 - gamma_rc), rounded up
+  float om_c_rd;         // 1 - c_screen, rounded down
+  const double* inv_pairnorm;  // 1 / ||W_y - W_j|| (tight mode)
+  double tight_f;              // 1 - gamma_{d+8} (FP64)
   uint8_t* accept;
   int32_t* yG;
   int32_t* label;
@@ -84,55 +102,226 @@ __device__ __forceinline__ void top2_push(double& t1, double& t2, double v) {
   }
 }
 
-__global__ void __launch_bounds__(kThreads) k_certify(CertArgs a) {
-  extern __shared__ __align__(16) unsigned char smem[];
-  double* s64 = reinterpret_cast<double*>(smem);        // kWarps x C refined logits
-  double* e64 = s64 + (size_t)kWarps * a.C;             // kWarps x C their error bounds
-  float* hs = reinterpret_cast<float*>(e64 + (size_t)kWarps * a.C);  // kRows x hstride
-  float* lg = hs + (size_t)kRows * a.hstride;           // kRows x lstride FP32 logits
-  __shared__ uint8_t acc_flag[kRows];
+// FP32 error-free transformations: a + b = s + e and a * b = p + e exactly
+// (Knuth's TwoSum; TwoProduct with a fused multiply-add).
+__device__ __forceinline__ void two_sum(float a, float b, float& s, float& e) {
+  s = __fadd_rn(a, b);
+  const float bb = __fsub_rn(s, a);
+  e = __fadd_rn(__fsub_rn(a, __fsub_rn(s, bb)), __fsub_rn(b, bb));
+}
 
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int64_t row0 = (int64_t)blockIdx.x * kRows;
-  const int nrows = (int)(a.n - row0 < kRows ? a.n - row0 : kRows);
-  const int d = a.d, C = a.C;
-
-  for (int idx = threadIdx.x; idx < kRows * d; idx += kThreads) {
-    const int r = idx / d, j = idx - r * d;
-    hs[r * a.hstride + j] = (r < nrows) ? a.H[(size_t)(row0 + r) * d + j] : 0.f;
+// Compensated dot product W_c . h + b_c (Ogita, Rump and Oishi's Dot2, summed
+// across the warp with the same transformations), returned as a normalised
+// pair hi + lo (|lo| <= ulp(hi)/2) whose exact sum is within
+// 2 gamma_{d+40}^2 (sum_j |W_cj h_j| + |b_c|) of the exact value. Every lane
+// gets the same bits: each butterfly step combines the two partners' pairs
+// symmetrically. wc[j * ws] and hrow[j * hs] address feature j of the
+// weights and of the row (global memory, or the transposed shared tiles).
+__device__ __forceinline__ void dot2_logit(const float* __restrict__ wc, int ws, const float* __restrict__ hrow, int hs,
+                                           float bias, int d, int lane, float& hi, float& lo) {
+  float p = 0.f, c = 0.f;
+  for (int j = lane; j < d; j += 32) {
+    const float w = wc[(size_t)j * ws], x = hrow[(size_t)j * hs];
+    const float pr = __fmul_rn(w, x);
+    const float er = __fmaf_rn(w, x, -pr);
+    float t, q;
+    two_sum(p, pr, t, q);
+    p = t;
+    c = __fadd_rn(c, __fadd_rn(q, er));
   }
-  if (threadIdx.x < kRows) acc_flag[threadIdx.x] = 0;
-  __syncthreads();
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float pb = __shfl_xor_sync(kFull, p, o), cb = __shfl_xor_sync(kFull, c, o);
+    float t, q;
+    two_sum(p, pb, t, q);
+    p = t;
+    c = __fadd_rn(__fadd_rn(c, cb), q);
+  }
+  float t, q;
+  two_sum(p, bias, t, q);
+  two_sum(t, __fadd_rn(c, q), hi, lo);
+}
 
-  // FP32 logits: lane = row, warps stride over classes (W loads are warp-uniform).
-  {
-    const float* hrow = hs + lane * a.hstride;
-    for (int c = warp; c < C; c += kWarps) {
-      const float* wc = a.W + (size_t)c * d;
-      float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
-      int j = 0;
-      for (; j + 4 <= d; j += 4) {
-        s0 = fmaf(__ldg(wc + j), hrow[j], s0);
-        s1 = fmaf(__ldg(wc + j + 1), hrow[j + 1], s1);
-        s2 = fmaf(__ldg(wc + j + 2), hrow[j + 2], s2);
-        s3 = fmaf(__ldg(wc + j + 3), hrow[j + 3], s3);
+// Absolute error allowance for subnormal intermediate results: at most
+// 2^-150 per rounding, (d + 40) * 2^-150 < 1e-39 in all for d <= 1024.
+constexpr float kTinyF = 1e-35f;
+
+// Rounded-up bound E_c of |s~_c - s_c| for an FP32 logit s~_c:
+// gamma_{d+2} (||W_c|| ||z|| + |b_c|) (g32f carries the slack for its own
+// rounding), 2^-22 |s~_c| for the rounding of the interval ends, and kTinyF.
+__device__ __forceinline__ float logit_err(float g32f, float wn, float hn, float b, float sv) {
+  return __fmaf_ru(g32f, __fmaf_ru(wn, hn, fabsf(b)), __fmaf_ru(fabsf(sv), 2.3841858e-07f /* 2^-22 */, kTinyF));
+}
+
+// (ah, al) > (bh, bl) for pairs normalised by a final TwoSum (hi = RN(hi + lo)):
+// round-to-nearest is monotone, so this orders the exact sums.
+__device__ __forceinline__ bool pair_gt(float ah, float al, float bh, float bl) {
+  return ah > bh || (ah == bh && al > bl);
+}
+
+// Certify the rows r = warp, warp + nwarps, ... < nrows of a tile with one
+// warp, conservative radius (Eq. 21). The FP32 intervals s~_c +- E_c
+// (E_c = gamma_{d+2} (||W_c|| ||z|| + |b_c|), widened for the rounding of the
+// interval arithmetic itself) select every class that can be among the true
+// top two; those are recomputed with dot2_logit. The true runner-up is among
+// them, so the margin is that of the full logit vector. All per-class work is
+// FP32; the few FP64 operations per row (margin and radius) run once for up
+// to 32 rows, one lane per row (FP64 runs at a small fraction of the FP32
+// rate on this GPU).
+// Row r: features hb[r * hrs + j * hs], logits lg[r * lstride + c];
+// W_cj = wmat[c * wcs + j * wjs]; norms / bias per class in wn32 / bias.
+__device__ void certify_rows_fast(const CertArgs& a, int64_t row0, int nrows, int warp, int nwarps,
+                                  const float* __restrict__ hb, int hrs, int hs, const float* __restrict__ wmat,
+                                  int wcs, int wjs, const float* __restrict__ lg, const float* __restrict__ wn32,
+                                  const float* __restrict__ bias, int lane, uint8_t* acc_flag) {
+  const int d = a.d, C = a.C;
+  // per-row results parked in lane k (the warp's k-th row)
+  float r_h1 = 0.f, r_l1 = 0.f, r_e1 = 0.f, r_h2 = 0.f, r_l2 = 0.f, r_up = 0.f, r_kn = 0.f;
+  int r_y = 0, k = 0;
+  for (int r = warp; r < nrows; r += nwarps, ++k) {
+    const float* hrow = hb + (size_t)r * hrs;
+    const float* lrow = lg + (size_t)r * a.lstride;
+    float knp = 0.f;
+    for (int j = lane; j < d; j += 32) {
+      const float x = hrow[(size_t)j * hs];
+      knp = fmaf(x, x, knp);
+    }
+    const float kn = warp_sum_f(knp);
+    // upper bound of ||z||: kn is within gamma_{d/32+5} < 1e-5 of ||z||^2, up
+    // to d * 2^-150 lost where the squares are subnormal
+    const float hn = __fmul_ru(__fsqrt_ru(__fmaf_ru(kn, 1.0f + 1e-5f, kTinyF)), 1.0f + 1e-6f);
+
+    float l1 = -INFINITY, l2 = -INFINITY;
+    for (int c = lane; c < C; c += 32) {
+      const float sv = lrow[c];
+      const float E = logit_err(a.g32f, wn32[c], hn, bias[c], sv);
+      const float lo = __fsub_rd(sv, E);
+      if (lo > l1) {
+        l2 = l1;
+        l1 = lo;
+      } else if (lo > l2) {
+        l2 = lo;
       }
-      for (; j < d; ++j) s0 = fmaf(__ldg(wc + j), hrow[j], s0);
-      lg[lane * a.lstride + c] = ((s0 + s1) + (s2 + s3)) + __ldg(a.b + c);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const float o1 = __shfl_xor_sync(kFull, l1, o), o2 = __shfl_xor_sync(kFull, l2, o);
+      float t1 = l1, t2 = l2;
+      if (o1 > t1) {
+        t2 = t1;
+        t1 = o1;
+      } else if (o1 > t2) {
+        t2 = o1;
+      }
+      if (o2 > t1) {
+        t2 = t1;
+        t1 = o2;
+      } else if (o2 > t2) {
+        t2 = o2;
+      }
+      l1 = t1;
+      l2 = t2;
+    }
+    const float L2 = l2;
+
+    // refine the candidates in ascending class order (strict comparisons keep
+    // the lowest class on ties)
+    float b1h = -INFINITY, b1l = 0.f, b2h = -INFINITY, b2l = 0.f, e1 = 0.f;
+    float u1 = -INFINITY, u2 = -INFINITY;  // top two upper bounds v + e ...
+    int y = -1, cu1 = -1;                  // ... and the class of the first
+    for (int cb = 0; cb < C; cb += 32) {
+      const int c = cb + lane;
+      bool cand = false;
+      if (c < C) {
+        const float sv = lrow[c];
+        const float E = logit_err(a.g32f, wn32[c], hn, bias[c], sv);
+        cand = (__fadd_ru(sv, E) >= L2) || !(L2 == L2);
+      }
+      unsigned m = __ballot_sync(kFull, cand);
+      while (m) {
+        const int cc = cb + __ffs(m) - 1;
+        m &= m - 1;
+        const float bc = bias[cc];
+        float vh, vl;
+        dot2_logit(wmat + (size_t)cc * wcs, wjs, hrow, hs, bc, d, lane, vh, vl);
+        // bound of |hi + lo - exact|, rounded up (plus the absolute error of
+        // subnormal products)
+        const float e = __fmaf_ru(a.g2f, __fmaf_ru(wn32[cc], hn, fabsf(bc)), kTinyF);
+        if (pair_gt(vh, vl, b1h, b1l)) {
+          b2h = b1h;
+          b2l = b1l;
+          b1h = vh;
+          b1l = vl;
+          e1 = e;
+          y = cc;
+        } else if (pair_gt(vh, vl, b2h, b2l)) {
+          b2h = vh;
+          b2l = vl;
+        }
+        const float up = __fadd_ru(vh, __fadd_ru(vl, e));
+        if (up > u1) {
+          u2 = u1;
+          u1 = up;
+          cu1 = cc;
+        } else if (up > u2) {
+          u2 = up;
+        }
+      }
+    }
+    if (lane == k) {
+      r_h1 = b1h;
+      r_l1 = b1l;
+      r_e1 = e1;
+      r_h2 = b2h;
+      r_l2 = b2l;
+      r_up = (cu1 == y) ? u2 : u1;
+      r_y = y < 0 ? 0 : y;  // every refined logit NaN: the margin is NaN and the row is rejected
+      r_kn = kn;
     }
   }
-  __syncthreads();
-
-  double* ws = s64 + (size_t)warp * C;
-  double* we = e64 + (size_t)warp * C;
-  for (int r = warp; r < nrows; r += kWarps) {
+  // FP64 margin and radius, one lane per row
+  if (lane < k) {
+    const int r = warp + lane * nwarps;
     const int64_t row = row0 + r;
-    const float* hrow = hs + r * a.hstride;
-    const float* lrow = lg + r * a.lstride;
+    const double v1 = (double)r_h1 + (double)r_l1, v2 = (double)r_h2 + (double)r_l2;
+    const double mval = (v1 == v1 && v2 == v2) ? v1 - v2 : NAN;
+    // lower bound of the exact margin with downward rounding
+    const double mlo = __dsub_rd(__dsub_rd(v1, (double)r_e1), (double)r_up);
+    const double r64 = mval * a.inv_denom;
+    const double rs = (mlo > 0.0) ? __dmul_rd(mlo, a.inv_denom_safe) : 0.0;
+    const int32_t lab = a.payload ? a.payload[row] : r_y;
+    const bool acc = !(a.require_consistency && lab != r_y) && (r64 > 0.0);
+    // probe thresholds in FP32 with directed rounding (each step only lowers
+    // rr and tau): rr <= r_safe^2 (1 - eps_rc), tau as in probe_tc.cu
+    const float rs32 = __double2float_rd(rs);
+    const float rr = __fmul_rd(__fmul_rd(rs32, rs32), a.om_eps_rd);
+    const float Rt = __fmul_ru(rr, a.inv_omg_ru);
+    const float tau = __fmul_rd(__fsub_rd(__fmul_rd(a.om_c_rd, r_kn), Rt), 0.5f);
+    a.accept[row] = acc ? 1 : 0;
+    a.yG[row] = r_y;
+    a.label[row] = lab;
+    a.radius[row] = __double2float_rz(r64);
+    a.rr[row] = rr;
+    a.kn[row] = r_kn;
+    a.tau[row] = tau;
+    acc_flag[r] = acc ? 1 : 0;
+  }
+  __syncwarp();
+}
+
+// Certify one row with one warp: FP32 interval of every logit, FP64
+// refinement of the classes that can be among the true top two (all classes
+// for the tight radius), margin, radius, certified lower bound, thresholds
+// for the probe, and the skip rules of Algorithm 1. hrow: the row's d
+// features in global memory; lrow: its FP32 logits (shared memory); ws / we:
+// this warp's C-entry scratch for refined logits and their error bounds.
+__device__ void certify_row(const CertArgs& a, int64_t row, const float* __restrict__ hrow,
+                            const float* __restrict__ lrow, double* ws, double* we, int lane, uint8_t* acc_slot) {
+  const int d = a.d, C = a.C;
     float knp = 0.f;
     double hnp = 0.0;
     for (int j = lane; j < d; j += 32) {
-      const float x = hrow[j];
+      const float x = __ldg(hrow + j);
       knp = fmaf(x, x, knp);
       hnp = fma((double)x, (double)x, hnp);
     }
@@ -179,7 +368,7 @@ __global__ void __launch_bounds__(kThreads) k_certify(CertArgs a) {
         const float* wc = a.W + (size_t)cc * d;
         double p = 0.0, pa = 0.0;
         for (int j = lane; j < d; j += 32) {
-          const double t = (double)__ldg(wc + j) * (double)hrow[j];
+          const double t = (double)__ldg(wc + j) * (double)__ldg(hrow + j);
           p += t;
           pa += fabs(t);
         }
@@ -210,12 +399,12 @@ __global__ void __launch_bounds__(kThreads) k_certify(CertArgs a) {
     if (!a.tight) {
       double up_other = -INFINITY;
       for (int c = lane; c < C; c += 32)
-        if (c != y) up_other = fmax(up_other, ws[c] + we[c]);
+        if (c != y) up_other = fmax(up_other, __dadd_ru(ws[c], we[c]));
       up_other = warp_max_d(up_other);
       const double mval = (b1 == b1 && b2 == b2) ? b1 - b2 : NAN;
-      const double mlo = (sy - ey) - up_other;
-      r64 = a.kappa * mval / (a.sigma * sqrt2);
-      rs = (mlo > 0.0) ? a.kappa * mlo * (1.0 - 8 * kU64) / (a.sigma * (1.0 + kSigmaSlack) * sqrt2) : 0.0;
+      const double mlo = __dsub_rd(__dsub_rd(sy, ey), up_other);
+      r64 = mval * a.inv_denom;
+      rs = (mlo > 0.0) ? __dmul_rd(mlo, a.inv_denom_safe) : 0.0;
       if (!(mval == mval)) r64 = NAN;
     } else {
       double rmin = INFINITY, smin = INFINITY;
@@ -225,23 +414,26 @@ __global__ void __launch_bounds__(kThreads) k_certify(CertArgs a) {
         const double pn = a.pairnorm[(size_t)y * C + j];
         if (!(ws[j] == ws[j])) any_nan = true;
         if (!(pn > 0.0)) continue;
-        rmin = fmin(rmin, (sy - ws[j]) / pn);
-        smin = fmin(smin, ((sy - ey) - (ws[j] + we[j])) / (pn * (1.0 + 1e-14)));
+        const double ipn = a.inv_pairnorm[(size_t)y * C + j];
+        rmin = fmin(rmin, (sy - ws[j]) * ipn);
+        // ipn is within gamma_{d+4} / 2 of 1 / ||W_y - W_j||; tight_f removes that
+        const double num = __dsub_rd(__dsub_rd(sy, ey), __dadd_ru(ws[j], we[j]));
+        smin = fmin(smin, __dmul_rd(__dmul_rd(num, ipn), a.tight_f));
       }
       rmin = warp_min_d(rmin);
       smin = warp_min_d(smin);
       any_nan = __any_sync(kFull, any_nan);
       r64 = any_nan ? NAN : a.kappa * rmin;
-      rs = (smin > 0.0 && !any_nan) ? a.kappa * smin * (1.0 - 8 * kU64) : 0.0;
+      rs = (smin > 0.0 && !any_nan) ? __dmul_rd(a.kappa, smin) : 0.0;
     }
 
     if (lane == 0) {
       const int32_t lab = a.payload ? a.payload[row] : y;
       const bool acc = !(a.require_consistency && lab != y) && (r64 > 0.0);
-      const double rr64 = rs * rs * (1.0 - a.eps_rc);
-      const float rr = __double2float_rz(rr64);
-      const double Rt = (double)rr / (1.0 - a.gamma_rc) * (1.0 + 1e-15);
-      const float tau = __double2float_rd(((1.0 - a.c_scr) * (double)kn - Rt) * 0.5);
+      const float rs32 = __double2float_rd(rs);
+      const float rr = __fmul_rd(__fmul_rd(rs32, rs32), a.om_eps_rd);
+      const float Rt = __fmul_ru(rr, a.inv_omg_ru);
+      const float tau = __fmul_rd(__fsub_rd(__fmul_rd(a.om_c_rd, kn), Rt), 0.5f);
       a.accept[row] = acc ? 1 : 0;
       a.yG[row] = y;
       a.label[row] = lab;
@@ -249,9 +441,58 @@ __global__ void __launch_bounds__(kThreads) k_certify(CertArgs a) {
       a.rr[row] = rr;
       a.kn[row] = kn;
       a.tau[row] = tau;
-      acc_flag[r] = acc ? 1 : 0;
+      *acc_slot = acc ? 1 : 0;
     }
     __syncwarp();
+}
+
+__global__ void __launch_bounds__(kThreads) k_certify(CertArgs a) {
+  extern __shared__ __align__(16) unsigned char smem[];
+  double* s64 = reinterpret_cast<double*>(smem);        // kWarps x C refined logits
+  double* e64 = s64 + (size_t)kWarps * a.C;             // kWarps x C their error bounds
+  float* hs = reinterpret_cast<float*>(e64 + (size_t)kWarps * a.C);  // kRows x hstride
+  float* lg = hs + (size_t)kRows * a.hstride;           // kRows x lstride FP32 logits
+  __shared__ uint8_t acc_flag[kRows];
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int64_t row0 = (int64_t)blockIdx.x * kRows;
+  const int nrows = (int)(a.n - row0 < kRows ? a.n - row0 : kRows);
+  const int d = a.d, C = a.C;
+
+  for (int idx = threadIdx.x; idx < kRows * d; idx += kThreads) {
+    const int r = idx / d, j = idx - r * d;
+    hs[r * a.hstride + j] = (r < nrows) ? a.H[(size_t)(row0 + r) * d + j] : 0.f;
+  }
+  if (threadIdx.x < kRows) acc_flag[threadIdx.x] = 0;
+  __syncthreads();
+
+  // FP32 logits: lane = row, warps stride over classes (W loads are warp-uniform).
+  {
+    const float* hrow = hs + lane * a.hstride;
+    for (int c = warp; c < C; c += kWarps) {
+      const float* wc = a.W + (size_t)c * d;
+      float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+      int j = 0;
+      for (; j + 4 <= d; j += 4) {
+        s0 = fmaf(__ldg(wc + j), hrow[j], s0);
+        s1 = fmaf(__ldg(wc + j + 1), hrow[j + 1], s1);
+        s2 = fmaf(__ldg(wc + j + 2), hrow[j + 2], s2);
+        s3 = fmaf(__ldg(wc + j + 3), hrow[j + 3], s3);
+      }
+      for (; j < d; ++j) s0 = fmaf(__ldg(wc + j), hrow[j], s0);
+      lg[lane * a.lstride + c] = ((s0 + s1) + (s2 + s3)) + __ldg(a.b + c);
+    }
+  }
+  __syncthreads();
+
+  double* ws = s64 + (size_t)warp * C;
+  double* we = e64 + (size_t)warp * C;
+  if (a.tight) {
+    for (int r = warp; r < nrows; r += kWarps)
+      certify_row(a, row0 + r, a.H + (size_t)(row0 + r) * d, lg + r * a.lstride, ws, we, lane, &acc_flag[r]);
+  } else {
+    certify_rows_fast(a, row0, nrows, warp, kWarps, a.H + (size_t)row0 * d, d, 1, a.W, d, 1, lg, a.Wnorm32, a.b,
+                      lane, acc_flag);
   }
   __syncthreads();
   if (warp == 0) {
@@ -259,6 +500,117 @@ __global__ void __launch_bounds__(kThreads) k_certify(CertArgs a) {
     const unsigned m = __ballot_sync(kFull, f);
     if (lane < nrows) a.rank[row0 + lane] = __popc(m & ((1u << lane) - 1u));
     if (lane == 0) a.bcount[blockIdx.x] = __popc(m);
+  }
+}
+
+// Certified insertion with the head resident in shared memory (C <= 256 and
+// W^T fits): persistent CTAs, tiles of 64 rows. The FP32 logits are a
+// register-tiled product: each thread accumulates 8 rows x 8 classes, reading
+// 8 features and 8 weights per k with four 128-bit shared loads, one FMA
+// chain per (row, class) in k order (the same error bound as above).
+constexpr int kWTile = 64;   // rows per tile
+constexpr int kHStride = 68; // h^T row stride (floats): 16-byte aligned, banks spread
+
+__global__ void __launch_bounds__(kThreads, 1) k_certify_wres(CertArgs a, int Cp, int dpad, int n_tiles) {
+  extern __shared__ __align__(16) unsigned char smem[];
+  float* wT = reinterpret_cast<float*>(smem);           // dpad x Cp (W transposed, zero padded)
+  float* hT = wT + (size_t)dpad * Cp;                   // dpad x kHStride (tile rows transposed)
+  float* lg = hT + (size_t)dpad * kHStride;             // kWTile x lstride FP32 logits
+  // FP64 scratch for the tight radius only
+  const int sC = a.tight ? a.C : 0;
+  double* s64 = reinterpret_cast<double*>(lg + (size_t)kWTile * a.lstride + ((kWTile * a.lstride) & 1));
+  double* e64 = s64 + (size_t)kWarps * sC;
+  float* wn_s = reinterpret_cast<float*>(e64 + (size_t)kWarps * sC);  // C norms (rounded up)
+  float* b_s = wn_s + a.C;                                              // C biases
+  __shared__ uint8_t acc_flag[kWTile];
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int d = a.d, C = a.C;
+  for (int idx = tid; idx < dpad * Cp; idx += kThreads) {
+    const int k = idx / Cp, c = idx - k * Cp;
+    wT[idx] = (c < C && k < d) ? __ldg(a.W + (size_t)c * d + k) : 0.f;
+  }
+  for (int c = tid; c < C; c += kThreads) {
+    wn_s[c] = __ldg(a.Wnorm32 + c);
+    b_s[c] = __ldg(a.b + c);
+  }
+  const int rg = tid & 7, cg = tid >> 3;  // rows {4rg..4rg+3, 32+4rg..32+4rg+3}, classes 8cg..8cg+7
+  const bool mine = cg * 8 < Cp;
+  double* ws = s64 + (size_t)warp * sC;
+  double* we = e64 + (size_t)warp * sC;
+
+  for (int tile = blockIdx.x; tile < n_tiles; tile += gridDim.x) {
+    const int64_t row0 = (int64_t)tile * kWTile;
+    const int nrows = (int)(a.n - row0 < kWTile ? a.n - row0 : kWTile);
+    // the tile's features: all loads of a thread issued before its stores
+    constexpr int kBatch = 16;
+    float buf[kBatch];
+    for (int base = 0; base < kWTile * dpad; base += kThreads * kBatch) {
+#pragma unroll
+      for (int i = 0; i < kBatch; ++i) {
+        const int idx = base + i * kThreads + tid;
+        const int r = idx / dpad, k = idx - r * dpad;
+        buf[i] = (idx < kWTile * dpad && r < nrows && k < d) ? __ldg(a.H + (size_t)(row0 + r) * d + k) : 0.f;
+      }
+      if (base == 0) __syncthreads();  // previous tile done with hT / lg (and wT written on the first pass)
+#pragma unroll
+      for (int i = 0; i < kBatch; ++i) {
+        const int idx = base + i * kThreads + tid;
+        if (idx < kWTile * dpad) {
+          const int r = idx / dpad, k = idx - r * dpad;
+          hT[k * kHStride + r] = buf[i];
+        }
+      }
+    }
+    if (tid < kWTile) acc_flag[tid] = 0;
+    __syncthreads();
+    if (mine) {
+      float acc[8][8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i)
+#pragma unroll
+        for (int j = 0; j < 8; ++j) acc[i][j] = 0.f;
+      const float* hp = hT + rg * 4;
+      const float* wp = wT + cg * 8;
+#pragma unroll 4
+      for (int k = 0; k < dpad; ++k) {
+        const float4 h0 = *reinterpret_cast<const float4*>(hp + k * kHStride);
+        const float4 h1 = *reinterpret_cast<const float4*>(hp + k * kHStride + 32);
+        const float4 w0 = *reinterpret_cast<const float4*>(wp + (size_t)k * Cp);
+        const float4 w1 = *reinterpret_cast<const float4*>(wp + (size_t)k * Cp + 4);
+        const float hv[8] = {h0.x, h0.y, h0.z, h0.w, h1.x, h1.y, h1.z, h1.w};
+        const float wv[8] = {w0.x, w0.y, w0.z, w0.w, w1.x, w1.y, w1.z, w1.w};
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+#pragma unroll
+          for (int j = 0; j < 8; ++j) acc[i][j] = fmaf(wv[j], hv[i], acc[i][j]);
+      }
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const int r = (i < 4) ? rg * 4 + i : 32 + rg * 4 + (i - 4);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          const int c = cg * 8 + j;
+          if (c < C) lg[r * a.lstride + c] = acc[i][j] + __ldg(a.b + c);
+        }
+      }
+    }
+    __syncthreads();
+    if (a.tight) {
+      for (int r = warp; r < nrows; r += kWarps)
+        certify_row(a, row0 + r, a.H + (size_t)(row0 + r) * d, lg + r * a.lstride, ws, we, lane, &acc_flag[r]);
+    } else {
+      certify_rows_fast(a, row0, nrows, warp, kWarps, hT, 1, kHStride, wT, 1, Cp, lg, wn_s, b_s, lane, acc_flag);
+    }
+    __syncthreads();
+    if (warp < 2 && row0 + warp * 32 < a.n) {
+      const int sub = warp * 32;
+      const int nsub = nrows - sub < 32 ? nrows - sub : 32;
+      const bool f = lane < nsub && acc_flag[sub + lane];
+      const unsigned m = __ballot_sync(kFull, f);
+      if (lane < nsub) a.rank[row0 + sub + lane] = __popc(m & ((1u << lane) - 1u));
+      if (lane == 0) a.bcount[(row0 + sub) / 32] = __popc(m);
+    }
   }
 }
 
@@ -390,6 +742,19 @@ void certify_insert(lipcache* h, const float* H, int64_t n, const int32_t* paylo
   a.c_scr = h->c_scr;
   a.g32 = gamma32(h->d + 2) * (1.0 + 1e-6);
   a.g64 = gamma64(h->d + 8) * (1.0 + 1e-6);
+  a.Wnorm32 = h->Wnorm32;
+  a.g32f = (float)(gamma32(h->d + 2) * (1.0 + 1e-4));
+  {
+    const double g = gamma32(h->d + 40);
+    a.g2f = (float)(2.0 * g * g * (1.0 + 1e-4));
+  }
+  a.om_eps_rd = std::nextafter((float)(1.0 - h->eps_rc), 0.0f);
+  a.inv_omg_ru = std::nextafter((float)(1.0 / (1.0 - gamma32(h->dpad / 32 + 33))), 2.0f);
+  a.om_c_rd = std::nextafter((float)(1.0 - h->c_scr), 0.0f);
+  a.inv_pairnorm = h->inv_pairnorm;
+  a.tight_f = 1.0 - gamma64(h->d + 8);
+  a.inv_denom = h->radius_scale / (h->sigma * 1.4142135623730951);
+  a.inv_denom_safe = h->radius_scale * (1.0 - 8 * kU64) / (h->sigma * (1.0 + kSigmaSlack) * 1.4142135623730951);
   a.accept = h->ins_accept;
   a.yG = h->ins_yG;
   a.label = h->ins_label;
@@ -400,10 +765,22 @@ void certify_insert(lipcache* h, const float* H, int64_t n, const int32_t* paylo
   a.rank = h->ins_rank;
   a.bcount = h->ins_bcount;
   const int nb = (int)((n + kRows - 1) / kRows);
-  const size_t smem = certify_smem_bytes(h->d, h->C);
-  LC_CUDA(cudaFuncSetAttribute(k_certify, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
-  k_certify<<<nb, kThreads, smem, s>>>(a);
-  LC_LAUNCH_CHECK("k_certify");
+  const int Cp = (h->C + 7) / 8 * 8;
+  const size_t smem_wres = sizeof(float) * ((size_t)h->dpad * Cp + (size_t)h->dpad * kHStride +
+                                            (size_t)kWTile * a.lstride + 1 + 2 * (size_t)h->C) +
+                           sizeof(double) * 2 * kWarps * (size_t)(a.tight ? h->C : 0);
+  if (h->C <= 256 && smem_wres <= 220 * 1024) {
+    const int n_tiles = (int)((n + kWTile - 1) / kWTile);
+    const int grid = n_tiles < h->num_sms ? n_tiles : h->num_sms;
+    LC_CUDA(cudaFuncSetAttribute(k_certify_wres, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_wres));
+    k_certify_wres<<<grid, kThreads, smem_wres, s>>>(a, Cp, h->dpad, n_tiles);
+    LC_LAUNCH_CHECK("k_certify_wres");
+  } else {
+    const size_t smem = certify_smem_bytes(h->d, h->C);
+    LC_CUDA(cudaFuncSetAttribute(k_certify, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+    k_certify<<<nb, kThreads, smem, s>>>(a);
+    LC_LAUNCH_CHECK("k_certify");
+  }
   k_scan<<<1, 1024, 0, s>>>(h->ins_bcount, h->ins_boffset, nb, h->ins_total);
   LC_LAUNCH_CHECK("k_scan");
   ScatterArgs sa;

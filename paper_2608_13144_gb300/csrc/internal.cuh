@@ -126,7 +126,9 @@ struct lipcache {
   float* W = nullptr;        // C x d
   float* b = nullptr;        // C
   double* Wnorm = nullptr;   // C
+  float* Wnorm32 = nullptr;  // C, ||W_c|| rounded up to FP32
   double* pairnorm = nullptr;  // C x C (tight mode)
+  double* inv_pairnorm = nullptr;  // C x C: 1 / pairnorm (0 where pairnorm is 0)
   double* gram[2] = {nullptr, nullptr};  // d x d FP64
   lc::SpecResult* spec = nullptr;        // device
   lc::SpecResult* spec_host = nullptr;   // pinned

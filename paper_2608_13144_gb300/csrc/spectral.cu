@@ -176,7 +176,8 @@ __global__ void __launch_bounds__(kPowerThreads) k_power(const float* __restrict
 // ||W_c|| for every class and, for the tight radius, ||W_y - W_j|| for every
 // pair (FP64).
 __global__ void k_row_norms(const float* __restrict__ W, int C, int d, double* __restrict__ Wnorm,
-                            double* __restrict__ pairnorm) {
+                            float* __restrict__ Wnorm32, double* __restrict__ pairnorm,
+                            double* __restrict__ inv_pairnorm) {
   const int y = blockIdx.y;
   const int j = blockIdx.x * blockDim.x + threadIdx.x;
   if (j >= C) return;
@@ -187,11 +188,13 @@ __global__ void k_row_norms(const float* __restrict__ W, int C, int d, double* _
       acc = fma(e, e, acc);
     }
     pairnorm[(size_t)y * C + j] = sqrt(acc);
+    inv_pairnorm[(size_t)y * C + j] = acc > 0.0 ? 1.0 / sqrt(acc) : 0.0;
   }
   if (j == y) {
     double n2 = 0.0;
     for (int k = 0; k < d; ++k) n2 = fma((double)W[(size_t)y * d + k], (double)W[(size_t)y * d + k], n2);
     Wnorm[y] = sqrt(n2);
+    Wnorm32[y] = __double2float_ru(sqrt(n2) * (1.0 + 1e-15));
   }
 }
 
@@ -216,7 +219,9 @@ void spectral_norm(lipcache* h, cudaStream_t s) {
   k_power<<<1, kPowerThreads, smem, s>>>(h->W, C, d, As, h->max_iter, h->spec);
   LC_LAUNCH_CHECK("k_power");
   dim3 rb(128), rg((C + 127) / 128, C);
-  k_row_norms<<<rg, rb, 0, s>>>(h->W, C, d, h->Wnorm, h->radius_mode == LIPCACHE_RADIUS_TIGHT ? h->pairnorm : nullptr);
+  const bool tight = h->radius_mode == LIPCACHE_RADIUS_TIGHT;
+  k_row_norms<<<rg, rb, 0, s>>>(h->W, C, d, h->Wnorm, h->Wnorm32, tight ? h->pairnorm : nullptr,
+                                tight ? h->inv_pairnorm : nullptr);
   LC_LAUNCH_CHECK("k_row_norms");
 }
 
