@@ -9,6 +9,8 @@ Functions (each follows the passage cited in the C source):
   logits                        Eq. 5
   certify                       Algorithm 1 with Eqs. 6, 20, 21 and Eq. 29
   probe                         Algorithm 2 with Eqs. 13-15
+  probe_writeback               Algorithm 2 with write-back of certified misses
+  consistency                   certified-consistency rate of the hits (Sec. 5)
   pair_dist                     ||q - k||_2 for given pairs
 """
 from __future__ import annotations
@@ -147,6 +149,54 @@ def probe(keys, radius, labels, Q, band_rel=1e-5) -> dict:
                     out["index"], out["label"], out["dist"], out["n_hits"], out["decision_band"],
                     out["selection_band"], float(band_rel))
     return out
+
+
+def probe_writeback(cache, W, b, sigma, Q, payload=None, require_consistency=False,
+                    radius_mode=RADIUS_CONSERVATIVE, scale=1.0, band_rel=1e-5) -> dict:
+    """Algorithm 2 with write-back enabled. The distances D_{k,i} are formed
+    once for the whole batch against the cache as it stood when the batch
+    arrived, so no query of a batch sees another query's write-back. Every
+    missed query is then certified as in Algorithm 1 (payload: the given
+    labels, else the proxy label y^G) and, if accepted, appended in query
+    order. ``cache`` holds keys / radius / label / yG as returned by
+    build_cache. Returns the probe result, ``inserted`` (new cache index of
+    each written-back query, -1 otherwise) and the grown cache."""
+    res = probe(cache["keys"], cache["radius"], cache["label"], Q, band_rel)
+    Q = _f32(Q)
+    cert = certify(W, b, sigma, Q, payload, require_consistency, radius_mode, scale)
+    add = (res["index"] < 0) & cert["accept"]
+    n0 = int(np.asarray(cache["keys"]).shape[0])
+    inserted = np.full(Q.shape[0], -1, dtype=np.int64)
+    inserted[add] = n0 + np.arange(int(add.sum()), dtype=np.int64)
+    grown = {
+        "keys": _f32(np.concatenate([np.asarray(cache["keys"], np.float32).reshape(n0, Q.shape[1]), Q[add]])),
+        "radius": np.concatenate([np.asarray(cache["radius"], np.float64), cert["radius"][add]]),
+        "label": np.concatenate([np.asarray(cache["label"], np.int32), cert["label"][add]]).astype(np.int32),
+        "yG": np.concatenate([np.asarray(cache["yG"], np.int32), cert["yG"][add]]).astype(np.int32),
+    }
+    return {"probe": res, "inserted": inserted, "cert": cert, "cache": grown}
+
+
+def consistency(W, b, Q, hit_index, yG_table) -> dict:
+    """Certified-consistency check of the hits (the rate reported in Sec. 5):
+    for every query with hit_index >= 0, whether the head's argmax on the
+    query (FP64 logits, Eq. 5; lowest class on ties) equals y^G of the hit
+    entry. ``consistent`` is 1 / 0 per hit and -1 on a miss; ``gap`` is the
+    query's FP64 top-two logit gap (+inf on a miss), for band exclusion."""
+    Q = _f32(Q)
+    hit_index = np.asarray(hit_index, dtype=np.int64)
+    yG_table = np.asarray(yG_table, dtype=np.int32)
+    B = Q.shape[0]
+    out = np.full(B, -1, dtype=np.int8)
+    gap = np.full(B, np.inf)
+    for k in np.nonzero(hit_index >= 0)[0]:
+        s = logits(W, b, Q[k])
+        y = int(np.argmax(s))
+        top = np.sort(s)
+        gap[k] = top[-1] - top[-2]
+        out[k] = 1 if y == int(yG_table[hit_index[k]]) else 0
+    n_hits = int((hit_index >= 0).sum())
+    return {"consistent": out, "n_hits": n_hits, "n_consistent": int((out == 1).sum()), "gap": gap}
 
 
 def pair_dist(Q, K, qi, ki) -> np.ndarray:

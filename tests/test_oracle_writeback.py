@@ -1,0 +1,126 @@
+"""Pins for the oracle's write-back (Algorithm 2, miss branch) and its
+certified-consistency check (Sec. 5 metrics, Lemma of Sec. 4.2).
+
+Hand-derived golden values (tests/golden), the Lemma as an invariant, and an
+independent FP64 argmax through numpy's matmul.
+"""
+import numpy as np
+import pytest
+
+import oracle
+from conftest import golden
+
+
+def _cache(W, b, sigma, rows):
+    c = oracle.build_cache(np.array(W, np.float32), np.array(b, np.float32), sigma, np.array(rows, np.float32))
+    return {"keys": c["keys"], "radius": c["radius"], "label": c["label"], "yG": c["yG"]}
+
+
+def test_golden_writeback_proxy_labels():
+    g = golden("writeback_two_class.json")
+    W, b = np.array(g["W"], np.float32), np.array(g["b"], np.float32)
+    cache = _cache(W, b, g["sigma"], g["rows"])
+    r = oracle.probe_writeback(cache, W, b, g["sigma"], np.array(g["queries"], np.float32))
+    assert r["probe"]["index"].tolist() == g["expect_index"]
+    assert r["inserted"].tolist() == g["expect_inserted"]
+    np.testing.assert_allclose(r["cache"]["radius"], g["expect_radius"], rtol=1e-15)
+    assert r["cache"]["yG"].tolist() == g["expect_yG"]
+    assert r["cache"]["label"].tolist() == g["expect_yG"]  # proxy label = y^G
+    q = np.array(g["queries"], np.float32)
+    np.testing.assert_array_equal(r["cache"]["keys"][1:], q[r["inserted"] >= 0])
+
+
+def test_golden_writeback_require_consistency():
+    g = golden("writeback_two_class.json")
+    W, b = np.array(g["W"], np.float32), np.array(g["b"], np.float32)
+    cache = _cache(W, b, g["sigma"], g["rows"])
+    r = oracle.probe_writeback(cache, W, b, g["sigma"], np.array(g["queries"], np.float32),
+                               payload=np.array(g["payload"], np.int32), require_consistency=True)
+    assert r["inserted"].tolist() == g["expect_inserted_consistent"]
+    assert r["cache"]["label"].tolist() == g["expect_label_consistent"]
+
+
+@pytest.mark.parametrize("which", ["inflated", "certified"])
+def test_golden_consistency(which):
+    g = golden("consistency_two_class.json")
+    W, b = np.array(g["W"], np.float32), np.array(g["b"], np.float32)
+    keys = np.array(g["keys"], np.float32)
+    Q = np.array(g["queries"], np.float32)
+    radius = np.array([g["radius_" + which]], np.float64)
+    p = oracle.probe(keys, radius, np.array(g["yG"], np.int32), Q)
+    assert p["index"].tolist() == g["expect_hit_" + which]
+    c = oracle.consistency(W, b, Q, p["index"], np.array(g["yG"], np.int32))
+    assert c["consistent"].tolist() == g["expect_consistent_" + which]
+    exp = np.array(g["expect_consistent_" + which])
+    assert c["n_hits"] == int((exp >= 0).sum()) and c["n_consistent"] == int((exp == 1).sum())
+
+
+def _instance(seed, C, d, n_rows, n_q):
+    rng = np.random.default_rng(seed)
+    W = rng.standard_normal((C, d)).astype(np.float32)
+    b = (0.1 * rng.standard_normal(C)).astype(np.float32)
+    rows = (2 * rng.standard_normal((n_rows, d))).astype(np.float32)
+    return rng, W, b, rows
+
+
+@pytest.mark.parametrize("seed,C,d", [(0, 3, 2), (1, 5, 4), (2, 4, 8)])
+def test_writeback_batch_semantics(seed, C, d):
+    """The batch is probed against the old cache (same result as a plain
+    probe), only misses are written back, in query order, and each
+    written-back query hits the grown cache (it lies at distance 0 from its
+    own entry, whose radius is positive)."""
+    rng, W, b, rows = _instance(seed, C, d, 24, 64)
+    s = oracle.sigma_max(W)
+    cache = _cache(W, b, s, rows)
+    Q = (2 * rng.standard_normal((64, d))).astype(np.float32)
+    Q[::4] = rows[rng.integers(0, len(rows), 16)] + 0.01  # some hits
+    r = oracle.probe_writeback(cache, W, b, s, Q)
+    plain = oracle.probe(cache["keys"], cache["radius"], cache["label"], Q)
+    np.testing.assert_array_equal(r["probe"]["index"], plain["index"])
+    ins = r["inserted"]
+    assert np.all(ins[plain["index"] >= 0] == -1)
+    n0 = len(cache["keys"])
+    new = ins[ins >= 0]
+    np.testing.assert_array_equal(new, n0 + np.arange(len(new)))
+    assert np.all(r["cache"]["radius"][n0:] > 0)
+    again = oracle.probe(r["cache"]["keys"], r["cache"]["radius"], r["cache"]["label"], Q[ins >= 0])
+    assert np.all(again["index"] >= 0)
+    assert np.all(again["dist"] == 0.0)
+
+
+def _argmax_numpy(W, b, Q):
+    s = Q.astype(np.float64) @ W.astype(np.float64).T + b.astype(np.float64)
+    return np.argmax(s, axis=1)
+
+
+@pytest.mark.parametrize("seed,C,d", [(3, 2, 2), (4, 3, 3), (5, 6, 4)])
+def test_consistency_lemma_and_planted_radius(seed, C, d):
+    """Certified radii: every hit strictly inside r(1 - 1e-9) is consistent
+    (the Lemma). Radii inflated 4x: the check flags exactly the hits whose
+    numpy FP64 argmax differs from the entry's y^G."""
+    rng, W, b, rows = _instance(seed, C, d, 16, 0)
+    s = oracle.sigma_max(W)
+    cache = _cache(W, b, s, rows)
+    n = len(cache["keys"])
+    assert n > 0
+    pick = rng.integers(0, n, 400)
+    u = rng.standard_normal((400, d))
+    u /= np.linalg.norm(u, axis=1, keepdims=True)
+    Q = (cache["keys"][pick] + u * (cache["radius"][pick] * rng.random(400) * 3.5)[:, None]).astype(np.float32)
+
+    p = oracle.probe(cache["keys"], cache["radius"], cache["label"], Q)
+    c = oracle.consistency(W, b, Q, p["index"], cache["yG"])
+    hit = p["index"] >= 0
+    assert c["n_hits"] == int(hit.sum()) > 0
+    inner = hit & (p["dist"] < cache["radius"][np.maximum(p["index"], 0)] * (1 - 1e-9))
+    assert np.all(c["consistent"][inner] == 1)
+
+    big = cache["radius"] * 4
+    p4 = oracle.probe(cache["keys"], big, cache["label"], Q)
+    c4 = oracle.consistency(W, b, Q, p4["index"], cache["yG"])
+    h4 = p4["index"] >= 0
+    want = (_argmax_numpy(W, b, Q) == cache["yG"][np.maximum(p4["index"], 0)]).astype(np.int8)
+    clear = h4 & (c4["gap"] > 1e-9)
+    np.testing.assert_array_equal(c4["consistent"][clear], want[clear])
+    assert np.all(c4["consistent"][~h4] == -1)
+    assert c4["n_consistent"] < c4["n_hits"]  # the inflated radii do cross the boundary
