@@ -169,6 +169,54 @@ lipcache_status lipcache_probe(lipcache_t* h, const float* Q, int64_t B, int64_t
                                float* out_dist, lipcache_stream_t stream);
 
 /*
+ * Lookup with write-back (Algorithm 2 with its write-back flag set): probe
+ * the batch as lipcache_probe does, then certify every missed query as
+ * lipcache_insert does and append the accepted ones, in query order, all on
+ * `stream` with no host round trip in between. The whole batch is probed
+ * against the cache as it stood when the call began (Algorithm 2 forms the
+ * distances D_{k,i} once, before its per-query loop), so a query never hits
+ * an entry written back by the same batch. Hits are never inserted.
+ *   Q, B, out_label, out_dist   as for lipcache_probe
+ *   out_index     B int64 (device), required: i*, or -1 on a miss
+ *   payload       B int32 (device), nullable -> proxy labels y^G (the label
+ *                 Algorithm 2 derives from the GuardNet logits)
+ *   require_consistency  as for lipcache_insert
+ *   out_inserted  B int64 (device), nullable: new cache index of a written-
+ *                 back query, else -1 (hit, or skipped by Algorithm 1's rules)
+ *   n_inserted    host, nullable: number of entries appended
+ * Synchronises `stream`. All or nothing: if size + B > capacity nothing is
+ * probed or written and E_FULL is returned (the number of misses is not known
+ * in advance). Errors: those of lipcache_probe and lipcache_insert.
+ */
+lipcache_status lipcache_probe_writeback(lipcache_t* h, const float* Q, int64_t B, const int32_t* payload,
+                                         int32_t require_consistency, int64_t* out_index, int32_t* out_label,
+                                         float* out_dist, int64_t* out_inserted, int64_t* n_inserted,
+                                         lipcache_stream_t stream);
+
+/*
+ * Certified-consistency check (the rate reported with every experiment of
+ * Sec. 5; by the Lemma of Sec. 4.2 it is 1 for certified radii): for every
+ * query k with hit_index[k] >= 0, whether the head's argmax on q_k (Eq. 5,
+ * lowest class on ties) equals y^G of entry hit_index[k]. The argmax is that
+ * of the insert path (FP32 logits with proven error bounds, candidates
+ * recomputed with a compensated dot product), so it can differ from the
+ * exact one only when the two largest logits are within ~1e-9 relative.
+ *   Q               B x d FP32 (device)
+ *   hit_index       B int64 (device), e.g. lipcache_probe's out_index;
+ *                   values must be -1 or in [0, size)
+ *   out_consistent  B int8 (device), nullable: 1 consistent, 0 not, -1 miss
+ *   n_hits          host, nullable: queries with hit_index >= 0
+ *   n_consistent    host, nullable: of those, the consistent ones
+ * Synchronises `stream`. Errors: E_STATE (no head), E_INVALID (NULL Q or
+ * hit_index, or an index outside [-1, size): reported after the kernel ran;
+ * out_consistent is then -1 for such queries and they are not counted),
+ * E_NOMEM, E_CUDA.
+ */
+lipcache_status lipcache_consistency(lipcache_t* h, const float* Q, int64_t B, const int64_t* hit_index,
+                                     int8_t* out_consistent, int64_t* n_hits, int64_t* n_consistent,
+                                     lipcache_stream_t stream);
+
+/*
  * lipcache_probe for callers holding HOST buffers: copies Q to the device,
  * probes, copies the results back and synchronises `stream`.
  *   Q_host     B x d FP32 (host; pinned memory gives asynchronous copies)

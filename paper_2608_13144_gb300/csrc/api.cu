@@ -183,8 +183,8 @@ LC_API lipcache_status lipcache_create(int32_t d, int32_t C, int64_t capacity, i
     dev_alloc(h->table.radius, rows);
     dev_alloc(h->table.label, rows);
     dev_alloc(h->table.yG, rows);
-    dev_alloc(h->ins_total, 1);
-    LC_CUDA(cudaMallocHost(&h->ins_total_host, sizeof(int64_t)));
+    dev_alloc(h->ins_total, 4);
+    LC_CUDA(cudaMallocHost(&h->ins_total_host, 4 * sizeof(int64_t)));
     dev_alloc(h->stats, 1);
     LC_CUDA(cudaMemset(h->stats, 0, sizeof(lc::DevStats)));
     LC_CUDA(cudaMallocHost(&h->stats_host, sizeof(lc::DevStats)));
@@ -269,6 +269,54 @@ LC_API lipcache_status lipcache_probe(lipcache_t* h, const float* Q, int64_t B, 
     LC_REQUIRE(((uintptr_t)Q & 3) == 0, LIPCACHE_E_INVALID, "Q must be 4-byte aligned");
     use_device(h);
     lc::probe(h, Q, B, out_index, out_label, out_dist, reinterpret_cast<cudaStream_t>(stream));
+  });
+}
+
+LC_API lipcache_status lipcache_probe_writeback(lipcache_t* h, const float* Q, int64_t B, const int32_t* payload,
+                                                int32_t require_consistency, int64_t* out_index, int32_t* out_label,
+                                                float* out_dist, int64_t* out_inserted, int64_t* n_inserted,
+                                                lipcache_stream_t stream) {
+  if (n_inserted) *n_inserted = 0;
+  return guarded([&] {
+    check_handle(h);
+    LC_REQUIRE(h->head_set, LIPCACHE_E_STATE, "probe before set_head");
+    LC_REQUIRE(B >= 0 && B <= (1LL << 22), LIPCACHE_E_INVALID, "B must be in [0, 2^22]");
+    if (B == 0) return;
+    LC_REQUIRE(Q != nullptr && out_index != nullptr, LIPCACHE_E_INVALID, "Q and out_index are required");
+    LC_REQUIRE(((uintptr_t)Q & 3) == 0, LIPCACHE_E_INVALID, "Q must be 4-byte aligned");
+    LC_REQUIRE(B <= h->capacity - h->size, LIPCACHE_E_FULL, "write-back of B queries could exceed the capacity");
+    use_device(h);
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    lc::probe(h, Q, B, out_index, out_label, out_dist, s);
+    lc::certify_insert(h, Q, B, payload, require_consistency, out_inserted, nullptr, s, out_index);
+    LC_CUDA(cudaMemcpyAsync(h->ins_total_host, h->ins_total, sizeof(int64_t), cudaMemcpyDeviceToHost, s));
+    LC_CUDA(cudaStreamSynchronize(s));
+    const int64_t acc = *h->ins_total_host;
+    h->size += acc;
+    if (n_inserted) *n_inserted = acc;
+  });
+}
+
+LC_API lipcache_status lipcache_consistency(lipcache_t* h, const float* Q, int64_t B, const int64_t* hit_index,
+                                            int8_t* out_consistent, int64_t* n_hits, int64_t* n_consistent,
+                                            lipcache_stream_t stream) {
+  if (n_hits) *n_hits = 0;
+  if (n_consistent) *n_consistent = 0;
+  return guarded([&] {
+    check_handle(h);
+    LC_REQUIRE(h->head_set, LIPCACHE_E_STATE, "consistency check before set_head");
+    LC_REQUIRE(B >= 0 && B <= (1LL << 22), LIPCACHE_E_INVALID, "B must be in [0, 2^22]");
+    if (B == 0) return;
+    LC_REQUIRE(Q != nullptr && hit_index != nullptr, LIPCACHE_E_INVALID, "Q and hit_index are required");
+    LC_REQUIRE(((uintptr_t)Q & 3) == 0, LIPCACHE_E_INVALID, "Q must be 4-byte aligned");
+    use_device(h);
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    lc::consistency_check(h, Q, B, hit_index, out_consistent, s);
+    LC_CUDA(cudaMemcpyAsync(h->ins_total_host + 1, h->ins_total + 1, 3 * sizeof(int64_t), cudaMemcpyDeviceToHost, s));
+    LC_CUDA(cudaStreamSynchronize(s));
+    if (n_hits) *n_hits = h->ins_total_host[1];
+    if (n_consistent) *n_consistent = h->ins_total_host[2];
+    LC_REQUIRE(h->ins_total_host[3] == 0, LIPCACHE_E_INVALID, "hit_index holds values outside [-1, size)");
   });
 }
 

@@ -59,6 +59,7 @@ struct CertArgs {
   float om_eps_rd;       // 1 - eps_rc, rounded down
   float inv_omg_ru;      // 1 / (1 - gamma_rc), rounded up
   float om_c_rd;         // 1 - c_screen, rounded down
+  const int64_t* miss_of;      // nullable: row accepted only if miss_of[row] < 0 (write-back)
   const double* inv_pairnorm;  // 1 / ||W_y - W_j|| (tight mode)
   double tight_f;              // 1 - gamma_{d+8} (FP64)
   uint8_t* accept;
@@ -290,7 +291,7 @@ __device__ void certify_rows_fast(const CertArgs& a, int64_t row0, int nrows, in
     const double r64 = mval * a.inv_denom;
     const double rs = (mlo > 0.0) ? __dmul_rd(mlo, a.inv_denom_safe) : 0.0;
     const int32_t lab = a.payload ? a.payload[row] : r_y;
-    const bool acc = !(a.require_consistency && lab != r_y) && (r64 > 0.0);
+    const bool acc = !(a.require_consistency && lab != r_y) && (r64 > 0.0) && !(a.miss_of && a.miss_of[row] >= 0);
     // probe thresholds in FP32 with directed rounding (each step only lowers
     // rr and tau): rr <= r_safe^2 (1 - eps_rc), tau as in probe_tc.cu
     const float rs32 = __double2float_rd(rs);
@@ -429,7 +430,7 @@ __device__ void certify_row(const CertArgs& a, int64_t row, const float* __restr
 
     if (lane == 0) {
       const int32_t lab = a.payload ? a.payload[row] : y;
-      const bool acc = !(a.require_consistency && lab != y) && (r64 > 0.0);
+      const bool acc = !(a.require_consistency && lab != y) && (r64 > 0.0) && !(a.miss_of && a.miss_of[row] >= 0);
       const float rs32 = __double2float_rd(rs);
       const float rr = __fmul_rd(__fmul_rd(rs32, rs32), a.om_eps_rd);
       const float Rt = __fmul_ru(rr, a.inv_omg_ru);
@@ -685,6 +686,37 @@ __global__ void __launch_bounds__(256) k_scatter(ScatterArgs a) {
   }
 }
 
+// Certified-consistency check of probe hits: the insert path's argmax y^G of
+// each query (already in yq) against y^G of the hit entry. counts[0..2]:
+// hits, consistent hits, indices outside [-1, size).
+__global__ void __launch_bounds__(256) k_consistency(const int64_t* __restrict__ hit, const int32_t* __restrict__ yq,
+                                                     const int32_t* __restrict__ yG_table, int64_t size, int64_t B,
+                                                     int8_t* __restrict__ out, int64_t* __restrict__ counts) {
+  const int64_t k = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  int h = 0, c = 0, bad = 0;
+  if (k < B) {
+    const int64_t i = hit[k];
+    int8_t v = -1;
+    if (i >= 0 && i < size) {
+      h = 1;
+      c = yq[k] == yG_table[i];
+      v = (int8_t)c;
+    } else if (i != -1) {
+      bad = 1;
+    }
+    if (out) out[k] = v;
+  }
+  const unsigned full = 0xffffffffu;
+  h = __popc(__ballot_sync(full, h));
+  c = __popc(__ballot_sync(full, c));
+  bad = __popc(__ballot_sync(full, bad));
+  if ((threadIdx.x & 31) == 0) {
+    if (h) atomicAdd(reinterpret_cast<unsigned long long*>(counts), (unsigned long long)h);
+    if (c) atomicAdd(reinterpret_cast<unsigned long long*>(counts + 1), (unsigned long long)c);
+    if (bad) atomicAdd(reinterpret_cast<unsigned long long*>(counts + 2), (unsigned long long)bad);
+  }
+}
+
 template <typename T>
 void grow(T*& p, int64_t n) {
   if (p) cudaFree(p);
@@ -718,8 +750,12 @@ size_t certify_smem_bytes(int d, int C) {
   return sizeof(double) * 2 * kWarps * (size_t)C + sizeof(float) * (size_t)kRows * (hstride + lstride);
 }
 
-void certify_insert(lipcache* h, const float* H, int64_t n, const int32_t* payload, int require_consistency,
-                    int64_t* out_index, float* out_radius, cudaStream_t s) {
+namespace {
+
+// Per-row certification of H (n rows) into the insert scratch: accept, y^G,
+// label, radius, probe thresholds, per-32-row ranks and counts.
+void launch_certify(lipcache* h, const float* H, int64_t n, const int32_t* payload, int require_consistency,
+                    const int64_t* miss_of, cudaStream_t s) {
   ensure_insert_scratch(h, n);
   CertArgs a;
   a.H = H;
@@ -751,6 +787,7 @@ void certify_insert(lipcache* h, const float* H, int64_t n, const int32_t* paylo
   a.om_eps_rd = std::nextafter((float)(1.0 - h->eps_rc), 0.0f);
   a.inv_omg_ru = std::nextafter((float)(1.0 / (1.0 - gamma32(h->dpad / 32 + 33))), 2.0f);
   a.om_c_rd = std::nextafter((float)(1.0 - h->c_scr), 0.0f);
+  a.miss_of = miss_of;
   a.inv_pairnorm = h->inv_pairnorm;
   a.tight_f = 1.0 - gamma64(h->d + 8);
   a.inv_denom = h->radius_scale / (h->sigma * 1.4142135623730951);
@@ -781,6 +818,14 @@ void certify_insert(lipcache* h, const float* H, int64_t n, const int32_t* paylo
     k_certify<<<nb, kThreads, smem, s>>>(a);
     LC_LAUNCH_CHECK("k_certify");
   }
+}
+
+}  // namespace
+
+void certify_insert(lipcache* h, const float* H, int64_t n, const int32_t* payload, int require_consistency,
+                    int64_t* out_index, float* out_radius, cudaStream_t s, const int64_t* miss_of) {
+  launch_certify(h, H, n, payload, require_consistency, miss_of, s);
+  const int nb = (int)((n + kRows - 1) / kRows);
   k_scan<<<1, 1024, 0, s>>>(h->ins_bcount, h->ins_boffset, nb, h->ins_total);
   LC_LAUNCH_CHECK("k_scan");
   ScatterArgs sa;
@@ -803,6 +848,15 @@ void certify_insert(lipcache* h, const float* H, int64_t n, const int32_t* paylo
   sa.out_radius = out_radius;
   k_scatter<<<(unsigned)((n + 7) / 8), 256, 0, s>>>(sa);
   LC_LAUNCH_CHECK("k_scatter");
+}
+
+void consistency_check(lipcache* h, const float* Q, int64_t B, const int64_t* hit_index, int8_t* out,
+                       cudaStream_t s) {
+  launch_certify(h, Q, B, nullptr, 0, nullptr, s);
+  LC_CUDA(cudaMemsetAsync(h->ins_total + 1, 0, 3 * sizeof(int64_t), s));
+  k_consistency<<<(unsigned)((B + 255) / 256), 256, 0, s>>>(hit_index, h->ins_yG, h->table.yG, h->size, B, out,
+                                                           h->ins_total + 1);
+  LC_LAUNCH_CHECK("k_consistency");
 }
 
 }  // namespace lc

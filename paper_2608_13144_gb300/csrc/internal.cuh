@@ -147,8 +147,8 @@ struct lipcache {
   int32_t* ins_rank = nullptr;
   int32_t* ins_bcount = nullptr;
   int32_t* ins_boffset = nullptr;
-  int64_t* ins_total = nullptr;       // device
-  int64_t* ins_total_host = nullptr;  // pinned
+  int64_t* ins_total = nullptr;       // device, 4: rows appended; consistency counts
+  int64_t* ins_total_host = nullptr;  // pinned, 4
 
   // probe scratch (grows)
   int64_t q_cap = 0;  // rows (multiple of 128)
@@ -184,8 +184,14 @@ namespace lc {
 // spectral.cu
 void spectral_norm(lipcache* h, cudaStream_t s);
 // certify.cu
+// Certify H and append the accepted rows; miss_of (nullable, n entries) limits
+// acceptance to rows with miss_of[row] < 0 (write-back of probe misses).
 void certify_insert(lipcache* h, const float* H, int64_t n, const int32_t* payload, int require_consistency,
-                    int64_t* out_index, float* out_radius, cudaStream_t s);
+                    int64_t* out_index, float* out_radius, cudaStream_t s, const int64_t* miss_of = nullptr);
+// Certified-consistency check: argmax of the head on Q against y^G of the hit
+// entries; counts (hits, consistent, invalid index) land in ins_total[1..3].
+void consistency_check(lipcache* h, const float* Q, int64_t B, const int64_t* hit_index, int8_t* out,
+                       cudaStream_t s);
 // probe.cu
 void probe(lipcache* h, const float* Q, int64_t B, int64_t* out_index, int32_t* out_label, float* out_dist,
            cudaStream_t s);

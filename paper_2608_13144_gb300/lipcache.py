@@ -103,6 +103,42 @@ class LipCache:
         check(self.L.lipcache_probe(self._h, _ptr(Q), B, _ptr(idx), _ptr(lab), _ptr(dist), _stream(self.device)))
         return idx, lab, dist
 
+    def probe_writeback(self, Q: torch.Tensor, payload: torch.Tensor | None = None,
+                        require_consistency: bool = False):
+        """Probe, then certify and append the missed queries (Algorithm 2 with
+        write-back). The batch is probed against the cache as it was before
+        the call. Returns (index, label, dist, inserted, n_inserted);
+        inserted[k] is the new cache index of query k or -1."""
+        Q = self._dev(Q, torch.float32, "Q")
+        B = Q.shape[0]
+        if Q.dim() != 2 or (B and Q.shape[1] != self.d):
+            raise ValueError("Q must be B x d")
+        if payload is not None:
+            payload = self._dev(payload, torch.int32, "payload")
+        idx = torch.empty(B, dtype=torch.int64, device=self.device)
+        lab = torch.empty(B, dtype=torch.int32, device=self.device)
+        dist = torch.empty(B, dtype=torch.float32, device=self.device)
+        ins = torch.empty(B, dtype=torch.int64, device=self.device)
+        n = C.c_int64()
+        check(self.L.lipcache_probe_writeback(self._h, _ptr(Q), B, _ptr(payload), int(bool(require_consistency)),
+                                              _ptr(idx), _ptr(lab), _ptr(dist), _ptr(ins), C.byref(n),
+                                              _stream(self.device)))
+        return idx, lab, dist, ins, n.value
+
+    def consistency(self, Q: torch.Tensor, hit_index: torch.Tensor):
+        """Certified-consistency check of hits: (per-query int8 1/0/-1,
+        n_hits, n_consistent)."""
+        Q = self._dev(Q, torch.float32, "Q")
+        hit_index = self._dev(hit_index, torch.int64, "hit_index")
+        B = Q.shape[0]
+        if Q.dim() != 2 or (B and Q.shape[1] != self.d) or hit_index.shape != (B,):
+            raise ValueError("Q must be B x d and hit_index must have B entries")
+        out = torch.empty(B, dtype=torch.int8, device=self.device)
+        nh, nc = C.c_int64(), C.c_int64()
+        check(self.L.lipcache_consistency(self._h, _ptr(Q), B, _ptr(hit_index), _ptr(out), C.byref(nh),
+                                          C.byref(nc), _stream(self.device)))
+        return out, nh.value, nc.value
+
     def probe_noalloc(self, Q: torch.Tensor, out):
         """probe() without any device allocation, for callers that cannot
         allocate while they run: the scratch is a fixed array inside the

@@ -59,6 +59,12 @@ def test_null_handle_calls(lib):
     assert lib.lipcache_set_head(None, None, None, None, None) == 1
     assert lib.lipcache_probe(None, None, 0, None, None, None, None) == 1
     assert lib.lipcache_insert(None, None, 0, None, 0, None, None, None, None) == 1
+    n = C.c_int64(7)
+    assert lib.lipcache_probe_writeback(None, None, 0, None, 0, None, None, None, None, C.byref(n), None) == 1
+    assert n.value == 0
+    nh, nc = C.c_int64(7), C.c_int64(7)
+    assert lib.lipcache_consistency(None, None, 0, None, None, C.byref(nh), C.byref(nc), None) == 1
+    assert nh.value == 0 and nc.value == 0
 
 
 def test_create_without_gpu_fails_cleanly(lib):
