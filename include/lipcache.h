@@ -79,7 +79,7 @@ typedef struct lipcache_info {
   int32_t sigma_iterations; /* power iterations used by the last set_head */
   double sigma;             /* sigma_max(W) of the current head (0 before set_head) */
   double sigma_residual;    /* ||W^T W v - theta v|| / theta at exit */
-  double radius_scale;      /* kappa in (0, 1]: radius tightening factor (Sec. 5.4) */
+  double radius_scale;      /* kappa in (0, 1]: radius tightening factor (Sec. 5.6) */
   double eps_recheck;       /* relative deflation of r^2 covering the FP32 recheck error */
   double c_screen;          /* relative slack of the tensor-core screen */
   int64_t candidates;       /* screen candidates rechecked since the last reset */
@@ -251,7 +251,7 @@ lipcache_status lipcache_probe_noalloc(lipcache_t* h, const float* Q, int64_t B,
  * or TENSOR when d > 256. */
 lipcache_status lipcache_set_probe_path(lipcache_t* h, int32_t path);
 
-/* Radius tightening kappa in (0, 1] (Sec. 5.4): radii of rows inserted
+/* Radius tightening kappa in (0, 1] (Sec. 5.6): radii of rows inserted
  * afterwards are multiplied by kappa. Only while the cache is empty. */
 lipcache_status lipcache_set_radius_scale(lipcache_t* h, double kappa);
 

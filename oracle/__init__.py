@@ -11,6 +11,8 @@ Functions (each follows the passage cited in the C source):
   probe                         Algorithm 2 with Eqs. 13-15
   probe_writeback               Algorithm 2 with write-back of certified misses
   consistency                   certified-consistency rate of the hits (Sec. 5)
+  interclass_radius             empirical inter-class-distance radius (Sec. 5.4)
+  global_radius                 one global threshold for every entry (Sec. 5.4)
   pair_dist                     ||q - k||_2 for given pairs
 """
 from __future__ import annotations
@@ -197,6 +199,50 @@ def consistency(W, b, Q, hit_index, yG_table) -> dict:
         out[k] = 1 if y == int(yG_table[hit_index[k]]) else 0
     n_hits = int((hit_index >= 0).sum())
     return {"consistent": out, "n_hits": n_hits, "n_consistent": int((out == 1).sum()), "gap": gap}
+
+
+def global_radius(n, tau) -> np.ndarray:
+    """The global nearest-neighbour threshold compared with the certified
+    radius in Sec. 5.4: one radius tau for every cache entry, so a query hits
+    its nearest entry iff that entry is closer than tau."""
+    return np.full(int(n), float(tau), dtype=np.float64)
+
+
+def interclass_radius(keys, labels, n_classes, beta=1.0) -> dict:
+    """The empirical inter-class-distance radius compared with the certified
+    radius in Sec. 5.4. Reading (the paper names only "inter-class distance
+    statistics"): mu_c = mean of the cached keys with label c (FP64);
+    rho_c = beta / 2 * min over present classes c' != c of ||mu_c - mu_c'||,
+    i.e. beta times half the distance to the nearest other class centroid;
+    every entry gets rho of its label. Labels outside [0, C), classes without
+    entries, and classes with no other class present get radius 0."""
+    keys = np.asarray(keys, dtype=np.float64)
+    labels = np.asarray(labels, dtype=np.int64)
+    C = int(n_classes)
+    n, d = keys.shape if keys.ndim == 2 else (0, 0)
+    count = np.zeros(C, dtype=np.int64)
+    total = np.zeros((C, d), dtype=np.float64)
+    for i in range(n):
+        c = int(labels[i])
+        if 0 <= c < C:
+            count[c] += 1
+            total[c] += keys[i]
+    present = count > 0
+    mu = np.zeros_like(total)
+    mu[present] = total[present] / count[present][:, None]
+    rho = np.zeros(C, dtype=np.float64)
+    for c in range(C):
+        if not present[c]:
+            continue
+        best = np.inf
+        for c2 in range(C):
+            if c2 != c and present[c2]:
+                best = min(best, float(np.sqrt(np.sum((mu[c] - mu[c2]) ** 2))))
+        rho[c] = 0.0 if not np.isfinite(best) else beta * 0.5 * best
+    radius = np.zeros(n, dtype=np.float64)
+    ok = (labels >= 0) & (labels < C)
+    radius[ok] = rho[labels[ok]]
+    return {"rho": rho, "radius": radius, "centroid": mu, "count": count}
 
 
 def pair_dist(Q, K, qi, ki) -> np.ndarray:

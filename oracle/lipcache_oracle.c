@@ -143,7 +143,7 @@ void orc_logits(const float* W, const float* b, int C, int d, const float* z, do
  *   r*    = min_{j != y^G, ||W_y - W_j|| > 0} (s_y - s_j) / ||W_y - W_j||
  *                                                 (Remark 4.2, Eq. 29, mode 1;
  *                                                  +inf if every j is skipped)
- *   r    <- scale * r                            (radius tightening, Sec. 5.4)
+ *   r    <- scale * r                            (radius tightening, Sec. 5.6)
  *   payload = caller's label if given, else the proxy label y^G (Sec. 3.3)
  *   skip if consistency is required and payload != y^G, else skip if r <= 0.
  * ------------------------------------------------------------------------ */

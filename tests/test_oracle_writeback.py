@@ -124,3 +124,54 @@ def test_consistency_lemma_and_planted_radius(seed, C, d):
     np.testing.assert_array_equal(c4["consistent"][clear], want[clear])
     assert np.all(c4["consistent"][~h4] == -1)
     assert c4["n_consistent"] < c4["n_hits"]  # the inflated radii do cross the boundary
+
+
+# ---------------------------------------------------------------- empirical radii
+def test_golden_interclass_radius():
+    g = golden("interclass_radius.json")
+    r = oracle.interclass_radius(np.array(g["keys"], np.float32), g["labels"], g["C"], g["beta"])
+    np.testing.assert_allclose(r["rho"], g["expect_rho"], rtol=1e-15)
+    np.testing.assert_allclose(r["radius"], g["expect_radius"], rtol=1e-15)
+    half = oracle.interclass_radius(np.array(g["keys"], np.float32), g["labels"], g["C"], 0.5 * g["beta"])
+    np.testing.assert_allclose(half["rho"], 0.5 * np.array(g["expect_rho"]), rtol=1e-15)
+    one = oracle.interclass_radius(np.array(g["single_class_keys"], np.float32), g["single_class_labels"], g["C"])
+    assert one["rho"].tolist() == g["expect_single_class_rho"]
+
+
+def test_interclass_radius_invariances():
+    """Centroid distances are invariant under a common translation and entry
+    order and scale with the keys; checked against a numpy centroid
+    computation (np.add.at) of the same statistic."""
+    rng = np.random.default_rng(9)
+    keys = rng.standard_normal((300, 5)) * 3
+    labels = rng.integers(0, 6, 300)
+    base = oracle.interclass_radius(keys, labels, 7, 0.8)
+    sums = np.zeros((7, 5))
+    np.add.at(sums, labels, keys)
+    cnt = np.bincount(labels, minlength=7)
+    mu = sums[:6] / cnt[:6, None]
+    D = np.sqrt(((mu[:, None, :] - mu[None, :, :]) ** 2).sum(-1)) + np.diag(np.full(6, np.inf))
+    np.testing.assert_allclose(base["rho"][:6], 0.4 * D.min(1), rtol=1e-12)
+    assert base["rho"][6] == 0.0  # class 6 has no entries
+    perm = rng.permutation(300)
+    np.testing.assert_allclose(oracle.interclass_radius(keys[perm], labels[perm], 7, 0.8)["rho"], base["rho"],
+                               rtol=1e-12)
+    np.testing.assert_allclose(oracle.interclass_radius(keys + 7.5, labels, 7, 0.8)["rho"], base["rho"], rtol=1e-9)
+    np.testing.assert_allclose(oracle.interclass_radius(keys * 4, labels, 7, 0.8)["rho"], 4 * base["rho"],
+                               rtol=1e-12)
+
+
+def test_global_radius_hits_nearest_within_tau():
+    """With one global radius, a query hits iff its nearest cached entry is
+    closer than tau (checked with scipy's cKDTree)."""
+    from scipy.spatial import cKDTree
+    rng = np.random.default_rng(4)
+    keys = rng.standard_normal((200, 3)).astype(np.float32)
+    Q = rng.standard_normal((300, 3)).astype(np.float32)
+    tau = 0.3
+    p = oracle.probe(keys, oracle.global_radius(200, tau), np.arange(200, dtype=np.int32), Q)
+    dist, idx = cKDTree(keys.astype(np.float64)).query(Q.astype(np.float64))
+    clear = np.abs(dist - tau) > 1e-9
+    np.testing.assert_array_equal((p["index"] >= 0)[clear], (dist < tau)[clear])
+    hit = (p["index"] >= 0) & clear
+    np.testing.assert_array_equal(p["index"][hit], idx[hit])
