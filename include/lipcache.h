@@ -58,6 +58,11 @@ typedef enum lipcache_status {
 #define LIPCACHE_RADIUS_CONSERVATIVE 0 /* r  = m / (sigma_max(W) sqrt 2), Eq. 21 */
 #define LIPCACHE_RADIUS_TIGHT 1        /* r* = min_j (s_y - s_j) / ||W_y - W_j||, Eq. 29 */
 
+/* Radius policies of the probe (lipcache_set_radius_policy). */
+#define LIPCACHE_POLICY_CERTIFIED 0  /* per-entry certified radius (Eq. 21 or Eq. 29) */
+#define LIPCACHE_POLICY_GLOBAL 1     /* one global nearest-neighbour threshold (Sec. 5.4) */
+#define LIPCACHE_POLICY_INTERCLASS 2 /* radius from inter-class centroid distances (Sec. 5.4) */
+
 /* Probe kernels. Both return identical results; they differ in speed. */
 #define LIPCACHE_PROBE_AUTO 0   /* tensor path when supported (d <= 256), else exact */
 #define LIPCACHE_PROBE_TENSOR 1 /* tcgen05 TF32 screen, then exact FP32 recheck of candidates */
@@ -92,6 +97,9 @@ typedef struct lipcache_info {
   int64_t kernel_launches;  /* number of timed probes in kernel_ms_total */
   int32_t last_grid;        /* CTAs launched by the last probe's main kernel */
   int32_t last_cluster;     /* CTAs per cluster of that launch (1 = no cluster) */
+  int32_t radius_policy;    /* LIPCACHE_POLICY_* the probe uses */
+  int32_t reserved;
+  double policy_param;      /* tau (GLOBAL) or beta (INTERCLASS); 0 for CERTIFIED */
 } lipcache_info;
 
 /*
@@ -215,6 +223,31 @@ lipcache_status lipcache_probe_writeback(lipcache_t* h, const float* Q, int64_t 
 lipcache_status lipcache_consistency(lipcache_t* h, const float* Q, int64_t B, const int64_t* hit_index,
                                      int8_t* out_consistent, int64_t* n_hits, int64_t* n_consistent,
                                      lipcache_stream_t stream);
+
+/*
+ * Radius policy of the probe: the certified per-entry radius (the default),
+ * or one of the two empirical reuse boundaries Sec. 5.4 compares it with.
+ * The probe kernels are unchanged; only the per-entry thresholds they read
+ * are replaced (the certified ones are kept and come back with
+ * LIPCACHE_POLICY_CERTIFIED).
+ *   LIPCACHE_POLICY_CERTIFIED   param ignored
+ *   LIPCACHE_POLICY_GLOBAL      param = tau > 0: r_i = tau for every entry
+ *   LIPCACHE_POLICY_INTERCLASS  param = beta > 0: mu_c = mean key of the
+ *       entries with payload label c; r_i = rho_{label_i} with rho_c =
+ *       beta / 2 * min over present classes c' != c of ||mu_c - mu_c'||.
+ *       Labels outside [0, C), empty classes and a class with no other class
+ *       present get 0. The statistics are those of the cache at this call;
+ *       entries inserted later take rho of their label from this snapshot.
+ * Thresholds derive from r as the certified ones do from r_safe, so a hit
+ * always lies strictly inside the policy's radius. Empirical boundaries
+ * carry no certificate: lipcache_consistency measures what they give up.
+ *   rho_out  host, nullable: C per-class radii (tau for every class under
+ *            GLOBAL, 0 under CERTIFIED)
+ * Synchronises `stream`. Errors: E_STATE (no head), E_INVALID (policy, or
+ * param not finite and > 0), E_NOMEM, E_CUDA.
+ */
+lipcache_status lipcache_set_radius_policy(lipcache_t* h, int32_t policy, double param, double* rho_out,
+                                           lipcache_stream_t stream);
 
 /*
  * lipcache_probe for callers holding HOST buffers: copies Q to the device,

@@ -65,6 +65,12 @@ void release(lipcache* h) {
   dev_free(h->gram[1]);
   dev_free(h->spec);
   if (h->spec_host) cudaFreeHost(h->spec_host);
+  dev_free(h->rr_emp);
+  dev_free(h->tau_emp);
+  dev_free(h->rho);
+  dev_free(h->rho32);
+  dev_free(h->cls_sum);
+  dev_free(h->cls_cnt);
   dev_free(h->table.keys);
   dev_free(h->table.kn);
   dev_free(h->table.tau);
@@ -253,8 +259,13 @@ LC_API lipcache_status lipcache_insert(lipcache_t* h, const float* H, int64_t n,
     LC_CUDA(cudaMemcpyAsync(h->ins_total_host, h->ins_total, sizeof(int64_t), cudaMemcpyDeviceToHost, s));
     LC_CUDA(cudaStreamSynchronize(s));
     const int64_t acc = *h->ins_total_host;
+    const int64_t first = h->size;
     h->size += acc;
     if (n_accepted) *n_accepted = acc;
+    if (h->policy != LIPCACHE_POLICY_CERTIFIED && acc > 0) {
+      lc::policy_fill(h, first, acc, s);
+      LC_CUDA(cudaStreamSynchronize(s));
+    }
   });
 }
 
@@ -292,8 +303,13 @@ LC_API lipcache_status lipcache_probe_writeback(lipcache_t* h, const float* Q, i
     LC_CUDA(cudaMemcpyAsync(h->ins_total_host, h->ins_total, sizeof(int64_t), cudaMemcpyDeviceToHost, s));
     LC_CUDA(cudaStreamSynchronize(s));
     const int64_t acc = *h->ins_total_host;
+    const int64_t first = h->size;
     h->size += acc;
     if (n_inserted) *n_inserted = acc;
+    if (h->policy != LIPCACHE_POLICY_CERTIFIED && acc > 0) {
+      lc::policy_fill(h, first, acc, s);
+      LC_CUDA(cudaStreamSynchronize(s));
+    }
   });
 }
 
@@ -317,6 +333,24 @@ LC_API lipcache_status lipcache_consistency(lipcache_t* h, const float* Q, int64
     if (n_hits) *n_hits = h->ins_total_host[1];
     if (n_consistent) *n_consistent = h->ins_total_host[2];
     LC_REQUIRE(h->ins_total_host[3] == 0, LIPCACHE_E_INVALID, "hit_index holds values outside [-1, size)");
+  });
+}
+
+LC_API lipcache_status lipcache_set_radius_policy(lipcache_t* h, int32_t policy, double param, double* rho_out,
+                                                  lipcache_stream_t stream) {
+  return guarded([&] {
+    check_handle(h);
+    LC_REQUIRE(h->head_set, LIPCACHE_E_STATE, "set_radius_policy before set_head");
+    LC_REQUIRE(policy == LIPCACHE_POLICY_CERTIFIED || policy == LIPCACHE_POLICY_GLOBAL ||
+                   policy == LIPCACHE_POLICY_INTERCLASS,
+               LIPCACHE_E_INVALID, "unknown radius policy");
+    LC_REQUIRE(policy == LIPCACHE_POLICY_CERTIFIED || (std::isfinite(param) && param > 0.0), LIPCACHE_E_INVALID,
+               "the policy parameter must be finite and > 0");
+    use_device(h);
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    lc::set_radius_policy(h, policy, param, rho_out, s);
+    if (rho_out && policy == LIPCACHE_POLICY_CERTIFIED)
+      for (int c = 0; c < h->C; ++c) rho_out[c] = 0.0;
   });
 }
 
@@ -444,5 +478,8 @@ LC_API lipcache_status lipcache_get_info(lipcache_t* h, lipcache_info* info) {
     info->kernel_launches = h->t_count;
     info->last_grid = h->last_grid;
     info->last_cluster = h->last_cluster;
+    info->radius_policy = h->policy;
+    info->reserved = 0;
+    info->policy_param = h->policy_param;
   });
 }

@@ -56,9 +56,7 @@ struct CertArgs {
   float g2f;             // error factor of the compensated dot product
   double inv_denom;      // kappa / (sigma sqrt 2)
   double inv_denom_safe; // kappa (1 - 8u) / (sigma (1 + slack) sqrt 2)
-  float om_eps_rd;       // 1 - eps_rc, rounded down
-  float inv_omg_ru;      // 1 / (1 - gamma_rc), rounded up
-  float om_c_rd;         // 1 - c_screen, rounded down
+  ThreshConsts tc;       // constants of the probe thresholds
   const int64_t* miss_of;      // nullable: row accepted only if miss_of[row] < 0 (write-back)
   const double* inv_pairnorm;  // 1 / ||W_y - W_j|| (tight mode)
   double tight_f;              // 1 - gamma_{d+8} (FP64)
@@ -292,12 +290,8 @@ __device__ void certify_rows_fast(const CertArgs& a, int64_t row0, int nrows, in
     const double rs = (mlo > 0.0) ? __dmul_rd(mlo, a.inv_denom_safe) : 0.0;
     const int32_t lab = a.payload ? a.payload[row] : r_y;
     const bool acc = !(a.require_consistency && lab != r_y) && (r64 > 0.0) && !(a.miss_of && a.miss_of[row] >= 0);
-    // probe thresholds in FP32 with directed rounding (each step only lowers
-    // rr and tau): rr <= r_safe^2 (1 - eps_rc), tau as in probe_tc.cu
-    const float rs32 = __double2float_rd(rs);
-    const float rr = __fmul_rd(__fmul_rd(rs32, rs32), a.om_eps_rd);
-    const float Rt = __fmul_ru(rr, a.inv_omg_ru);
-    const float tau = __fmul_rd(__fsub_rd(__fmul_rd(a.om_c_rd, r_kn), Rt), 0.5f);
+    float rr, tau;
+    thresholds(__double2float_rd(rs), r_kn, a.tc, rr, tau);
     a.accept[row] = acc ? 1 : 0;
     a.yG[row] = r_y;
     a.label[row] = lab;
@@ -396,7 +390,6 @@ __device__ void certify_row(const CertArgs& a, int64_t row, const float* __restr
     const double sy = ws[y], ey = we[y];
 
     double r64, rs;
-    const double sqrt2 = 1.4142135623730951;
     if (!a.tight) {
       double up_other = -INFINITY;
       for (int c = lane; c < C; c += 32)
@@ -431,10 +424,8 @@ __device__ void certify_row(const CertArgs& a, int64_t row, const float* __restr
     if (lane == 0) {
       const int32_t lab = a.payload ? a.payload[row] : y;
       const bool acc = !(a.require_consistency && lab != y) && (r64 > 0.0) && !(a.miss_of && a.miss_of[row] >= 0);
-      const float rs32 = __double2float_rd(rs);
-      const float rr = __fmul_rd(__fmul_rd(rs32, rs32), a.om_eps_rd);
-      const float Rt = __fmul_ru(rr, a.inv_omg_ru);
-      const float tau = __fmul_rd(__fsub_rd(__fmul_rd(a.om_c_rd, kn), Rt), 0.5f);
+      float rr, tau;
+      thresholds(__double2float_rd(rs), kn, a.tc, rr, tau);
       a.accept[row] = acc ? 1 : 0;
       a.yG[row] = y;
       a.label[row] = lab;
@@ -784,9 +775,7 @@ void launch_certify(lipcache* h, const float* H, int64_t n, const int32_t* paylo
     const double g = gamma32(h->d + 40);
     a.g2f = (float)(2.0 * g * g * (1.0 + 1e-4));
   }
-  a.om_eps_rd = std::nextafter((float)(1.0 - h->eps_rc), 0.0f);
-  a.inv_omg_ru = std::nextafter((float)(1.0 / (1.0 - gamma32(h->dpad / 32 + 33))), 2.0f);
-  a.om_c_rd = std::nextafter((float)(1.0 - h->c_scr), 0.0f);
+  a.tc = thresh_consts(h->dpad);
   a.miss_of = miss_of;
   a.inv_pairnorm = h->inv_pairnorm;
   a.tight_f = 1.0 - gamma64(h->d + 8);

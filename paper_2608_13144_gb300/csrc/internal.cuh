@@ -71,6 +71,34 @@ inline double c_screen(int dpad) {
 // below); radii used for acceptance divide by sigma * (1 + kSigmaSlack).
 constexpr double kSigmaSlack = 1e-9;
 
+// Constants of the probe thresholds of one entry (see thresholds()).
+struct ThreshConsts {
+  float om_eps_rd;   // 1 - eps_rc, rounded down
+  float inv_omg_ru;  // 1 / (1 - gamma_{d_pad/32+33}), rounded up
+  float om_c_rd;     // 1 - c_screen, rounded down
+};
+
+inline ThreshConsts thresh_consts(int dpad) {
+  ThreshConsts t;
+  t.om_eps_rd = std::nextafter((float)(1.0 - eps_recheck(dpad)), 0.0f);
+  t.inv_omg_ru = std::nextafter((float)(1.0 / (1.0 - gamma32(dpad / 32 + 33))), 2.0f);
+  t.om_c_rd = std::nextafter((float)(1.0 - c_screen(dpad)), 0.0f);
+  return t;
+}
+
+#ifdef __CUDACC__
+// Probe thresholds of an entry with radius lower bound r_lo (FP32, already
+// rounded down) and FP32 squared norm kn, every step rounded so that it can
+// only lower them: the recheck threshold rr <= r_lo^2 (1 - eps_rc) on the
+// canonical FP32 squared distance, and the screen term
+// tau <= ((1 - c_screen) kn - rr / (1 - gamma)) / 2.
+__device__ __forceinline__ void thresholds(float r_lo, float kn, const ThreshConsts& t, float& rr, float& tau) {
+  rr = __fmul_rd(__fmul_rd(r_lo, r_lo), t.om_eps_rd);
+  const float Rt = __fmul_ru(rr, t.inv_omg_ru);
+  tau = __fmul_rd(__fsub_rd(__fmul_rd(t.om_c_rd, kn), Rt), 0.5f);
+}
+#endif
+
 // ---------------------------------------------------------------- state
 struct SpecResult {
   double sigma;
@@ -176,6 +204,21 @@ struct lipcache {
 
   double eps_rc = 0.0, c_scr = 0.0;
   lc::EncodeTiledFn encode = nullptr;
+
+  // radius policy (Sec. 5.4): the probe reads rr_emp / tau_emp instead of
+  // the certified thresholds when policy != LIPCACHE_POLICY_CERTIFIED
+  int policy = LIPCACHE_POLICY_CERTIFIED;
+  double policy_param = 0.0;
+  float* rr_emp = nullptr;   // table_rows
+  float* tau_emp = nullptr;  // table_rows
+  float* rho32 = nullptr;    // C: per-class radius, rounded down
+  double* rho = nullptr;     // C: per-class radius (FP64)
+  double* cls_sum = nullptr;       // per-block class sums (policy scratch)
+  int64_t* cls_cnt = nullptr;      // per-block class counts
+  int64_t cls_blocks = 0;
+
+  const float* probe_rr() const { return policy ? rr_emp : table.rr; }
+  const float* probe_tau() const { return policy ? tau_emp : table.tau; }
 };
 
 namespace lc {
@@ -188,6 +231,11 @@ void spectral_norm(lipcache* h, cudaStream_t s);
 // acceptance to rows with miss_of[row] < 0 (write-back of probe misses).
 void certify_insert(lipcache* h, const float* H, int64_t n, const int32_t* payload, int require_consistency,
                     int64_t* out_index, float* out_radius, cudaStream_t s, const int64_t* miss_of = nullptr);
+// policy.cu: switch the probe's thresholds to an empirical radius policy
+// (or back to the certified ones); rho_host (nullable) receives C radii.
+void set_radius_policy(lipcache* h, int policy, double param, double* rho_host, cudaStream_t s);
+// thresholds of entries [first, first + n) under the current policy
+void policy_fill(lipcache* h, int64_t first, int64_t n, cudaStream_t s);
 // Certified-consistency check: argmax of the head on Q against y^G of the hit
 // entries; counts (hits, consistent, invalid index) land in ins_total[1..3].
 void consistency_check(lipcache* h, const float* Q, int64_t B, const int64_t* hit_index, int8_t* out,

@@ -194,7 +194,7 @@ void probe(lipcache* h, const float* Q, int64_t B, int64_t* out_index, int32_t* 
       dim3 grid((unsigned)((h->size + kEK - 1) / kEK), (unsigned)((B + kEQ - 1) / kEQ));
       h->last_grid = (int)(grid.x * grid.y);
       h->last_cluster = 1;
-      k_probe_exact<<<grid, 256, 0, s>>>(h->qpad, B, h->table.keys, h->table.rr, h->size, h->dpad, h->best);
+      k_probe_exact<<<grid, 256, 0, s>>>(h->qpad, B, h->table.keys, h->probe_rr(), h->size, h->dpad, h->best);
       LC_LAUNCH_CHECK("k_probe_exact");
     }
     if (slot >= 0) {
@@ -224,7 +224,7 @@ void probe_external_scratch(lipcache* h, const float* Q, int64_t B, int64_t* out
       launch_probe_tc_external(h, B, qpad, kappa, best, s);
     } else {
       dim3 grid((unsigned)((h->size + kEK - 1) / kEK), (unsigned)((B + kEQ - 1) / kEQ));
-      k_probe_exact<<<grid, 256, 0, s>>>(qpad, B, h->table.keys, h->table.rr, h->size, h->dpad, best);
+      k_probe_exact<<<grid, 256, 0, s>>>(qpad, B, h->table.keys, h->probe_rr(), h->size, h->dpad, best);
       LC_LAUNCH_CHECK("k_probe_exact");
     }
   }

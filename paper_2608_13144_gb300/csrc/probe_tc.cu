@@ -438,8 +438,8 @@ void launch(lipcache* h, int64_t B, const float* qpad, const float* kappa, unsig
   a.kappa = kappa;
   a.qpad = qpad;
   a.keys = h->table.keys;
-  a.tau = h->table.tau;
-  a.rr = h->table.rr;
+  a.tau = h->probe_tau();
+  a.rr = h->probe_rr();
   a.best = best;
   a.stats = h->stats;
   const Layout<BN> L{a.nch, a.nst};

@@ -8,6 +8,7 @@ from __future__ import annotations
 
 import ctypes as C
 
+import numpy as np
 import torch
 
 from . import _lib
@@ -15,6 +16,7 @@ from ._lib import Info, check
 
 RADIUS_MODES = {"conservative": _lib.RADIUS_CONSERVATIVE, "tight": _lib.RADIUS_TIGHT}
 PROBE_PATHS = {"auto": _lib.PROBE_AUTO, "tensor": _lib.PROBE_TENSOR, "exact": _lib.PROBE_EXACT}
+RADIUS_POLICIES = {"certified": 0, "global": 1, "interclass": 2}
 
 
 def _stream(device: torch.device):
@@ -167,6 +169,16 @@ class LipCache:
     # -- options / introspection
     def set_probe_path(self, path: str):
         check(self.L.lipcache_set_probe_path(self._h, PROBE_PATHS[path]))
+
+    def set_radius_policy(self, policy: str, param: float = 0.0):
+        """Switch the probe to the certified radius or to an empirical
+        boundary ("global": one threshold tau = param; "interclass": beta =
+        param times half the distance between class centroids). Returns the
+        C per-class radii as a numpy array."""
+        rho = np.zeros(self.C, dtype=np.float64)
+        check(self.L.lipcache_set_radius_policy(self._h, RADIUS_POLICIES[policy], float(param),
+                                                rho.ctypes.data, _stream(self.device)))
+        return rho
 
     def set_radius_scale(self, kappa: float):
         check(self.L.lipcache_set_radius_scale(self._h, float(kappa)))
