@@ -158,148 +158,169 @@ __device__ __forceinline__ bool pair_gt(float ah, float al, float bh, float bl) 
   return ah > bh || (ah == bh && al > bl);
 }
 
-// Certify the rows r = warp, warp + nwarps, ... < nrows of a tile with one
-// warp, conservative radius (Eq. 21). The FP32 intervals s~_c +- E_c
-// (E_c = gamma_{d+2} (||W_c|| ||z|| + |b_c|), widened for the rounding of the
-// interval arithmetic itself) select every class that can be among the true
-// top two; those are recomputed with dot2_logit. The true runner-up is among
-// them, so the margin is that of the full logit vector. All per-class work is
-// FP32; the few FP64 operations per row (margin and radius) run once for up
-// to 32 rows, one lane per row (FP64 runs at a small fraction of the FP32
-// rate on this GPU).
-// Row r: features hb[r * hrs + j * hs], logits lg[r * lstride + c];
-// W_cj = wmat[c * wcs + j * wjs]; norms / bias per class in wn32 / bias.
+// Per-row result of the candidate refinement: the best and second-best
+// refined logits (pairs hi + lo), the error bound of the best, the largest
+// upper bound v + e among the other candidates, ||z||^2 (FP32) and y^G.
+struct RowVals {
+  float h1, l1, e1, h2, l2, up, kn;
+  int y;
+};
+
+// Upper bound of ||z|| from the FP32 sum of squares kn (any order: within
+// gamma_d < 1e-4 of ||z||^2 for d <= 1024, plus d * 2^-150 for subnormal
+// squares).
+__device__ __forceinline__ float norm_upper(float kn) {
+  return __fmul_ru(__fsqrt_ru(__fmaf_ru(kn, 1.0f + 1e-4f, kTinyF)), 1.0f + 1e-6f);
+}
+
+// Bound of |hi + lo - s_c| for a refined logit, rounded up (plus the absolute
+// error of subnormal products).
+__device__ __forceinline__ float refined_err(float g2f, float wn, float hn, float b) {
+  return __fmaf_ru(g2f, __fmaf_ru(wn, hn, fabsf(b)), kTinyF);
+}
+
+// Running selection over refined candidates, visited in any order: the best
+// by (value desc, class asc), the second-best value, and the top two upper
+// bounds with the class of the first, so that the largest upper bound among
+// the classes other than the best is available at the end.
+struct Top2 {
+  float b1h = -INFINITY, b1l = 0.f, b2h = -INFINITY, b2l = 0.f, e1 = 0.f;
+  float u1 = -INFINITY, u2 = -INFINITY;
+  int y = -1, cu1 = -1;
+  bool nan = false;  // a refined logit is NaN: the row is rejected
+  __device__ __forceinline__ void push(int c, float vh, float vl, float e) {
+    nan |= !(vh == vh && vl == vl);
+    const bool eq1 = vh == b1h && vl == b1l;
+    if (pair_gt(vh, vl, b1h, b1l) || (eq1 && c < y)) {
+      b2h = b1h;
+      b2l = b1l;
+      b1h = vh;
+      b1l = vl;
+      e1 = e;
+      y = c;
+    } else if (pair_gt(vh, vl, b2h, b2l) || (vh == b2h && vl == b2l)) {
+      b2h = vh;
+      b2l = vl;
+    }
+    const float up = __fadd_ru(vh, __fadd_ru(vl, e));
+    if (up > u1) {
+      u2 = u1;
+      u1 = up;
+      cu1 = c;
+    } else if (up > u2) {
+      u2 = up;
+    }
+  }
+  __device__ __forceinline__ RowVals result(float kn) const {
+    RowVals v;
+    v.h1 = nan ? NAN : b1h;
+    v.l1 = b1l;
+    v.e1 = e1;
+    v.h2 = b2h;
+    v.l2 = b2l;
+    v.up = (cu1 == y) ? u2 : u1;
+    v.kn = kn;
+    v.y = y < 0 ? 0 : y;  // every refined logit NaN: the margin is NaN and the row is rejected
+    return v;
+  }
+};
+
+// FP64 margin, radius, certified lower bound and probe thresholds of one row
+// (one thread), and the skip rules of Algorithm 1.
+__device__ void row_finals(const CertArgs& a, int64_t row, const RowVals& v, uint8_t* acc_slot) {
+  const double v1 = (double)v.h1 + (double)v.l1, v2 = (double)v.h2 + (double)v.l2;
+  const double mval = (v1 == v1 && v2 == v2) ? v1 - v2 : NAN;
+  // lower bound of the exact margin with downward rounding
+  const double mlo = __dsub_rd(__dsub_rd(v1, (double)v.e1), (double)v.up);
+  const double r64 = mval * a.inv_denom;
+  const double rs = (mlo > 0.0) ? __dmul_rd(mlo, a.inv_denom_safe) : 0.0;
+  const int32_t lab = a.payload ? a.payload[row] : v.y;
+  const bool acc = !(a.require_consistency && lab != v.y) && (r64 > 0.0) && !(a.miss_of && a.miss_of[row] >= 0);
+  float rr, tau;
+  thresholds(__double2float_rd(rs), v.kn, a.tc, rr, tau);
+  a.accept[row] = acc ? 1 : 0;
+  a.yG[row] = v.y;
+  a.label[row] = lab;
+  a.radius[row] = __double2float_rz(r64);
+  a.rr[row] = rr;
+  a.kn[row] = v.kn;
+  a.tau[row] = tau;
+  *acc_slot = acc ? 1 : 0;
+}
+
+// One row with one warp, conservative radius (Eq. 21): the FP32 intervals
+// s~_c +- E_c select every class that can be among the true top two; those
+// are recomputed with dot2_logit. The true runner-up is among them, so the
+// margin is that of the full logit vector. Row: features hrow[j * hs], FP32
+// logits lrow[c]; W_cj = wmat[c * wcs + j * wjs]; per-class norms / biases in
+// wn32 / bias. Every lane returns the same values.
+__device__ RowVals warp_row_refine(const CertArgs& a, const float* __restrict__ hrow, int hs,
+                                   const float* __restrict__ lrow, const float* __restrict__ wmat, int wcs, int wjs,
+                                   const float* __restrict__ wn32, const float* __restrict__ bias, int lane) {
+  const int d = a.d, C = a.C;
+  float knp = 0.f;
+  for (int j = lane; j < d; j += 32) {
+    const float x = hrow[(size_t)j * hs];
+    knp = fmaf(x, x, knp);
+  }
+  const float kn = warp_sum_f(knp);
+  const float hn = norm_upper(kn);
+  float l1 = -INFINITY, l2 = -INFINITY;
+  for (int c = lane; c < C; c += 32) {
+    const float sv = lrow[c];
+    float lo = __fsub_rd(sv, logit_err(a.g32f, wn32[c], hn, bias[c], sv));
+    lo = (lo == lo) ? lo : -INFINITY;  // a NaN logit is no candidate for the top two
+    l2 = fmaxf(l2, fminf(l1, lo));
+    l1 = fmaxf(l1, lo);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float o1 = __shfl_xor_sync(kFull, l1, o), o2 = __shfl_xor_sync(kFull, l2, o);
+    l2 = fmaxf(l2, fminf(l1, o1));
+    l1 = fmaxf(l1, o1);
+    l2 = fmaxf(l2, fminf(l1, o2));
+    l1 = fmaxf(l1, o2);
+  }
+  const float L2 = l2;
+  Top2 t;
+  for (int cb = 0; cb < C; cb += 32) {
+    const int c = cb + lane;
+    bool cand = false;
+    if (c < C) {
+      const float sv = lrow[c];
+      cand = __fadd_ru(sv, logit_err(a.g32f, wn32[c], hn, bias[c], sv)) >= L2;
+    }
+    unsigned m = __ballot_sync(kFull, cand);
+    while (m) {
+      const int cc = cb + __ffs(m) - 1;
+      m &= m - 1;
+      const float bc = bias[cc];
+      float vh, vl;
+      dot2_logit(wmat + (size_t)cc * wcs, wjs, hrow, hs, bc, d, lane, vh, vl);
+      t.push(cc, vh, vl, refined_err(a.g2f, wn32[cc], hn, bc));
+    }
+  }
+  return t.result(kn);
+}
+
+// Rows r = warp, warp + nwarps, ... < nrows of a tile, one warp each; the
+// FP64 finals of up to 32 rows run once, one lane per row (FP64 runs at a
+// small fraction of the FP32 rate on this GPU).
+// Row r: features hb[r * hrs + j * hs], logits lg[r * lstride + c].
 __device__ void certify_rows_fast(const CertArgs& a, int64_t row0, int nrows, int warp, int nwarps,
                                   const float* __restrict__ hb, int hrs, int hs, const float* __restrict__ wmat,
                                   int wcs, int wjs, const float* __restrict__ lg, const float* __restrict__ wn32,
                                   const float* __restrict__ bias, int lane, uint8_t* acc_flag) {
-  const int d = a.d, C = a.C;
-  // per-row results parked in lane k (the warp's k-th row)
-  float r_h1 = 0.f, r_l1 = 0.f, r_e1 = 0.f, r_h2 = 0.f, r_l2 = 0.f, r_up = 0.f, r_kn = 0.f;
-  int r_y = 0, k = 0;
+  RowVals mine{};
+  int k = 0;
   for (int r = warp; r < nrows; r += nwarps, ++k) {
-    const float* hrow = hb + (size_t)r * hrs;
-    const float* lrow = lg + (size_t)r * a.lstride;
-    float knp = 0.f;
-    for (int j = lane; j < d; j += 32) {
-      const float x = hrow[(size_t)j * hs];
-      knp = fmaf(x, x, knp);
-    }
-    const float kn = warp_sum_f(knp);
-    // upper bound of ||z||: kn is within gamma_{d/32+5} < 1e-5 of ||z||^2, up
-    // to d * 2^-150 lost where the squares are subnormal
-    const float hn = __fmul_ru(__fsqrt_ru(__fmaf_ru(kn, 1.0f + 1e-5f, kTinyF)), 1.0f + 1e-6f);
-
-    float l1 = -INFINITY, l2 = -INFINITY;
-    for (int c = lane; c < C; c += 32) {
-      const float sv = lrow[c];
-      const float E = logit_err(a.g32f, wn32[c], hn, bias[c], sv);
-      const float lo = __fsub_rd(sv, E);
-      if (lo > l1) {
-        l2 = l1;
-        l1 = lo;
-      } else if (lo > l2) {
-        l2 = lo;
-      }
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      const float o1 = __shfl_xor_sync(kFull, l1, o), o2 = __shfl_xor_sync(kFull, l2, o);
-      float t1 = l1, t2 = l2;
-      if (o1 > t1) {
-        t2 = t1;
-        t1 = o1;
-      } else if (o1 > t2) {
-        t2 = o1;
-      }
-      if (o2 > t1) {
-        t2 = t1;
-        t1 = o2;
-      } else if (o2 > t2) {
-        t2 = o2;
-      }
-      l1 = t1;
-      l2 = t2;
-    }
-    const float L2 = l2;
-
-    // refine the candidates in ascending class order (strict comparisons keep
-    // the lowest class on ties)
-    float b1h = -INFINITY, b1l = 0.f, b2h = -INFINITY, b2l = 0.f, e1 = 0.f;
-    float u1 = -INFINITY, u2 = -INFINITY;  // top two upper bounds v + e ...
-    int y = -1, cu1 = -1;                  // ... and the class of the first
-    for (int cb = 0; cb < C; cb += 32) {
-      const int c = cb + lane;
-      bool cand = false;
-      if (c < C) {
-        const float sv = lrow[c];
-        const float E = logit_err(a.g32f, wn32[c], hn, bias[c], sv);
-        cand = (__fadd_ru(sv, E) >= L2) || !(L2 == L2);
-      }
-      unsigned m = __ballot_sync(kFull, cand);
-      while (m) {
-        const int cc = cb + __ffs(m) - 1;
-        m &= m - 1;
-        const float bc = bias[cc];
-        float vh, vl;
-        dot2_logit(wmat + (size_t)cc * wcs, wjs, hrow, hs, bc, d, lane, vh, vl);
-        // bound of |hi + lo - exact|, rounded up (plus the absolute error of
-        // subnormal products)
-        const float e = __fmaf_ru(a.g2f, __fmaf_ru(wn32[cc], hn, fabsf(bc)), kTinyF);
-        if (pair_gt(vh, vl, b1h, b1l)) {
-          b2h = b1h;
-          b2l = b1l;
-          b1h = vh;
-          b1l = vl;
-          e1 = e;
-          y = cc;
-        } else if (pair_gt(vh, vl, b2h, b2l)) {
-          b2h = vh;
-          b2l = vl;
-        }
-        const float up = __fadd_ru(vh, __fadd_ru(vl, e));
-        if (up > u1) {
-          u2 = u1;
-          u1 = up;
-          cu1 = cc;
-        } else if (up > u2) {
-          u2 = up;
-        }
-      }
-    }
-    if (lane == k) {
-      r_h1 = b1h;
-      r_l1 = b1l;
-      r_e1 = e1;
-      r_h2 = b2h;
-      r_l2 = b2l;
-      r_up = (cu1 == y) ? u2 : u1;
-      r_y = y < 0 ? 0 : y;  // every refined logit NaN: the margin is NaN and the row is rejected
-      r_kn = kn;
-    }
+    const RowVals v = warp_row_refine(a, hb + (size_t)r * hrs, hs, lg + (size_t)r * a.lstride, wmat, wcs, wjs,
+                                      wn32, bias, lane);
+    if (lane == k) mine = v;
   }
-  // FP64 margin and radius, one lane per row
   if (lane < k) {
     const int r = warp + lane * nwarps;
-    const int64_t row = row0 + r;
-    const double v1 = (double)r_h1 + (double)r_l1, v2 = (double)r_h2 + (double)r_l2;
-    const double mval = (v1 == v1 && v2 == v2) ? v1 - v2 : NAN;
-    // lower bound of the exact margin with downward rounding
-    const double mlo = __dsub_rd(__dsub_rd(v1, (double)r_e1), (double)r_up);
-    const double r64 = mval * a.inv_denom;
-    const double rs = (mlo > 0.0) ? __dmul_rd(mlo, a.inv_denom_safe) : 0.0;
-    const int32_t lab = a.payload ? a.payload[row] : r_y;
-    const bool acc = !(a.require_consistency && lab != r_y) && (r64 > 0.0) && !(a.miss_of && a.miss_of[row] >= 0);
-    float rr, tau;
-    thresholds(__double2float_rd(rs), r_kn, a.tc, rr, tau);
-    a.accept[row] = acc ? 1 : 0;
-    a.yG[row] = r_y;
-    a.label[row] = lab;
-    a.radius[row] = __double2float_rz(r64);
-    a.rr[row] = rr;
-    a.kn[row] = r_kn;
-    a.tau[row] = tau;
-    acc_flag[r] = acc ? 1 : 0;
+    row_finals(a, row0 + r, mine, &acc_flag[r]);
   }
   __syncwarp();
 }
@@ -496,25 +517,94 @@ __global__ void __launch_bounds__(kThreads) k_certify(CertArgs a) {
 }
 
 // Certified insertion with the head resident in shared memory (C <= 256 and
-// W^T fits): persistent CTAs, tiles of 64 rows. The FP32 logits are a
-// register-tiled product: each thread accumulates 8 rows x 8 classes, reading
-// 8 features and 8 weights per k with four 128-bit shared loads, one FMA
-// chain per (row, class) in k order (the same error bound as above).
-constexpr int kWTile = 64;   // rows per tile
-constexpr int kHStride = 68; // h^T row stride (floats): 16-byte aligned, banks spread
+// W^T fits): persistent CTAs, tiles of 64 rows.
+//  1. The tile's features are transposed into shared memory (h^T).
+//  2. FP32 logits by a register-tiled product: each thread accumulates 8 rows
+//     x 8 classes, reading 8 features and 8 weights per k with four 128-bit
+//     shared loads, one FMA chain per (row, class) in k order (the error
+//     bound E_c holds for it).
+//  3. Conservative radius: thread (r, q) owns row r and a quarter q of the
+//     classes. It forms a quarter of ||z||^2, then the top two interval lower
+//     ends of its classes; the row's second-largest lower end L2 decides the
+//     candidates (upper end >= L2), which go to a per-row slot list and a
+//     compact pair list. Groups of 8 lanes refine one (row, class) pair each
+//     with the compensated dot product, and one thread per row selects y^G,
+//     the runner-up and the bounds from its slots (in any order, ties to the
+//     lowest class) and runs the FP64 finals. A row with more than
+//     kMaxCand candidates is redone by one warp with warp_row_refine.
+//     The tight radius runs certify_row (FP64) with one warp per row.
+constexpr int kWTile = 64;    // rows per tile
+constexpr int kHStride = 68;  // h^T row stride (floats): 16-byte aligned, banks spread
+constexpr int kMaxCand = 16;  // candidate slots per row
+constexpr int kGroup = 8;     // lanes per refined pair
 
-__global__ void __launch_bounds__(kThreads, 1) k_certify_wres(CertArgs a, int Cp, int dpad, int n_tiles) {
+struct TileSmem {
+  float knp[4][kWTile];     // quarter sums of ||z||^2
+  float2 top[4][kWTile];    // per-quarter top two interval lower ends
+  float hn[kWTile];         // upper bound of ||z||
+  float kn[kWTile];         // ||z||^2 (FP32)
+  int ncand[kWTile];        // candidates per row
+  int cls[kWTile][kMaxCand];
+  float rh[kWTile][kMaxCand], rl[kWTile][kMaxCand], re[kWTile][kMaxCand];
+  int pairs[kWTile * kMaxCand];  // r | slot << 8 | class << 16
+  int npairs, novf;
+  int ovf[kWTile];
+  uint8_t acc_flag[kWTile];
+};
+
+// Transposed copy of rows [row0, row0 + nrows) of H (zero past d and nrows)
+// into hT[k * kHStride + r]. With 16-byte rows each lane loads float4s of
+// its own row and stores four conflict-free scalars (lanes = rows).
+__device__ __forceinline__ void load_tile(const CertArgs& a, int64_t row0, int nrows, int dpad, float* hT, int tid,
+                                          bool vec) {
+  const int d = a.d;
+  if (vec) {
+    const int warp = tid >> 5, lane = tid & 31;
+    const int r = (warp & 1) * 32 + lane;
+    const bool live = r < nrows;
+    const float4* src = reinterpret_cast<const float4*>(a.H + (size_t)(row0 + (live ? r : 0)) * d);
+    constexpr int kB = 8;
+    for (int k40 = warp >> 1; k40 < dpad / 4; k40 += 4 * kB) {
+      float4 v[kB];
+#pragma unroll
+      for (int u = 0; u < kB; ++u) {
+        const int k4 = k40 + 4 * u;
+        v[u] = (live && 4 * k4 < d) ? __ldg(src + k4) : make_float4(0.f, 0.f, 0.f, 0.f);
+      }
+#pragma unroll
+      for (int u = 0; u < kB; ++u) {
+        const int k4 = k40 + 4 * u;
+        if (k4 < dpad / 4) {
+          float* dst = hT + (size_t)(4 * k4) * kHStride + r;
+          dst[0] = v[u].x;
+          dst[kHStride] = v[u].y;
+          dst[2 * kHStride] = v[u].z;
+          dst[3 * kHStride] = v[u].w;
+        }
+      }
+    }
+  } else {
+    for (int idx = tid; idx < kWTile * dpad; idx += kThreads) {
+      const int r = idx / dpad, k = idx - r * dpad;
+      hT[k * kHStride + r] = (r < nrows && k < d) ? __ldg(a.H + (size_t)(row0 + r) * d + k) : 0.f;
+    }
+  }
+}
+
+__global__ void __launch_bounds__(kThreads, 1) k_certify_wres(CertArgs a, int Cp, int dpad, int n_tiles, int vec) {
   extern __shared__ __align__(16) unsigned char smem[];
   float* wT = reinterpret_cast<float*>(smem);           // dpad x Cp (W transposed, zero padded)
   float* hT = wT + (size_t)dpad * Cp;                   // dpad x kHStride (tile rows transposed)
   float* lg = hT + (size_t)dpad * kHStride;             // kWTile x lstride FP32 logits
+  float* wn_s = lg + (size_t)kWTile * a.lstride;        // C norms (rounded up)
+  float* b_s = wn_s + a.C;                              // C biases
+  float* eA = b_s + a.C;                                // C: g32f ||W_c||, rounded up
+  float* eB = eA + a.C;                                 // C: g32f |b_c| + tiny, rounded up
   // FP64 scratch for the tight radius only
   const int sC = a.tight ? a.C : 0;
-  double* s64 = reinterpret_cast<double*>(lg + (size_t)kWTile * a.lstride + ((kWTile * a.lstride) & 1));
+  double* s64 = reinterpret_cast<double*>(eB + a.C + ((4 * a.C + kWTile * a.lstride) & 1));
   double* e64 = s64 + (size_t)kWarps * sC;
-  float* wn_s = reinterpret_cast<float*>(e64 + (size_t)kWarps * sC);  // C norms (rounded up)
-  float* b_s = wn_s + a.C;                                              // C biases
-  __shared__ uint8_t acc_flag[kWTile];
+  TileSmem& ts = *reinterpret_cast<TileSmem*>(e64 + (size_t)kWarps * sC);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int d = a.d, C = a.C;
@@ -523,38 +613,33 @@ __global__ void __launch_bounds__(kThreads, 1) k_certify_wres(CertArgs a, int Cp
     wT[idx] = (c < C && k < d) ? __ldg(a.W + (size_t)c * d + k) : 0.f;
   }
   for (int c = tid; c < C; c += kThreads) {
-    wn_s[c] = __ldg(a.Wnorm32 + c);
-    b_s[c] = __ldg(a.b + c);
+    const float wn = __ldg(a.Wnorm32 + c), bc = __ldg(a.b + c);
+    wn_s[c] = wn;
+    b_s[c] = bc;
+    eA[c] = __fmul_ru(a.g32f, wn);
+    eB[c] = __fmaf_ru(a.g32f, fabsf(bc), kTinyF);
   }
   const int rg = tid & 7, cg = tid >> 3;  // rows {4rg..4rg+3, 32+4rg..32+4rg+3}, classes 8cg..8cg+7
   const bool mine = cg * 8 < Cp;
   double* ws = s64 + (size_t)warp * sC;
   double* we = e64 + (size_t)warp * sC;
+  const int r3 = tid & (kWTile - 1), q3 = tid >> 6;  // phase 3: row, class quarter
+  const int cq = (C + 3) / 4, c_lo = q3 * cq, c_hi = min(C, c_lo + cq);
+  const int dq = (d + 3) / 4, k_lo = q3 * dq, k_hi = min(d, k_lo + dq);
 
   for (int tile = blockIdx.x; tile < n_tiles; tile += gridDim.x) {
     const int64_t row0 = (int64_t)tile * kWTile;
     const int nrows = (int)(a.n - row0 < kWTile ? a.n - row0 : kWTile);
-    // the tile's features: all loads of a thread issued before its stores
-    constexpr int kBatch = 16;
-    float buf[kBatch];
-    for (int base = 0; base < kWTile * dpad; base += kThreads * kBatch) {
-#pragma unroll
-      for (int i = 0; i < kBatch; ++i) {
-        const int idx = base + i * kThreads + tid;
-        const int r = idx / dpad, k = idx - r * dpad;
-        buf[i] = (idx < kWTile * dpad && r < nrows && k < d) ? __ldg(a.H + (size_t)(row0 + r) * d + k) : 0.f;
-      }
-      if (base == 0) __syncthreads();  // previous tile done with hT / lg (and wT written on the first pass)
-#pragma unroll
-      for (int i = 0; i < kBatch; ++i) {
-        const int idx = base + i * kThreads + tid;
-        if (idx < kWTile * dpad) {
-          const int r = idx / dpad, k = idx - r * dpad;
-          hT[k * kHStride + r] = buf[i];
-        }
-      }
+    __syncthreads();  // previous tile done with hT / lg / ts (and wT written on the first pass)
+    load_tile(a, row0, nrows, dpad, hT, tid, vec != 0);
+    if (tid < kWTile) {
+      ts.acc_flag[tid] = 0;
+      ts.ncand[tid] = 0;
     }
-    if (tid < kWTile) acc_flag[tid] = 0;
+    if (tid == 0) {
+      ts.npairs = 0;
+      ts.novf = 0;
+    }
     __syncthreads();
     if (mine) {
       float acc[8][8];
@@ -583,22 +668,125 @@ __global__ void __launch_bounds__(kThreads, 1) k_certify_wres(CertArgs a, int Cp
 #pragma unroll
         for (int j = 0; j < 8; ++j) {
           const int c = cg * 8 + j;
-          if (c < C) lg[r * a.lstride + c] = acc[i][j] + __ldg(a.b + c);
+          if (c < C) lg[r * a.lstride + c] = acc[i][j] + b_s[c];
         }
       }
     }
-    __syncthreads();
     if (a.tight) {
+      __syncthreads();
       for (int r = warp; r < nrows; r += kWarps)
-        certify_row(a, row0 + r, a.H + (size_t)(row0 + r) * d, lg + r * a.lstride, ws, we, lane, &acc_flag[r]);
+        certify_row(a, row0 + r, a.H + (size_t)(row0 + r) * d, lg + r * a.lstride, ws, we, lane, &ts.acc_flag[r]);
     } else {
-      certify_rows_fast(a, row0, nrows, warp, kWarps, hT, 1, kHStride, wT, 1, Cp, lg, wn_s, b_s, lane, acc_flag);
+      // quarter of ||z||^2 (independent of the logits)
+      {
+        float p = 0.f;
+        for (int k = k_lo; k < k_hi; ++k) {
+          const float x = hT[k * kHStride + r3];
+          p = fmaf(x, x, p);
+        }
+        ts.knp[q3][r3] = p;
+      }
+      __syncthreads();
+      const float kn = (ts.knp[0][r3] + ts.knp[1][r3]) + (ts.knp[2][r3] + ts.knp[3][r3]);
+      const float hn = norm_upper(kn);
+      if (q3 == 0) {
+        ts.kn[r3] = kn;
+        ts.hn[r3] = hn;
+      }
+      const float* lrow = lg + (size_t)r3 * a.lstride;
+      float l1 = -INFINITY, l2 = -INFINITY;
+      for (int c = c_lo; c < c_hi; ++c) {
+        const float sv = lrow[c];
+        const float E = __fmaf_ru(eA[c], hn, __fmaf_ru(fabsf(sv), 2.3841858e-07f /* 2^-22 */, eB[c]));
+        float lo = __fsub_rd(sv, E);
+        lo = (lo == lo) ? lo : -INFINITY;
+        l2 = fmaxf(l2, fminf(l1, lo));
+        l1 = fmaxf(l1, lo);
+      }
+      ts.top[q3][r3] = make_float2(l1, l2);
+      __syncthreads();
+      float L1 = -INFINITY, L2 = -INFINITY;
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const float2 t = ts.top[q][r3];
+        L2 = fmaxf(L2, fminf(L1, t.x));
+        L1 = fmaxf(L1, t.x);
+        L2 = fmaxf(L2, fminf(L1, t.y));
+        L1 = fmaxf(L1, t.y);
+      }
+      if (r3 < nrows) {
+        for (int c = c_lo; c < c_hi; ++c) {
+          const float sv = lrow[c];
+          const float E = __fmaf_ru(eA[c], hn, __fmaf_ru(fabsf(sv), 2.3841858e-07f, eB[c]));
+          if (__fadd_ru(sv, E) >= L2) {
+            const int slot = atomicAdd(&ts.ncand[r3], 1);
+            if (slot < kMaxCand) {
+              ts.cls[r3][slot] = c;
+              ts.pairs[atomicAdd(&ts.npairs, 1)] = r3 | (slot << 8) | (c << 16);
+            }
+          }
+        }
+      }
+      __syncthreads();
+      // refine the pairs, kGroup lanes each
+      {
+        const int g = tid / kGroup, sub = tid % kGroup;
+        const int np = ts.npairs;
+        for (int base = 0; base < np; base += kThreads / kGroup) {
+          const int pi = base + g;
+          const int pk = ts.pairs[pi < np ? pi : 0];
+          const int r = pk & 0xff, slot = (pk >> 8) & 0xff, c = pk >> 16;
+          float p = 0.f, cc = 0.f;
+          for (int k = sub; k < d; k += kGroup) {
+            const float w = wT[(size_t)k * Cp + c], x = hT[k * kHStride + r];
+            const float pr = __fmul_rn(w, x);
+            const float er = __fmaf_rn(w, x, -pr);
+            float t, q;
+            two_sum(p, pr, t, q);
+            p = t;
+            cc = __fadd_rn(cc, __fadd_rn(q, er));
+          }
+#pragma unroll
+          for (int o = kGroup / 2; o > 0; o >>= 1) {
+            const float pb = __shfl_xor_sync(kFull, p, o), cb = __shfl_xor_sync(kFull, cc, o);
+            float t, q;
+            two_sum(p, pb, t, q);
+            p = t;
+            cc = __fadd_rn(__fadd_rn(cc, cb), q);
+          }
+          if (pi < np && sub == 0) {
+            float t, q, hi, lo;
+            two_sum(p, b_s[c], t, q);
+            two_sum(t, __fadd_rn(cc, q), hi, lo);
+            ts.rh[r][slot] = hi;
+            ts.rl[r][slot] = lo;
+            ts.re[r][slot] = refined_err(a.g2f, wn_s[c], ts.hn[r], b_s[c]);
+          }
+        }
+      }
+      __syncthreads();
+      if (tid < nrows) {
+        const int r = tid, n = ts.ncand[r];
+        if (n > kMaxCand) {
+          ts.ovf[atomicAdd(&ts.novf, 1)] = r;
+        } else {
+          Top2 t;
+          for (int sl = 0; sl < n; ++sl) t.push(ts.cls[r][sl], ts.rh[r][sl], ts.rl[r][sl], ts.re[r][sl]);
+          row_finals(a, row0 + r, t.result(ts.kn[r]), &ts.acc_flag[r]);
+        }
+      }
+      __syncthreads();
+      for (int i = warp; i < ts.novf; i += kWarps) {
+        const int r = ts.ovf[i];
+        const RowVals v = warp_row_refine(a, hT + r, kHStride, lg + (size_t)r * a.lstride, wT, 1, Cp, wn_s, b_s, lane);
+        if (lane == 0) row_finals(a, row0 + r, v, &ts.acc_flag[r]);
+      }
     }
     __syncthreads();
     if (warp < 2 && row0 + warp * 32 < a.n) {
       const int sub = warp * 32;
       const int nsub = nrows - sub < 32 ? nrows - sub : 32;
-      const bool f = lane < nsub && acc_flag[sub + lane];
+      const bool f = lane < nsub && ts.acc_flag[sub + lane];
       const unsigned m = __ballot_sync(kFull, f);
       if (lane < nsub) a.rank[row0 + sub + lane] = __popc(m & ((1u << lane) - 1u));
       if (lane == 0) a.bcount[(row0 + sub) / 32] = __popc(m);
@@ -793,13 +981,14 @@ void launch_certify(lipcache* h, const float* H, int64_t n, const int32_t* paylo
   const int nb = (int)((n + kRows - 1) / kRows);
   const int Cp = (h->C + 7) / 8 * 8;
   const size_t smem_wres = sizeof(float) * ((size_t)h->dpad * Cp + (size_t)h->dpad * kHStride +
-                                            (size_t)kWTile * a.lstride + 1 + 2 * (size_t)h->C) +
-                           sizeof(double) * 2 * kWarps * (size_t)(a.tight ? h->C : 0);
+                                            (size_t)kWTile * a.lstride + 1 + 4 * (size_t)h->C) +
+                           sizeof(double) * 2 * kWarps * (size_t)(a.tight ? h->C : 0) + sizeof(TileSmem);
   if (h->C <= 256 && smem_wres <= 220 * 1024) {
     const int n_tiles = (int)((n + kWTile - 1) / kWTile);
     const int grid = n_tiles < h->num_sms ? n_tiles : h->num_sms;
     LC_CUDA(cudaFuncSetAttribute(k_certify_wres, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_wres));
-    k_certify_wres<<<grid, kThreads, smem_wres, s>>>(a, Cp, h->dpad, n_tiles);
+    const int vec = (h->d % 4 == 0 && ((uintptr_t)H & 15) == 0) ? 1 : 0;
+    k_certify_wres<<<grid, kThreads, smem_wres, s>>>(a, Cp, h->dpad, n_tiles, vec);
     LC_LAUNCH_CHECK("k_certify_wres");
   } else {
     const size_t smem = certify_smem_bytes(h->d, h->C);

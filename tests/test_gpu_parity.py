@@ -211,7 +211,7 @@ def built(dev):
 def test_insert_parity(built, name):
     s = built(name)
     assert abs(s["sigma"] - s["s_ref"]) <= 1e-10 * s["s_ref"]
-    check_insert(s["g_index"], s["g_radius"], s["n_acc"], s["ref"])
+    check_insert(s["g_index"], s["g_radius"], s["n_acc"], s["ref"], (s["W"], s["b"], s["rows"], 1.0))
 
 
 @pytest.mark.parametrize("path", PATHS)
@@ -253,7 +253,7 @@ def test_radius_scale(dev):
     cache, sigma = make_cache(dev, W, b, w.N, kappa=0.5)
     idx, rad, n = cache.insert(T(rows, dev))
     ref = oracle.build_cache(W, b, oracle.sigma_max(W), rows, scale=0.5)
-    check_insert(idx.cpu().numpy(), rad.cpu().numpy(), n, ref)
+    check_insert(idx.cpu().numpy(), rad.cpu().numpy(), n, ref, (W, b, rows, 0.5))
     orc = oracle.probe(ref["keys"], ref["radius"], ref["label"], Q)
     for path in PATHS:
         gi, gl, gd = run_probe(cache, Q, dev, w.batch, path)
@@ -304,7 +304,7 @@ def test_ragged_shapes(dev, path, d, C, N, B):
     cache, sigma = make_cache(dev, W, b, N + 5)
     idx, rad, n = cache.insert(T(rows, dev))
     ref = oracle.build_cache(W, b, oracle.sigma_max(W), rows)
-    check_insert(idx.cpu().numpy(), rad.cpu().numpy(), n, ref)
+    check_insert(idx.cpu().numpy(), rad.cpu().numpy(), n, ref, (W, b, rows, 1.0))
     orc = oracle.probe(ref["keys"], ref["radius"], ref["label"], Q)
     gi, gl, gd = run_probe(cache, Q, dev, 64, path)
     check_probe(gi, gl, gd, ref, Q, orc)
@@ -343,4 +343,31 @@ def test_probe_host_matches_device(dev, path):
     b2 = [t.numpy() for t in cache.probe_host(hq)]
     for x, y in zip(a, b2):
         assert np.array_equal(x, y)
+    cache.close()
+
+
+@pytest.mark.parametrize("mode", ["conservative", "tight"])
+def test_many_tied_runners_up(dev, mode):
+    """19 identical head rows: every row has at least 19 classes whose FP32
+    intervals overlap (more than the insert kernel's per-row candidate
+    slots), so the whole-warp fallback decides them. Rows whose best class
+    is unique keep an exact margin; rows won by the tied group are skipped
+    (m = 0) on both sides."""
+    rng = np.random.default_rng(21)
+    d, C = 32, 24
+    W = (rng.standard_normal((C, d)) / np.sqrt(d)).astype(np.float32)
+    W[1:20] = W[1]
+    b = (0.1 * rng.standard_normal(C)).astype(np.float32)
+    b[1:20] = b[1]
+    rows = np.concatenate([3 * W[0] + 0.3 * rng.standard_normal((150, d)),
+                           3 * W[1] + 0.3 * rng.standard_normal((150, d)),
+                           rng.standard_normal((100, d))]).astype(np.float32)
+    ref = oracle.build_cache(W, b, oracle.sigma_max(W), rows, radius_mode=int(mode == "tight"))
+    cache, _ = make_cache(dev, W, b, len(rows), mode)
+    idx, rad, n = cache.insert(T(rows, dev))
+    check_insert(idx.cpu().numpy(), rad.cpu().numpy(), n, ref, None if mode == "tight" else (W, b, rows, 1.0))
+    assert n > 100
+    if mode == "conservative":
+        assert n < len(rows)  # rows won by the tied group are skipped
+    # (the tight radius skips classes with W_j = W_y, Eq. 29, so it keeps them)
     cache.close()

@@ -116,7 +116,7 @@ def test_writeback_workload(dev, name, path):
     ref = oracle.build_cache(W, b, sigma, rows)
     cache, _ = make_cache(dev, W, b, len(rows) + len(Q), path)
     gidx, grad, nacc = cache.insert(T(rows, dev))
-    check_insert(gidx.cpu().numpy(), grad.cpu().numpy(), nacc, ref)
+    check_insert(gidx.cpu().numpy(), grad.cpu().numpy(), nacc, ref, (W, b, rows, 1.0))
     cur = {k: ref[k] for k in ("keys", "radius", "label", "yG")}
     total_ins = 0
     for s, e in synth.batches(len(Q), w.batch):
