@@ -32,6 +32,7 @@
 // product (k_certify_wres); otherwise each CTA streams W from L2 (k_certify).
 // Insertion order is kept by a block-count scan and a scatter.
 #include "internal.cuh"
+#include "tc_ptx.cuh"
 
 namespace lc {
 namespace {
@@ -642,25 +643,30 @@ __global__ void __launch_bounds__(kThreads, 1) k_certify_wres(CertArgs a, int Cp
     }
     __syncthreads();
     if (mine) {
-      float acc[8][8];
+      // accumulators in pairs of classes (2j, 2j+1): one packed FP32x2 FMA
+      // (each half an IEEE fma, round to nearest) per row and class pair
+      uint64_t acc[8][4];
 #pragma unroll
       for (int i = 0; i < 8; ++i)
 #pragma unroll
-        for (int j = 0; j < 8; ++j) acc[i][j] = 0.f;
+        for (int j = 0; j < 4; ++j) acc[i][j] = 0ull;
       const float* hp = hT + rg * 4;
       const float* wp = wT + cg * 8;
 #pragma unroll 4
       for (int k = 0; k < dpad; ++k) {
         const float4 h0 = *reinterpret_cast<const float4*>(hp + k * kHStride);
         const float4 h1 = *reinterpret_cast<const float4*>(hp + k * kHStride + 32);
-        const float4 w0 = *reinterpret_cast<const float4*>(wp + (size_t)k * Cp);
-        const float4 w1 = *reinterpret_cast<const float4*>(wp + (size_t)k * Cp + 4);
+        const ulonglong2 w0 = *reinterpret_cast<const ulonglong2*>(wp + (size_t)k * Cp);
+        const ulonglong2 w1 = *reinterpret_cast<const ulonglong2*>(wp + (size_t)k * Cp + 4);
         const float hv[8] = {h0.x, h0.y, h0.z, h0.w, h1.x, h1.y, h1.z, h1.w};
-        const float wv[8] = {w0.x, w0.y, w0.z, w0.w, w1.x, w1.y, w1.z, w1.w};
+        const uint64_t wv[4] = {w0.x, w0.y, w1.x, w1.y};
 #pragma unroll
-        for (int i = 0; i < 8; ++i)
+        for (int i = 0; i < 8; ++i) {
+          const uint32_t hb = __float_as_uint(hv[i]);
+          const uint64_t hh = ptx::pack_f32x2(hb, hb);
 #pragma unroll
-          for (int j = 0; j < 8; ++j) acc[i][j] = fmaf(wv[j], hv[i], acc[i][j]);
+          for (int j = 0; j < 4; ++j) acc[i][j] = ptx::fma_f32x2(wv[j], hh, acc[i][j]);
+        }
       }
 #pragma unroll
       for (int i = 0; i < 8; ++i) {
@@ -668,7 +674,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_certify_wres(CertArgs a, int Cp
 #pragma unroll
         for (int j = 0; j < 8; ++j) {
           const int c = cg * 8 + j;
-          if (c < C) lg[r * a.lstride + c] = acc[i][j] + b_s[c];
+          const float v = __uint_as_float((uint32_t)(acc[i][j >> 1] >> (32 * (j & 1))));
+          if (c < C) lg[r * a.lstride + c] = v + b_s[c];
         }
       }
     }
@@ -715,15 +722,21 @@ __global__ void __launch_bounds__(kThreads, 1) k_certify_wres(CertArgs a, int Cp
         L1 = fmaxf(L1, t.y);
       }
       if (r3 < nrows) {
+        // candidate mask first (a loop without side effects pipelines its
+        // loads), then the slots; a quarter holds at most 64 classes
+        unsigned long long cm = 0;
         for (int c = c_lo; c < c_hi; ++c) {
           const float sv = lrow[c];
           const float E = __fmaf_ru(eA[c], hn, __fmaf_ru(fabsf(sv), 2.3841858e-07f, eB[c]));
-          if (__fadd_ru(sv, E) >= L2) {
-            const int slot = atomicAdd(&ts.ncand[r3], 1);
-            if (slot < kMaxCand) {
-              ts.cls[r3][slot] = c;
-              ts.pairs[atomicAdd(&ts.npairs, 1)] = r3 | (slot << 8) | (c << 16);
-            }
+          cm |= (unsigned long long)(__fadd_ru(sv, E) >= L2) << (c - c_lo);
+        }
+        while (cm) {
+          const int c = c_lo + __ffsll((long long)cm) - 1;
+          cm &= cm - 1;
+          const int slot = atomicAdd(&ts.ncand[r3], 1);
+          if (slot < kMaxCand) {
+            ts.cls[r3][slot] = c;
+            ts.pairs[atomicAdd(&ts.npairs, 1)] = r3 | (slot << 8) | (c << 16);
           }
         }
       }
@@ -839,29 +852,56 @@ struct ScatterArgs {
   float* out_radius;
 };
 
-// Append accepted rows in input order; one warp per row.
-__global__ void __launch_bounds__(256) k_scatter(ScatterArgs a) {
+// Append accepted rows in input order. Each warp moves kScatterRows rows:
+// lane u < kScatterRows resolves row u's destination and copies its
+// per-entry fields, then the warp copies the keys of all its rows with every
+// load issued before the stores (float4s for 16-byte rows).
+constexpr int kScatterRows = 8;
+
+__global__ void __launch_bounds__(256) k_scatter(ScatterArgs a, int vec) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int64_t row = (int64_t)blockIdx.x * 8 + warp;
-  if (row >= a.n) return;
-  const bool acc = a.accept[row] != 0;
-  const int64_t dst = acc ? a.size0 + a.boff[row / kRows] + a.rank[row] : -1;
-  if (acc) {
-    float* kd = a.t.keys + (size_t)dst * a.dpad;
-    const float* hs = a.H + (size_t)row * a.d;
-    for (int j = lane; j < a.dpad; j += 32) kd[j] = j < a.d ? hs[j] : 0.f;
-    if (lane == 0) {
-      a.t.kn[dst] = a.kn[row];
-      a.t.tau[dst] = a.tau[row];
-      a.t.rr[dst] = a.rr[row];
-      a.t.radius[dst] = a.radius[row];
-      a.t.label[dst] = a.label[row];
-      a.t.yG[dst] = a.yG[row];
+  const int64_t row0 = ((int64_t)blockIdx.x * 8 + warp) * kScatterRows;
+  if (row0 >= a.n) return;
+  int64_t mydst = -2;  // past the end
+  if (lane < kScatterRows && row0 + lane < a.n) {
+    const int64_t row = row0 + lane;
+    mydst = a.accept[row] ? a.size0 + a.boff[row / kRows] + a.rank[row] : -1;
+    if (mydst >= 0) {
+      a.t.kn[mydst] = a.kn[row];
+      a.t.tau[mydst] = a.tau[row];
+      a.t.rr[mydst] = a.rr[row];
+      a.t.radius[mydst] = a.radius[row];
+      a.t.label[mydst] = a.label[row];
+      a.t.yG[mydst] = a.yG[row];
     }
-  }
-  if (lane == 0) {
-    if (a.out_index) a.out_index[row] = dst;
+    if (a.out_index) a.out_index[row] = mydst;
     if (a.out_radius) a.out_radius[row] = a.radius[row];
+  }
+  int64_t dst[kScatterRows];
+#pragma unroll
+  for (int u = 0; u < kScatterRows; ++u) dst[u] = __shfl_sync(0xffffffffu, mydst, u);
+  if (vec) {
+    const int n4 = a.dpad / 4, d4 = a.d / 4;
+    for (int j4 = lane; j4 < n4; j4 += 32) {
+      float4 v[kScatterRows];
+#pragma unroll
+      for (int u = 0; u < kScatterRows; ++u)
+        v[u] = (dst[u] >= 0 && j4 < d4) ? __ldg(reinterpret_cast<const float4*>(a.H + (size_t)(row0 + u) * a.d) + j4)
+                                        : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+      for (int u = 0; u < kScatterRows; ++u)
+        if (dst[u] >= 0) reinterpret_cast<float4*>(a.t.keys + (size_t)dst[u] * a.dpad)[j4] = v[u];
+    }
+  } else {
+    for (int j = lane; j < a.dpad; j += 32) {
+      float v[kScatterRows];
+#pragma unroll
+      for (int u = 0; u < kScatterRows; ++u)
+        v[u] = (dst[u] >= 0 && j < a.d) ? __ldg(a.H + (size_t)(row0 + u) * a.d + j) : 0.f;
+#pragma unroll
+      for (int u = 0; u < kScatterRows; ++u)
+        if (dst[u] >= 0) a.t.keys[(size_t)dst[u] * a.dpad + j] = v[u];
+    }
   }
 }
 
@@ -1024,7 +1064,9 @@ void certify_insert(lipcache* h, const float* H, int64_t n, const int32_t* paylo
   sa.t = h->table;
   sa.out_index = out_index;
   sa.out_radius = out_radius;
-  k_scatter<<<(unsigned)((n + 7) / 8), 256, 0, s>>>(sa);
+  const int vec = (h->d % 4 == 0 && ((uintptr_t)H & 15) == 0) ? 1 : 0;
+  const int64_t rows_per_block = 8 * kScatterRows;
+  k_scatter<<<(unsigned)((n + rows_per_block - 1) / rows_per_block), 256, 0, s>>>(sa, vec);
   LC_LAUNCH_CHECK("k_scatter");
 }
 
