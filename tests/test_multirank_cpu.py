@@ -53,3 +53,16 @@ def test_single_rank_aggregation_is_identity():
     assert d.world == int(os.environ.get("WORLD_SIZE", "1"))
     if d.world == 1:
         assert bench.aggregate(d, 500.0, 2.0) == (250.0, 2.0)
+
+
+def test_insert_roofline_arithmetic():
+    """The insert's ALU roofline: 2 C d flops per row over the run time
+    against SMs x 128 lanes x 2 flops x clock."""
+    import bench
+    import synth
+    w = synth.WORKLOADS["scale"]
+    r = bench.insert_summary(w, w.N, 20.0, 152, {"sm_max_mhz": 2070})
+    assert r["rows_per_s"] == w.N / 0.02
+    assert abs(r["roofline"]["achieved"] - 2 * w.N * w.C * w.d / 0.02 / 1e12) < 1e-9
+    assert abs(r["roofline"]["peak"] - 152 * 128 * 2 * 2070e6 / 1e12) < 1e-9
+    assert r["roofline"]["bound"] == "alu" and 0 < r["roofline"]["frac"] < 1
