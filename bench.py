@@ -47,7 +47,7 @@ def parse():
     p.add_argument("--warmup", type=int, default=5)
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
     p.add_argument("--workload", default="scale", choices=sorted(synth.WORKLOADS))
-    p.add_argument("--path", default="auto", choices=["auto", "tensor", "exact"])
+    p.add_argument("--path", default="auto", choices=["auto", "tensor", "tensor_single", "tensor_pair", "exact"])
     p.add_argument("--cpu-seconds", type=float, default=15.0, help="budget of the oracle CPU baseline")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cache-rows", type=int, default=0, help="override the workload's cache size N (profiling)")
@@ -164,7 +164,8 @@ def workload_data(w: synth.Workload):
     return W, b, rows, Q
 
 
-def roofline(w: synth.Workload, N: int, B: int, kernel_ms: float, pk: dict, pk_kind: str) -> dict:
+def roofline(w: synth.Workload, N: int, B: int, kernel_ms: float, pk: dict, pk_kind: str,
+             kernel: str = "k_probe_tc") -> dict:
     flops = 2.0 * B * N * w.d
     bytes_ = N * (4.0 * w.d + 4.0) + 4.0 * B * w.d + 16.0 * B
     tf32_peak = pk["bf16_tflops"] * TF32_OVER_BF16
@@ -177,19 +178,30 @@ def roofline(w: synth.Workload, N: int, B: int, kernel_ms: float, pk: dict, pk_k
         return {"bound": "tensor", "achieved": ach, "peak": tf32_peak, "unit": "TFLOP/s", "frac": ach / tf32_peak,
                 "traffic": None, "algorithmic_flops": flops, "algorithmic_bytes": bytes_,
                 "peak_source": f"{pk_kind} bf16 burst x nominal tf32/bf16 ratio {TF32_OVER_BF16:.4f}",
-                "kernel": "k_probe_tc", "kernel_ms": kernel_ms,
+                "kernel": kernel, "kernel_ms": kernel_ms,
                 "hbm_frac": bytes_ / s / 1e9 / hbm_peak}
     ach = bytes_ / s / 1e9
     return {"bound": "hbm", "achieved": ach, "peak": hbm_peak, "unit": "GB/s", "frac": ach / hbm_peak,
             "traffic": None, "algorithmic_flops": flops, "algorithmic_bytes": bytes_,
-            "peak_source": f"{pk_kind} copy bandwidth", "kernel": "k_probe_tc", "kernel_ms": kernel_ms}
+            "peak_source": f"{pk_kind} copy bandwidth", "kernel": kernel, "kernel_ms": kernel_ms}
 
 
-def recorded_traffic(workload: str):
-    """DRAM bytes per probe launch recorded in profiles/k_probe_tc_scale.md
+# main probe kernel per path: name, ncu summary, the sources its hash covers
+PROBE_KERNELS = {
+    4: ("k_probe_pair", "k_probe_pair_scale.md", ("probe_pair.cu", "tc_ptx.cuh", "probe_common.cuh")),
+    3: ("k_probe_tc", "k_probe_tc_scale.md", ("probe_tc.cu", "tc_ptx.cuh", "probe_common.cuh")),
+    2: ("k_probe_exact", None, ()),
+}
+
+
+def recorded_traffic(workload: str, path_id: int = 3):
+    """DRAM bytes per probe launch recorded in the kernel's profiles/ summary
     from an ncu capture, or None when the kernel sources changed since."""
     import hashlib
-    path = os.path.join(ROOT, "profiles", "k_probe_tc_scale.md")
+    name, summary, sources = PROBE_KERNELS[path_id]
+    if summary is None:
+        return None
+    path = os.path.join(ROOT, "profiles", summary)
     if not os.path.exists(path):
         return None
     rec = {}
@@ -199,7 +211,7 @@ def recorded_traffic(workload: str):
             if line.startswith(key + ":"):
                 rec[key] = line.split(":", 1)[1].strip()
     h = hashlib.sha256()
-    for f in ("probe_tc.cu", "tc_ptx.cuh", "probe_common.cuh"):
+    for f in sources:
         with open(os.path.join(ROOT, "paper_2608_13144_gb300", "csrc", f), "rb") as fh:
             h.update(fh.read())
     if rec.get("sources_sha256_16") != h.hexdigest()[:16] or rec.get("traffic_workload") != workload:
@@ -320,16 +332,17 @@ def run_ours(args, dist: Dist):
         cpu = cpu_baseline(w, W, b, rows, Q, args.cpu_seconds)
     cache.close()
 
-    rf = roofline(w, N, B, kernel_ms, pk, pk_kind)
-    if info["last_probe_path"] == 1 and w.N == synth.WORKLOADS[w.name].N:
-        rf["traffic"] = recorded_traffic(w.name)
+    path_id = info["last_probe_path"]
+    rf = roofline(w, N, B, kernel_ms, pk, pk_kind, PROBE_KERNELS[path_id][0])
+    if path_id in (3, 4) and w.N == synth.WORKLOADS[w.name].N:
+        rf["traffic"] = recorded_traffic(w.name, path_id)
     line = {
         "metric": METRIC, "value": value, "unit": "queries/s", "n_gpus": dist.world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": tmax / args.steps * 1e3, "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None, "dtype": "tf32" if info["last_probe_path"] == 1 else "fp32",
+        "scaling": "weak", "vs_baseline": None, "dtype": "tf32" if info["last_probe_path"] in (3, 4) else "fp32",
         "data": "synthetic (seeded Gaussian-mixture GuardNet features; no datasets or trained weights)",
         "config": {"workload": w.name, "N": N, "d": w.d, "C": w.C, "batch": B, "radius": "conservative",
-                   "probe_path": {1: "tensor", 2: "exact"}[info["last_probe_path"]],
+                   "probe_path": {2: "exact", 3: "tensor_single", 4: "tensor_pair"}[info["last_probe_path"]],
                    "parallelism": f"replicas{dist.world}" if dist.world > 1 else "single",
                    "l2": f"inputs larger than L2 ({N * (4 * info['d_pad'] + 16) / 1e9:.2f} GB key table)"},
         "pairs_per_s": value * N,

@@ -63,10 +63,14 @@ typedef enum lipcache_status {
 #define LIPCACHE_POLICY_GLOBAL 1     /* one global nearest-neighbour threshold (Sec. 5.4) */
 #define LIPCACHE_POLICY_INTERCLASS 2 /* radius from inter-class centroid distances (Sec. 5.4) */
 
-/* Probe kernels. Both return identical results; they differ in speed. */
-#define LIPCACHE_PROBE_AUTO 0   /* tensor path when supported (d <= 256), else exact */
-#define LIPCACHE_PROBE_TENSOR 1 /* tcgen05 TF32 screen, then exact FP32 recheck of candidates */
-#define LIPCACHE_PROBE_EXACT 2  /* exact FP32 distance of every pair on CUDA cores */
+/* Probe kernels. All return identical results; they differ in speed. */
+#define LIPCACHE_PROBE_AUTO 0          /* tensor path when supported (d <= 256), else exact */
+#define LIPCACHE_PROBE_TENSOR 1        /* tcgen05 TF32 screen, then exact FP32 recheck of candidates;
+                                          the kernel is chosen by shape: TENSOR_SINGLE for
+                                          d_pad <= 128, TENSOR_PAIR above (when clusters of four fit) */
+#define LIPCACHE_PROBE_EXACT 2         /* exact FP32 distance of every pair on CUDA cores */
+#define LIPCACHE_PROBE_TENSOR_SINGLE 3 /* the tensor screen with single-CTA MMAs (clusters of two) */
+#define LIPCACHE_PROBE_TENSOR_PAIR 4   /* the tensor screen with CTA-pair MMAs (clusters of four) */
 
 /* Limits checked by lipcache_create. */
 #define LIPCACHE_MAX_DIM 1024
@@ -90,7 +94,7 @@ typedef struct lipcache_info {
   int64_t candidates;       /* screen candidates rechecked since the last reset */
   int64_t device_errors;    /* kernel-reported errors since the last reset */
   int32_t probe_path;       /* LIPCACHE_PROBE_* configured for lipcache_probe */
-  int32_t last_probe_path;  /* path that served the last probe */
+  int32_t last_probe_path;  /* kernel that served the last probe: _EXACT, _TENSOR_SINGLE or _TENSOR_PAIR */
   float last_probe_ms;      /* main-kernel time of the last probe (timing enabled) */
   int32_t num_sms;          /* SMs of the device */
   double kernel_ms_total;   /* summed main-kernel time of timed probes since the last reset */

@@ -16,7 +16,7 @@ STATUS_NAMES = {0: "OK", 1: "E_INVALID", 2: "E_STATE", 3: "E_DEGENERATE_HEAD", 4
                 6: "E_CUDA", 7: "E_NOMEM", 8: "E_DEVICE"}
 RADIUS_CONSERVATIVE, RADIUS_TIGHT = 0, 1
 NOALLOC_SCRATCH_BYTES = 4259840  # LIPCACHE_NOALLOC_SCRATCH_BYTES
-PROBE_AUTO, PROBE_TENSOR, PROBE_EXACT = 0, 1, 2
+PROBE_AUTO, PROBE_TENSOR, PROBE_EXACT, PROBE_TENSOR_SINGLE, PROBE_TENSOR_PAIR = 0, 1, 2, 3, 4
 
 # Every symbol the header declares; tests check the library exports them all.
 EXPORTS = ["lipcache_create", "lipcache_set_head", "lipcache_insert", "lipcache_probe", "lipcache_probe_host",

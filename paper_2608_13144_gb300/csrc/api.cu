@@ -390,10 +390,10 @@ LC_API lipcache_status lipcache_probe_host(lipcache_t* h, const float* Q_host, i
 LC_API lipcache_status lipcache_set_probe_path(lipcache_t* h, int32_t path) {
   return guarded([&] {
     check_handle(h);
-    LC_REQUIRE(path == LIPCACHE_PROBE_AUTO || path == LIPCACHE_PROBE_TENSOR || path == LIPCACHE_PROBE_EXACT,
-               LIPCACHE_E_INVALID, "unknown probe path");
-    LC_REQUIRE(path != LIPCACHE_PROBE_TENSOR || lc::tensor_path_supported(h->dpad), LIPCACHE_E_INVALID,
-               "the tensor probe supports d <= 256");
+    LC_REQUIRE(path >= LIPCACHE_PROBE_AUTO && path <= LIPCACHE_PROBE_TENSOR_PAIR, LIPCACHE_E_INVALID,
+               "unknown probe path");
+    LC_REQUIRE(path == LIPCACHE_PROBE_AUTO || path == LIPCACHE_PROBE_EXACT || lc::tensor_path_supported(h->dpad),
+               LIPCACHE_E_INVALID, "the tensor probe supports d <= 256");
     h->probe_path = path;
   });
 }

@@ -204,6 +204,7 @@ struct lipcache {
 
   double eps_rc = 0.0, c_scr = 0.0;
   lc::EncodeTiledFn encode = nullptr;
+  int pair_clusters = -1;  // resident clusters of the pair probe kernel (-1: not yet queried)
 
   // radius policy (Sec. 5.4): the probe reads rr_emp / tau_emp instead of
   // the certified thresholds when policy != LIPCACHE_POLICY_CERTIFIED
@@ -244,13 +245,19 @@ void consistency_check(lipcache* h, const float* Q, int64_t B, const int64_t* hi
 void probe(lipcache* h, const float* Q, int64_t B, int64_t* out_index, int32_t* out_label, float* out_dist,
            cudaStream_t s);
 bool tensor_path_supported(int dpad);
-// probe_tc.cu
-void launch_probe_tc(lipcache* h, int64_t B, cudaStream_t s);
+// probe_tc.cu: the tensor probe; `path` is LIPCACHE_PROBE_TENSOR (kernel
+// chosen by shape), _TENSOR_SINGLE or _TENSOR_PAIR. Returns the kernel that
+// ran (_TENSOR_SINGLE or _TENSOR_PAIR).
+int launch_probe_tc(lipcache* h, int64_t B, int path, cudaStream_t s);
+// probe_pair.cu
+int probe_pair_clusters(lipcache* h);
+void launch_probe_pair(lipcache* h, int64_t B, const float* qpad, const float* kappa, unsigned long long* best,
+                       cudaStream_t s);
 // probe.cu / probe_tc.cu: the probe on caller-provided scratch memory
 void probe_external_scratch(lipcache* h, const float* Q, int64_t B, int64_t* out_index, int32_t* out_label,
                             float* out_dist, float* qpad, float* kappa, unsigned long long* best, cudaStream_t s);
-void launch_probe_tc_external(lipcache* h, int64_t B, const float* qpad, const float* kappa, unsigned long long* best,
-                              cudaStream_t s);
+int launch_probe_tc_external(lipcache* h, int64_t B, int path, const float* qpad, const float* kappa,
+                             unsigned long long* best, cudaStream_t s);
 // api.cu: run fn(ctx) with the C ABI's error handling (status + message)
 lipcache_status run_guarded(void (*fn)(void*), void* ctx);
 // api.cu: harvest completed timing events (blocking on the oldest if `all`

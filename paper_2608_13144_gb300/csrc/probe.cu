@@ -188,8 +188,8 @@ void probe(lipcache* h, const float* Q, int64_t B, int64_t* out_index, int32_t* 
       slot = (int)(h->t_issued % lipcache::kTimingRing);
       LC_CUDA(cudaEventRecord(h->tev0[slot], s));
     }
-    if (path == LIPCACHE_PROBE_TENSOR) {
-      launch_probe_tc(h, B, s);
+    if (path != LIPCACHE_PROBE_EXACT) {
+      h->last_probe_path = launch_probe_tc(h, B, path, s);
     } else {
       dim3 grid((unsigned)((h->size + kEK - 1) / kEK), (unsigned)((B + kEQ - 1) / kEQ));
       h->last_grid = (int)(grid.x * grid.y);
@@ -220,8 +220,8 @@ void probe_external_scratch(lipcache* h, const float* Q, int64_t B, int64_t* out
   if (path == LIPCACHE_PROBE_AUTO) path = tensor_path_supported(h->dpad) ? LIPCACHE_PROBE_TENSOR : LIPCACHE_PROBE_EXACT;
   h->last_probe_path = path;
   if (h->size > 0) {
-    if (path == LIPCACHE_PROBE_TENSOR) {
-      launch_probe_tc_external(h, B, qpad, kappa, best, s);
+    if (path != LIPCACHE_PROBE_EXACT) {
+      h->last_probe_path = launch_probe_tc_external(h, B, path, qpad, kappa, best, s);
     } else {
       dim3 grid((unsigned)((h->size + kEK - 1) / kEK), (unsigned)((B + kEQ - 1) / kEQ));
       k_probe_exact<<<grid, 256, 0, s>>>(qpad, B, h->table.keys, h->probe_rr(), h->size, h->dpad, best);

@@ -9,8 +9,9 @@
 //     a > (1 - c) |q|^2 / 2 + ((1 - c) |k|^2 - R_k) / 2 = kappa_q + tau_k,
 // with kappa_q (per query, k_prologue) rounded down and tau_k (per key,
 // stored at insertion) rounded down. The epilogue keeps a pair iff
-// fl(a - tau_k) >= kappa_q, which therefore never drops an acceptable pair;
-// the separable form costs one subtraction and one max per pair.
+// fl(a - tau_k) >= kappa_q, which therefore never drops an acceptable pair.
+// It first tests each 32-key chunk with fl(max a - min tau) >= kappa_q (one
+// three-input max per two pairs), which no chunk holding a kept pair fails.
 //
 // Schedule. Persistent CTAs, one per SM, launched as clusters of two. The two
 // CTAs of a cluster own two adjacent key tiles and stream the SAME sequence of
@@ -311,12 +312,21 @@ __global__ void __launch_bounds__(kThreads, 1)
       unit_range(a, u, rank, kt, qt0, qt1);
       const bool live = kt < a.n_kt;
       const int key0 = kt * BN + half * kColsPerWarp;
-      // this warp's screen terms for the unit's key tile, staged once per unit
+      // this warp's screen terms for the unit's key tile, staged once per
+      // unit, and their minimum over each 32-key chunk
       __syncwarp();
       if (live)
         for (int v4 = lane; v4 < kColsPerWarp / 4; v4 += 32)
           reinterpret_cast<float4*>(my_tau)[v4] = __ldg(reinterpret_cast<const float4*>(a.tau + key0) + v4);
       __syncwarp();
+      float tmin[kChunks];
+#pragma unroll
+      for (int ch = 0; ch < kChunks; ++ch) {
+        float m = live ? my_tau[ch * 32 + lane] : INFINITY;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) m = fminf(m, __shfl_xor_sync(0xffffffffu, m, o));
+        tmin[ch] = m;
+      }
       float kap = __ldg(a.kappa + qt0 * kBM + quarter * 32 + lane);
       for (int qt = qt0; qt < qt1; ++qt, ++t) {
         const int buf = t & 1;
@@ -336,19 +346,17 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int ch = 0; ch < kChunks; ++ch) {
             if (ch + 1 < kChunks) ptx::tmem_ld32(tbase + (uint32_t)((ch + 1) * 32), r[(ch + 1) & 1]);
             const uint32_t* v = r[ch & 1];
-            // fl(a - tau) for two columns per instruction, folded into two
-            // independent three-input max chains
-            const uint4* t4 = reinterpret_cast<const uint4*>(my_tau + ch * 32);
+            // Coarse test of the chunk: a_j - tau_j <= max_j a_j - min_j tau_j
+            // exactly, and rounding is monotone, so a chunk whose
+            // fl(max a - min tau) is below kappa holds no pair that passes
+            // fl(a_j - tau_j) >= kappa. Two independent three-input max chains.
             float m0 = -INFINITY, m1 = -INFINITY;
 #pragma unroll
-            for (int j4 = 0; j4 < 8; ++j4) {
-              const uint4 tv = t4[j4];
-              const uint64_t d0 = ptx::sub_f32x2(ptx::pack_f32x2(v[4 * j4 + 0], v[4 * j4 + 1]), ptx::pack_f32x2(tv.x, tv.y));
-              const uint64_t d1 = ptx::sub_f32x2(ptx::pack_f32x2(v[4 * j4 + 2], v[4 * j4 + 3]), ptx::pack_f32x2(tv.z, tv.w));
-              m0 = ptx::max3_f32(m0, __uint_as_float((uint32_t)d0), __uint_as_float((uint32_t)(d0 >> 32)));
-              m1 = ptx::max3_f32(m1, __uint_as_float((uint32_t)d1), __uint_as_float((uint32_t)(d1 >> 32)));
+            for (int j = 0; j < 16; j += 2) {
+              m0 = ptx::max3_f32(m0, __uint_as_float(v[j]), __uint_as_float(v[j + 1]));
+              m1 = ptx::max3_f32(m1, __uint_as_float(v[16 + j]), __uint_as_float(v[16 + j + 1]));
             }
-            if (fmaxf(m0, m1) >= kap) {
+            if (__fsub_rn(fmaxf(m0, m1), tmin[ch]) >= kap) {
               uint32_t mask = 0;
 #pragma unroll
               for (int j = 0; j < 32; ++j)
@@ -474,17 +482,27 @@ void launch(lipcache* h, int64_t B, const float* qpad, const float* kappa, unsig
 
 int tc_key_tile(int dpad) { return dpad <= 128 ? 256 : 128; }
 
-void launch_probe_tc_external(lipcache* h, int64_t B, const float* qpad, const float* kappa, unsigned long long* best,
-                              cudaStream_t s) {
+int launch_probe_tc_external(lipcache* h, int64_t B, int path, const float* qpad, const float* kappa,
+                             unsigned long long* best, cudaStream_t s) {
   LC_REQUIRE(tensor_path_supported(h->dpad), LIPCACHE_E_INVALID, "the tensor probe supports d <= 256");
+  // Pair MMAs read a third less shared memory per flop; that decides for
+  // d_pad > 128, where the single-CTA kernel has to use 128-key tiles. At
+  // d_pad <= 128 its 256-key tiles on all SMs (clusters of four leave some
+  // idle) are faster.
+  const bool pair = path == LIPCACHE_PROBE_TENSOR_PAIR || (path == LIPCACHE_PROBE_TENSOR && h->dpad > 128);
+  if (pair && probe_pair_clusters(h) >= 1) {
+    launch_probe_pair(h, B, qpad, kappa, best, s);
+    return LIPCACHE_PROBE_TENSOR_PAIR;
+  }
   if (tc_key_tile(h->dpad) == 256)
     launch<256>(h, B, qpad, kappa, best, s);
   else
     launch<128>(h, B, qpad, kappa, best, s);
+  return LIPCACHE_PROBE_TENSOR_SINGLE;
 }
 
-void launch_probe_tc(lipcache* h, int64_t B, cudaStream_t s) {
-  launch_probe_tc_external(h, B, h->qpad, h->kappa, h->best, s);
+int launch_probe_tc(lipcache* h, int64_t B, int path, cudaStream_t s) {
+  return launch_probe_tc_external(h, B, path, h->qpad, h->kappa, h->best, s);
 }
 
 }  // namespace lc

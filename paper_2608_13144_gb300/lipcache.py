@@ -15,7 +15,8 @@ from . import _lib
 from ._lib import Info, check
 
 RADIUS_MODES = {"conservative": _lib.RADIUS_CONSERVATIVE, "tight": _lib.RADIUS_TIGHT}
-PROBE_PATHS = {"auto": _lib.PROBE_AUTO, "tensor": _lib.PROBE_TENSOR, "exact": _lib.PROBE_EXACT}
+PROBE_PATHS = {"auto": _lib.PROBE_AUTO, "tensor": _lib.PROBE_TENSOR, "exact": _lib.PROBE_EXACT,
+               "tensor_single": _lib.PROBE_TENSOR_SINGLE, "tensor_pair": _lib.PROBE_TENSOR_PAIR}
 RADIUS_POLICIES = {"certified": 0, "global": 1, "interclass": 2}
 
 

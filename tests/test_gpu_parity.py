@@ -10,7 +10,7 @@ from parity_utils import check_insert, check_probe
 torch = pytest.importorskip("torch")
 pytestmark = pytest.mark.gpu
 
-PATHS = ["exact", "tensor"]
+PATHS = ["exact", "tensor", "tensor_single", "tensor_pair"]
 
 
 @pytest.fixture(scope="module")
@@ -43,7 +43,7 @@ def run_probe(cache, Q, dev, batch, path):
         for k in range(3):
             outs[k].append(o[k].cpu().numpy())
     info = cache.info()
-    assert info["device_errors"] == 0 and info["last_probe_path"] == {"exact": 2, "tensor": 1}[path]
+    assert info["device_errors"] == 0 and info["last_probe_path"] in {"exact": (2,), "tensor": (3, 4), "tensor_single": (3,), "tensor_pair": (4,)}[path]
     return [np.concatenate(x) if x else np.zeros(0) for x in outs]
 
 
@@ -230,10 +230,11 @@ def test_tensor_equals_exact(built, dev, name):
     dropped an accepted pair would show up here."""
     s = built(name)
     a = run_probe(s["cache"], s["Q"], dev, s["w"].batch, "exact")
-    b = run_probe(s["cache"], s["Q"], dev, s["w"].batch, "tensor")
-    for x, y in zip(a, b):
-        assert np.array_equal(x.view(np.uint8) if x.dtype == np.float32 else x,
-                              y.view(np.uint8) if y.dtype == np.float32 else y)
+    for path in ("tensor", "tensor_single", "tensor_pair"):
+        b = run_probe(s["cache"], s["Q"], dev, s["w"].batch, path)
+        for x, y in zip(a, b):
+            assert np.array_equal(x.view(np.uint8) if x.dtype == np.float32 else x,
+                                  y.view(np.uint8) if y.dtype == np.float32 else y), path
 
 
 @pytest.mark.parametrize("name", ["tiny", "cifar100"])
