@@ -13,6 +13,8 @@ Functions (each follows the passage cited in the C source):
   consistency                   certified-consistency rate of the hits (Sec. 5)
   interclass_radius             empirical inter-class-distance radius (Sec. 5.4)
   global_radius                 one global threshold for every entry (Sec. 5.4)
+  select_radius_dedup           selection S: radius-prioritised de-duplication (Algorithm 1, Sec. 5.5)
+  radius_rz32                   FP32 radius rounded toward zero (the order key of the selection)
   pair_dist                     ||q - k||_2 for given pairs
 """
 from __future__ import annotations
@@ -243,6 +245,60 @@ def interclass_radius(keys, labels, n_classes, beta=1.0) -> dict:
     ok = (labels >= 0) & (labels < C)
     radius[ok] = rho[labels[ok]]
     return {"rho": rho, "radius": radius, "centroid": mu, "count": count}
+
+
+def radius_rz32(r) -> np.ndarray:
+    """FP64 radii rounded toward zero to FP32 (NaN stays NaN)."""
+    r = np.asarray(r, dtype=np.float64)
+    with np.errstate(over="ignore"):
+        f = r.astype(np.float32)  # beyond the FP32 range: inf, corrected below
+    over = np.isfinite(r) & (np.abs(f.astype(np.float64)) > np.abs(r))
+    f[over] = np.nextafter(f[over], np.float32(0))
+    return f
+
+
+def select_radius_dedup(rows, cert, keys0=None, radius0=None, budget_total=0, budget_per_class=0, n_classes=0):
+    """Selection strategy S of Algorithm 1, read as radius-prioritised
+    de-duplication (the default strategy of Sec. 5.5; the paper gives no
+    formula). The certified candidates (cert["accept"]) are visited in order
+    of decreasing radius, the radius rounded toward zero to FP32 (ties: lower
+    row first). A candidate is skipped if it lies strictly inside the
+    certified ball of an entry already kept -- an entry of the existing cache
+    (keys0, radius0) or one selected earlier in this pass -- i.e. if the
+    lookup would already hit it (Eq. 13), or if its class (payload label in
+    [0, C)) has budget_per_class selected entries or the pass has
+    budget_total (0 = unlimited). Returns the selected rows in visiting
+    order."""
+    rows = np.asarray(rows, dtype=np.float32)
+    acc = np.asarray(cert["accept"], dtype=bool)
+    r64 = np.asarray(cert["radius"], dtype=np.float64)
+    lab = np.asarray(cert["label"], dtype=np.int64)
+    r32 = radius_rz32(r64)
+    cand = np.nonzero(acc)[0]
+    order = sorted(cand.tolist(), key=lambda i: (-float(r32[i]), i))
+    kept_z = [np.asarray(z, dtype=np.float64) for z in (keys0 if keys0 is not None else [])]
+    kept_r = [float(x) for x in (radius0 if radius0 is not None else [])]
+    per = {}
+    out = []
+    for i in order:
+        if budget_total and len(out) >= budget_total:
+            break
+        c = int(lab[i])
+        if budget_per_class and 0 <= c < max(n_classes, 1) and per.get(c, 0) >= budget_per_class:
+            continue
+        z = rows[i].astype(np.float64)
+        covered = False
+        for kz, kr in zip(kept_z, kept_r):
+            if np.sqrt(np.sum((z - kz) ** 2)) < kr:
+                covered = True
+                break
+        if covered:
+            continue
+        out.append(i)
+        kept_z.append(z)
+        kept_r.append(float(r64[i]))
+        per[c] = per.get(c, 0) + 1
+    return np.asarray(out, dtype=np.int64)
 
 
 def pair_dist(Q, K, qi, ki) -> np.ndarray:

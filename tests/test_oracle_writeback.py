@@ -175,3 +175,73 @@ def test_global_radius_hits_nearest_within_tau():
     np.testing.assert_array_equal((p["index"] >= 0)[clear], (dist < tau)[clear])
     hit = (p["index"] >= 0) & clear
     np.testing.assert_array_equal(p["index"][hit], idx[hit])
+
+
+# ---------------------------------------------------------------- selection strategy S
+def test_golden_select_radius_dedup():
+    g = golden("select_radius_dedup.json")
+    W, b = np.array(g["W"], np.float32), np.array(g["b"], np.float32)
+    rows = np.array(g["rows"], np.float32)
+    cert = oracle.certify(W, b, g["sigma"], rows)
+    assert oracle.select_radius_dedup(rows, cert).tolist() == g["expect"]
+    assert oracle.select_radius_dedup(rows, cert, budget_per_class=1, n_classes=2).tolist() == g["expect_per_class_1"]
+    assert oracle.select_radius_dedup(rows, cert, budget_total=2).tolist() == g["expect_total_2"]
+    sel = oracle.select_radius_dedup(rows, cert, keys0=np.array(g["existing_keys"], np.float32),
+                                     radius0=np.array(g["existing_radius"]))
+    assert sel.tolist() == g["expect_with_existing"]
+
+
+def _check_greedy(rows, cert, sel, keys0, radius0, budget_total, budget_per_class, C):
+    """The selection is the unique greedy result for the visiting order iff
+    (i) no kept entry lies inside the ball of an entry kept before it and
+    (ii) every candidate not kept lies inside such a ball or met an
+    exhausted budget at its turn. Checked here by brute force over the order."""
+    r32 = oracle.radius_rz32(cert["radius"])
+    order = sorted(np.nonzero(cert["accept"])[0].tolist(), key=lambda i: (-float(r32[i]), i))
+    chosen = set(sel.tolist())
+    kept_z = [z.astype(np.float64) for z in keys0]
+    kept_r = list(radius0)
+    per, total, pos = {}, 0, 0
+    for i in order:
+        z = rows[i].astype(np.float64)
+        covered = any(np.linalg.norm(z - kz) < kr for kz, kr in zip(kept_z, kept_r))
+        c = int(cert["label"][i])
+        full = (budget_total and total >= budget_total) or (budget_per_class and per.get(c, 0) >= budget_per_class)
+        if i in chosen:
+            assert not covered and not full
+            assert sel[pos] == i  # kept entries come out in visiting order
+            pos += 1
+            kept_z.append(z)
+            kept_r.append(float(cert["radius"][i]))
+            per[c] = per.get(c, 0) + 1
+            total += 1
+        else:
+            assert covered or full
+    assert pos == len(sel)
+
+
+@pytest.mark.parametrize("seed,C,d,bt,bc", [(0, 3, 2, 0, 0), (1, 4, 3, 0, 3), (2, 5, 2, 7, 0), (3, 2, 4, 0, 0),
+                                            (4, 6, 3, 10, 2)])
+def test_select_radius_dedup_is_the_greedy(seed, C, d, bt, bc):
+    rng, W, b, rows = _instance(seed, C, d, 300, 0)
+    rows = (0.5 * rows).astype(np.float32)  # dense enough that balls overlap
+    s = oracle.sigma_max(W)
+    cert = oracle.certify(W, b, s, rows)
+    keys0 = rows[:5] + np.float32(0.01)
+    radius0 = np.full(5, 0.3)
+    sel = oracle.select_radius_dedup(rows, cert, keys0, radius0, bt, bc, C)
+    assert 0 < len(sel) < int(cert["accept"].sum())
+    _check_greedy(rows, cert, sel, keys0, radius0, bt, bc, C)
+    if bt:
+        assert len(sel) <= bt
+    if bc:
+        assert np.bincount(cert["label"][sel], minlength=C).max() <= bc
+
+
+def test_radius_rz32_rounds_toward_zero():
+    r = np.array([1.0, 0.1, 1 / 3, 2.0 ** -130, 3.5e38, 0.0, np.inf])
+    f = oracle.radius_rz32(r)
+    assert np.all(f.astype(np.float64)[:6] <= r[:6]) and f[6] == np.inf
+    with np.errstate(over="ignore"):
+        nxt = np.nextafter(f[:6], np.float32(np.inf)).astype(np.float64)
+    assert np.all(nxt > r[:6])  # the largest FP32 value not above r
