@@ -180,6 +180,40 @@ lipcache_status lipcache_insert(lipcache_t* h, const float* H, int64_t n, const 
 lipcache_status lipcache_probe(lipcache_t* h, const float* Q, int64_t B, int64_t* out_index, int32_t* out_label,
                                float* out_dist, lipcache_stream_t stream);
 
+/* Selection strategies S (Algorithm 1, last steps; lipcache_insert_select). */
+#define LIPCACHE_SELECT_ALL 0          /* every certified candidate, in input order (= lipcache_insert) */
+#define LIPCACHE_SELECT_RADIUS_DEDUP 1 /* radius-prioritised de-duplication (Sec. 5.5) */
+
+/*
+ * Algorithm 1 with a selection strategy S: certify the n candidate rows as
+ * lipcache_insert does, then append the ones S selects.
+ *   LIPCACHE_SELECT_RADIUS_DEDUP (the default strategy of Sec. 5.5; the paper
+ *   names it without a formula): the certified candidates are visited in
+ *   order of decreasing radius (the FP32 radius, ties to the lower row); a
+ *   candidate is skipped if lipcache_probe would already hit it -- it lies
+ *   strictly inside the ball of an entry of the cache, present before the
+ *   call or kept earlier in it -- or if its class (payload label in [0, C))
+ *   has budget_per_class entries kept by this call, or the call has kept
+ *   budget_total. Kept rows are appended in visiting order. The coverage test
+ *   is the probe's conservative one, so a skipped row is always exactly
+ *   covered; a row within ~2e-6 relative of a ball's boundary may be kept
+ *   where exact arithmetic would skip it.
+ *   LIPCACHE_SELECT_ALL: lipcache_insert (budgets must be 0).
+ *   budget_total, budget_per_class   <= 0: unlimited
+ *   out_index    n int64 (device), nullable: cache index of a kept row, else -1
+ *   out_radius   n FP32 (device), nullable: as for lipcache_insert
+ *   n_selected   host, nullable: rows appended
+ * Requires the certified radius policy (the coverage test uses the certified
+ * balls). Synchronises `stream` (once per 4,096 candidates). All or nothing
+ * on capacity: E_FULL, before any work, if size + min(n, budget_total)
+ * exceeds it. Errors: those of lipcache_insert and lipcache_probe; E_STATE
+ * under an empirical radius policy; E_INVALID for an unknown strategy.
+ */
+lipcache_status lipcache_insert_select(lipcache_t* h, const float* H, int64_t n, const int32_t* payload,
+                                       int32_t require_consistency, int32_t strategy, int64_t budget_total,
+                                       int32_t budget_per_class, int64_t* out_index, float* out_radius,
+                                       int64_t* n_selected, lipcache_stream_t stream);
+
 /*
  * Lookup with write-back (Algorithm 2 with its write-back flag set): probe
  * the batch as lipcache_probe does, then certify every missed query as

@@ -276,8 +276,13 @@ def select_radius_dedup(rows, cert, keys0=None, radius0=None, budget_total=0, bu
     r32 = radius_rz32(r64)
     cand = np.nonzero(acc)[0]
     order = sorted(cand.tolist(), key=lambda i: (-float(r32[i]), i))
-    kept_z = [np.asarray(z, dtype=np.float64) for z in (keys0 if keys0 is not None else [])]
-    kept_r = [float(x) for x in (radius0 if radius0 is not None else [])]
+    k0 = np.asarray(keys0 if keys0 is not None else np.zeros((0, rows.shape[1])), dtype=np.float64)
+    r0 = np.asarray(radius0 if radius0 is not None else np.zeros(0), dtype=np.float64)
+    kept_z = np.zeros((len(k0) + len(cand), rows.shape[1]), dtype=np.float64)  # entries kept so far
+    kept_r = np.zeros(len(k0) + len(cand), dtype=np.float64)
+    kept_z[:len(k0)] = k0
+    kept_r[:len(k0)] = r0
+    m = len(k0)
     per = {}
     out = []
     for i in order:
@@ -287,16 +292,13 @@ def select_radius_dedup(rows, cert, keys0=None, radius0=None, budget_total=0, bu
         if budget_per_class and 0 <= c < max(n_classes, 1) and per.get(c, 0) >= budget_per_class:
             continue
         z = rows[i].astype(np.float64)
-        covered = False
-        for kz, kr in zip(kept_z, kept_r):
-            if np.sqrt(np.sum((z - kz) ** 2)) < kr:
-                covered = True
-                break
-        if covered:
+        # the lookup of Eq. 13 against every entry kept so far (direct differences, FP64)
+        if m and np.any(np.sqrt(np.sum((kept_z[:m] - z) ** 2, axis=1)) < kept_r[:m]):
             continue
         out.append(i)
-        kept_z.append(z)
-        kept_r.append(float(r64[i]))
+        kept_z[m] = z
+        kept_r[m] = r64[i]
+        m += 1
         per[c] = per.get(c, 0) + 1
     return np.asarray(out, dtype=np.int64)
 

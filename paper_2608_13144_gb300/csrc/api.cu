@@ -65,6 +65,7 @@ void release(lipcache* h) {
   dev_free(h->gram[1]);
   dev_free(h->spec);
   if (h->spec_host) cudaFreeHost(h->spec_host);
+  lc::release_select(h);
   dev_free(h->rr_emp);
   dev_free(h->tau_emp);
   dev_free(h->rho);
@@ -280,6 +281,41 @@ LC_API lipcache_status lipcache_probe(lipcache_t* h, const float* Q, int64_t B, 
     LC_REQUIRE(((uintptr_t)Q & 3) == 0, LIPCACHE_E_INVALID, "Q must be 4-byte aligned");
     use_device(h);
     lc::probe(h, Q, B, out_index, out_label, out_dist, reinterpret_cast<cudaStream_t>(stream));
+  });
+}
+
+LC_API lipcache_status lipcache_insert_select(lipcache_t* h, const float* H, int64_t n, const int32_t* payload,
+                                              int32_t require_consistency, int32_t strategy, int64_t budget_total,
+                                              int32_t budget_per_class, int64_t* out_index, float* out_radius,
+                                              int64_t* n_selected, lipcache_stream_t stream) {
+  if (n_selected) *n_selected = 0;
+  return guarded([&] {
+    check_handle(h);
+    LC_REQUIRE(strategy == LIPCACHE_SELECT_ALL || strategy == LIPCACHE_SELECT_RADIUS_DEDUP, LIPCACHE_E_INVALID,
+               "unknown selection strategy");
+    if (strategy == LIPCACHE_SELECT_ALL) {
+      LC_REQUIRE(budget_total <= 0 && budget_per_class <= 0, LIPCACHE_E_INVALID,
+                 "LIPCACHE_SELECT_ALL takes no budget");
+      const lipcache_status st = lipcache_insert(h, H, n, payload, require_consistency, out_index, out_radius,
+                                                 n_selected, stream);
+      if (st != LIPCACHE_OK) throw lc::Error(st, lipcache_last_error());
+      return;
+    }
+    LC_REQUIRE(h->head_set, LIPCACHE_E_STATE, "insert before set_head");
+    LC_REQUIRE(h->policy == LIPCACHE_POLICY_CERTIFIED, LIPCACHE_E_STATE,
+               "selection needs the certified radius policy");
+    LC_REQUIRE(n >= 0 && n < (1LL << 31), LIPCACHE_E_INVALID, "n must be in [0, 2^31)");
+    if (n == 0) return;
+    LC_REQUIRE(H != nullptr, LIPCACHE_E_INVALID, "H is NULL");
+    LC_REQUIRE(((uintptr_t)H & 3) == 0, LIPCACHE_E_INVALID, "H must be 4-byte aligned");
+    const int64_t most = budget_total > 0 && budget_total < n ? budget_total : n;
+    LC_REQUIRE(most <= h->capacity - h->size, LIPCACHE_E_FULL, "the selection could exceed the cache capacity");
+    use_device(h);
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    const int64_t kept = lc::select_insert(h, H, n, payload, require_consistency, budget_total, budget_per_class,
+                                           out_index, out_radius, s);
+    LC_CUDA(cudaStreamSynchronize(s));
+    if (n_selected) *n_selected = kept;
   });
 }
 

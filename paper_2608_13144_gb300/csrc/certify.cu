@@ -1070,6 +1070,11 @@ void certify_insert(lipcache* h, const float* H, int64_t n, const int32_t* paylo
   LC_LAUNCH_CHECK("k_scatter");
 }
 
+void certify_rows(lipcache* h, const float* H, int64_t n, const int32_t* payload, int require_consistency,
+                  cudaStream_t s) {
+  launch_certify(h, H, n, payload, require_consistency, nullptr, s);
+}
+
 void consistency_check(lipcache* h, const float* Q, int64_t B, const int64_t* hit_index, int8_t* out,
                        cudaStream_t s) {
   launch_certify(h, Q, B, nullptr, 0, nullptr, s);

@@ -117,6 +117,26 @@ struct DevStats {
   int pad;
 };
 
+// Scratch of the selection strategy (select.cu), grown on demand.
+struct SelectScratch {
+  unsigned long long* keys = nullptr;
+  int64_t keys_cap = 0;
+  float* G = nullptr;  // chunk members' features
+  int64_t G_cap = 0;
+  int32_t* rows = nullptr;
+  int64_t rows_cap = 0;
+  int64_t* hit = nullptr;
+  int64_t hit_cap = 0;
+  uint32_t* cov = nullptr;
+  int64_t cov_cap = 0;
+  int32_t* list = nullptr;
+  int64_t list_cap = 0;
+  int32_t* class_cnt = nullptr;
+  int64_t class_cap = 0;
+  int64_t* small = nullptr;       // device: accepted, kept, chunk count
+  int64_t* small_host = nullptr;  // pinned
+};
+
 // Per-entry table of the cache (structure of arrays, capacity entries).
 struct Table {
   float* keys = nullptr;     // capacity x dpad, zero padded
@@ -205,6 +225,7 @@ struct lipcache {
   double eps_rc = 0.0, c_scr = 0.0;
   lc::EncodeTiledFn encode = nullptr;
   int pair_clusters = -1;  // resident clusters of the pair probe kernel (-1: not yet queried)
+  lc::SelectScratch sel;
 
   // radius policy (Sec. 5.4): the probe reads rr_emp / tau_emp instead of
   // the certified thresholds when policy != LIPCACHE_POLICY_CERTIFIED
@@ -237,6 +258,15 @@ void certify_insert(lipcache* h, const float* H, int64_t n, const int32_t* paylo
 void set_radius_policy(lipcache* h, int policy, double param, double* rho_host, cudaStream_t s);
 // thresholds of entries [first, first + n) under the current policy
 void policy_fill(lipcache* h, int64_t first, int64_t n, cudaStream_t s);
+// certify.cu: certification of H into the insert scratch only (no append)
+void certify_rows(lipcache* h, const float* H, int64_t n, const int32_t* payload, int require_consistency,
+                  cudaStream_t s);
+// select.cu: radius-prioritised de-duplication of the certified rows of H
+// into the cache; returns the number of entries appended.
+int64_t select_insert(lipcache* h, const float* H, int64_t n, const int32_t* payload, int require_consistency,
+                      int64_t budget_total, int budget_per_class, int64_t* out_index, float* out_radius,
+                      cudaStream_t s);
+void release_select(lipcache* h);
 // Certified-consistency check: argmax of the head on Q against y^G of the hit
 // entries; counts (hits, consistent, invalid index) land in ins_total[1..3].
 void consistency_check(lipcache* h, const float* Q, int64_t B, const int64_t* hit_index, int8_t* out,

@@ -18,6 +18,7 @@ RADIUS_MODES = {"conservative": _lib.RADIUS_CONSERVATIVE, "tight": _lib.RADIUS_T
 PROBE_PATHS = {"auto": _lib.PROBE_AUTO, "tensor": _lib.PROBE_TENSOR, "exact": _lib.PROBE_EXACT,
                "tensor_single": _lib.PROBE_TENSOR_SINGLE, "tensor_pair": _lib.PROBE_TENSOR_PAIR}
 RADIUS_POLICIES = {"certified": 0, "global": 1, "interclass": 2}
+SELECT_STRATEGIES = {"all": 0, "radius_dedup": 1}
 
 
 def _stream(device: torch.device):
@@ -90,6 +91,25 @@ class LipCache:
         check(self.L.lipcache_insert(self._h, _ptr(H), n, _ptr(payload), int(bool(require_consistency)),
                                      _ptr(index), _ptr(radius), C.byref(acc), _stream(self.device)))
         return index, radius, acc.value
+
+    def insert_select(self, H: torch.Tensor, payload: torch.Tensor | None = None, require_consistency: bool = False,
+                      strategy: str = "radius_dedup", budget_total: int = 0, budget_per_class: int = 0):
+        """Algorithm 1 with a selection strategy S ("radius_dedup": radius-
+        prioritised de-duplication; "all": insert). Returns (index, radius,
+        n_selected); index[i] is the cache index of row i or -1."""
+        H = self._dev(H, torch.float32, "H")
+        n = H.shape[0]
+        if H.dim() != 2 or (n and H.shape[1] != self.d):
+            raise ValueError("H must be n x d")
+        if payload is not None:
+            payload = self._dev(payload, torch.int32, "payload")
+        index = torch.empty(n, dtype=torch.int64, device=self.device)
+        radius = torch.empty(n, dtype=torch.float32, device=self.device)
+        got = C.c_int64()
+        check(self.L.lipcache_insert_select(self._h, _ptr(H), n, _ptr(payload), int(bool(require_consistency)),
+                                            SELECT_STRATEGIES[strategy], int(budget_total), int(budget_per_class),
+                                            _ptr(index), _ptr(radius), C.byref(got), _stream(self.device)))
+        return index, radius, got.value
 
     # -- Algorithm 2
     def probe(self, Q: torch.Tensor, out=None):

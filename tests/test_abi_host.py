@@ -65,6 +65,10 @@ def test_null_handle_calls(lib):
     nh, nc = C.c_int64(7), C.c_int64(7)
     assert lib.lipcache_consistency(None, None, 0, None, None, C.byref(nh), C.byref(nc), None) == 1
     assert nh.value == 0 and nc.value == 0
+    ns = C.c_int64(7)
+    assert lib.lipcache_insert_select(None, None, 0, None, 0, 1, 0, 0, None, None, C.byref(ns), None) == 1
+    assert ns.value == 0
+    assert lib.lipcache_set_radius_policy(None, 1, 1.0, None, None) == 1
 
 
 def test_create_without_gpu_fails_cleanly(lib):
