@@ -296,7 +296,7 @@ def test_empty_and_zero_sizes(dev, path):
 
 @pytest.mark.parametrize("path", PATHS)
 @pytest.mark.parametrize("d,C,N,B", [(20, 5, 300, 77), (33, 3, 1000, 130), (1, 2, 50, 10), (256, 7, 513, 129),
-                                     (96, 12, 2049, 300)])
+                                     (96, 12, 2049, 300), (64, 300, 700, 100), (160, 40, 900, 260)])
 def test_ragged_shapes(dev, path, d, C, N, B):
     w = synth.WORKLOADS["tiny"].scaled(d=d, C=C, components=C, N=N, n_queries=B, sphere_radius=3.0)
     W, b = synth.head(w)
@@ -371,4 +371,23 @@ def test_many_tied_runners_up(dev, mode):
     if mode == "conservative":
         assert n < len(rows)  # rows won by the tied group are skipped
     # (the tight radius skips classes with W_j = W_y, Eq. 29, so it keeps them)
+    cache.close()
+
+
+def test_large_dim_exact_path(dev):
+    """d = 1024 (the largest supported): the streaming certify kernel and the
+    exact probe; the tensor paths refuse d > 256."""
+    from paper_2608_13144_gb300._lib import LipCacheError
+    w = synth.WORKLOADS["tiny"].scaled(d=1024, C=12, components=12, N=600, n_queries=150, sphere_radius=6.0)
+    W, b = synth.head(w)
+    rows = synth.cache_rows(w)
+    Q, _ = synth.queries(w, rows)
+    cache, sigma = make_cache(dev, W, b, w.N)
+    idx, rad, n = cache.insert(T(rows, dev))
+    ref = oracle.build_cache(W, b, oracle.sigma_max(W), rows)
+    check_insert(idx.cpu().numpy(), rad.cpu().numpy(), n, ref, (W, b, rows, 1.0))
+    with pytest.raises(LipCacheError):
+        cache.set_probe_path("tensor")
+    gi, gl, gd = run_probe(cache, Q, dev, 64, "exact")
+    check_probe(gi, gl, gd, ref, Q, oracle.probe(ref["keys"], ref["radius"], ref["label"], Q))
     cache.close()
