@@ -1,0 +1,97 @@
+"""The 4M-entry scale workload at full size, in the launch configuration the
+benchmark times (insert batches of 65,536, probe batches of 4,096 on the
+default path), against the FP64 oracle on sampled outputs it can afford
+(pytest -m gpu)."""
+import numpy as np
+import pytest
+
+import oracle
+import synth
+from parity_utils import check_probe
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def scale():
+    if not torch.cuda.is_available():
+        pytest.skip("no GPU")
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2608_13144_gb300.lipcache import LipCache
+    dev = torch.device("cuda", 0)
+    w = synth.WORKLOADS["scale"]
+    W, b = synth.head(w)
+    rows = synth.cache_rows(w)
+    Q, src = synth.queries(w, rows)
+    cache = LipCache(w.d, w.C, w.N, device=dev)
+    sigma = cache.set_head(torch.from_numpy(W).to(dev), torch.from_numpy(b).to(dev))
+    rows_d = torch.from_numpy(rows).to(dev)
+    idx, rad = [], []
+    for s, e in synth.batches(w.N, w.insert_batch):
+        i, r, _ = cache.insert(rows_d[s:e])
+        idx.append(i.cpu().numpy())
+        rad.append(r.cpu().numpy())
+    del rows_d
+    ref = oracle.build_cache(W, b, oracle.sigma_max(W), rows)
+    yield dict(w=w, W=W, b=b, rows=rows, Q=Q, src=src, cache=cache, dev=dev, sigma=sigma,
+               g_index=np.concatenate(idx), g_radius=np.concatenate(rad), ref=ref)
+    cache.close()
+
+
+def test_scale_insert_full(scale):
+    """Every one of the 4M rows: acceptance and cache index bit-exact, radius
+    within 1e-5 (the oracle's FP64 certification of all rows)."""
+    s = scale
+    ref = s["ref"]
+    assert abs(s["sigma"] - oracle.sigma_max(s["W"])) <= 1e-10
+    np.testing.assert_array_equal(s["g_index"], ref["index"])
+    r = ref["cert"]["radius"]
+    m = np.isfinite(r) & (r > 0)
+    np.testing.assert_allclose(s["g_radius"][m], r[m], rtol=1e-5)
+    assert s["cache"].size == len(ref["keys"])
+
+
+def test_scale_probe_sampled(scale):
+    """One 4,096-query batch on the default path: every GPU hit is an exact
+    hit (FP64 distance below the FP64 radius), and 96 sampled queries (72
+    near-duplicates, 24 fresh draws) match the oracle's brute force over the
+    whole 4M-entry cache outside the 1e-5 band."""
+    s = scale
+    w, ref, Q = s["w"], s["ref"], s["Q"]
+    B = w.batch
+    q = Q[:B]
+    cache = s["cache"]
+    cache.set_probe_path("auto")
+    gi, gl, gd = [t.cpu().numpy() for t in cache.probe(torch.from_numpy(q).to(s["dev"]))]
+    assert cache.info()["device_errors"] == 0 and cache.info()["last_probe_path"] == 3
+    hits = gi >= 0
+    assert hits.sum() > 0
+    D = oracle.pair_dist(q, ref["keys"], np.nonzero(hits)[0], gi[hits])
+    assert np.all(D < ref["radius"][gi[hits]])
+    np.testing.assert_array_equal(gl[hits], ref["label"][gi[hits]])
+    rng = np.random.default_rng(3)
+    dup = np.nonzero(s["src"][:B] >= 0)[0]
+    fresh = np.nonzero(s["src"][:B] < 0)[0]
+    pick = np.sort(np.concatenate([rng.choice(dup, 72, replace=False), rng.choice(fresh, 24, replace=False)]))
+    orc = oracle.probe(ref["keys"], ref["radius"], ref["label"], q[pick])
+    check_probe(gi[pick], gl[pick], gd[pick], ref, q[pick], orc)
+
+
+def test_scale_tensor_equals_exact(scale):
+    """The same batch through the exact kernel (every pair on CUDA cores) and
+    both tensor kernels: bit-identical outputs at full size."""
+    s = scale
+    q = torch.from_numpy(s["Q"][: s["w"].batch]).to(s["dev"])
+    cache = s["cache"]
+    outs = {}
+    for path in ("exact", "tensor_single", "tensor_pair"):
+        cache.set_probe_path(path)
+        outs[path] = [t.cpu().numpy() for t in cache.probe(q)]
+        assert cache.info()["device_errors"] == 0
+    cache.set_probe_path("auto")
+    for path in ("tensor_single", "tensor_pair"):
+        for x, y in zip(outs["exact"], outs[path]):
+            assert np.array_equal(x.view(np.uint8) if x.dtype == np.float32 else x,
+                                  y.view(np.uint8) if y.dtype == np.float32 else y), path
