@@ -534,6 +534,13 @@ __global__ void __launch_bounds__(kThreads) k_certify(CertArgs a) {
 //     lowest class) and runs the FP64 finals. A row with more than
 //     kMaxCand candidates is redone by one warp with warp_row_refine.
 //     The tight radius runs certify_row (FP64) with one warp per row.
+// Start moving `bytes` (a multiple of 16) from global memory at `src` (16-byte
+// aligned) into L2, without waiting.
+__device__ __forceinline__ void prefetch_l2_bulk(const void* src, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(reinterpret_cast<uint64_t>(src)), "r"(bytes)
+               : "memory");
+}
+
 constexpr int kWTile = 64;    // rows per tile
 constexpr int kHStride = 68;  // h^T row stride (floats): 16-byte aligned, banks spread
 constexpr int kMaxCand = 16;  // candidate slots per row
@@ -633,6 +640,13 @@ __global__ void __launch_bounds__(kThreads, 1) k_certify_wres(CertArgs a, int Cp
     const int nrows = (int)(a.n - row0 < kWTile ? a.n - row0 : kWTile);
     __syncthreads();  // previous tile done with hT / lg / ts (and wT written on the first pass)
     load_tile(a, row0, nrows, dpad, hT, tid, vec != 0);
+    // the next tile's rows (contiguous) start moving into L2 now, so its load
+    // phase reads L2 instead of waiting on DRAM
+    if (vec && tid == 0 && tile + (int)gridDim.x < n_tiles) {
+      const int64_t r1 = (int64_t)(tile + gridDim.x) * kWTile;
+      const int64_t n1 = a.n - r1 < kWTile ? a.n - r1 : kWTile;
+      prefetch_l2_bulk(a.H + (size_t)r1 * d, (uint32_t)(n1 * d * sizeof(float)));
+    }
     if (tid < kWTile) {
       ts.acc_flag[tid] = 0;
       ts.ncand[tid] = 0;
