@@ -55,9 +55,10 @@ def test_scale_insert_full(scale):
 
 def test_scale_probe_sampled(scale):
     """One 4,096-query batch on the default path: every GPU hit is an exact
-    hit (FP64 distance below the FP64 radius), and 96 sampled queries (72
-    near-duplicates, 24 fresh draws) match the oracle's brute force over the
-    whole 4M-entry cache outside the 1e-5 band."""
+    hit (FP64 distance below the FP64 radius), and every near-duplicate query
+    of the batch (where the hits are) plus 128 fresh draws match the
+    oracle's brute force over the whole 4M-entry cache outside the 1e-5
+    band."""
     s = scale
     w, ref, Q = s["w"], s["ref"], s["Q"]
     B = w.batch
@@ -74,7 +75,7 @@ def test_scale_probe_sampled(scale):
     rng = np.random.default_rng(3)
     dup = np.nonzero(s["src"][:B] >= 0)[0]
     fresh = np.nonzero(s["src"][:B] < 0)[0]
-    pick = np.sort(np.concatenate([rng.choice(dup, 72, replace=False), rng.choice(fresh, 24, replace=False)]))
+    pick = np.sort(np.concatenate([dup, rng.choice(fresh, 128, replace=False)]))
     orc = oracle.probe(ref["keys"], ref["radius"], ref["label"], q[pick])
     check_probe(gi[pick], gl[pick], gd[pick], ref, q[pick], orc)
 
