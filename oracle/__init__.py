@@ -15,6 +15,7 @@ Functions (each follows the passage cited in the C source):
   global_radius                 one global threshold for every entry (Sec. 5.4)
   select_radius_dedup           selection S: radius-prioritised de-duplication (Algorithm 1, Sec. 5.5)
   radius_rz32                   FP32 radius rounded toward zero (the order key of the selection)
+  select_kcenter                selection S: K-center per class (Sec. 5.5)
   pair_dist                     ||q - k||_2 for given pairs
 """
 from __future__ import annotations
@@ -301,6 +302,45 @@ def select_radius_dedup(rows, cert, keys0=None, radius0=None, budget_total=0, bu
         m += 1
         per[c] = per.get(c, 0) + 1
     return np.asarray(out, dtype=np.int64)
+
+
+def select_kcenter(rows, cert, budget_per_class, n_classes) -> dict:
+    """Selection strategy S read as K-center (the alternative named in
+    Sec. 5.5; no formula given): for each class c (payload label in [0, C))
+    among the certified candidates, Gonzalez's farthest-point greedy: the
+    first centre is the candidate with the largest certified radius, each
+    next one the candidate farthest (Euclidean, FP64) from the centres chosen
+    so far; ties go to the lower row; stop at budget_per_class centres or
+    when the class is exhausted. Returns the selected rows (classes in
+    ascending order, each class in selection order) and, per step, the
+    relative gap between the chosen candidate's distance and the runner-up's
+    (to tell near-ties apart)."""
+    rows = np.asarray(rows, dtype=np.float32)
+    acc = np.asarray(cert["accept"], dtype=bool)
+    lab = np.asarray(cert["label"], dtype=np.int64)
+    rad = np.asarray(cert["radius"], dtype=np.float64)
+    out, gaps = [], []
+    for c in range(int(n_classes)):
+        cand = np.nonzero(acc & (lab == c))[0]
+        if len(cand) == 0 or budget_per_class <= 0:
+            continue
+        Z = rows[cand].astype(np.float64)
+        r = rad[cand]
+        first = int(np.lexsort((cand, -r))[0])  # largest radius, then lowest row
+        chosen = [first]
+        mind = np.sqrt(np.sum((Z - Z[first]) ** 2, axis=1))
+        mind[first] = -1.0
+        while len(chosen) < min(budget_per_class, len(cand)):
+            best = float(mind.max())
+            j = int(np.nonzero(mind == best)[0][0])  # candidates are in row order: lowest row on ties
+            rest = np.delete(mind, j)
+            second = float(rest.max()) if len(rest) else -1.0
+            gaps.append((best - second) / best if best > 0 else 0.0)
+            chosen.append(j)
+            mind = np.minimum(mind, np.sqrt(np.sum((Z - Z[j]) ** 2, axis=1)))
+            mind[chosen] = -1.0
+        out.extend(cand[chosen].tolist())
+    return {"selected": np.asarray(out, dtype=np.int64), "gaps": np.asarray(gaps)}
 
 
 def pair_dist(Q, K, qi, ki) -> np.ndarray:

@@ -245,3 +245,37 @@ def test_radius_rz32_rounds_toward_zero():
     with np.errstate(over="ignore"):
         nxt = np.nextafter(f[:6], np.float32(np.inf)).astype(np.float64)
     assert np.all(nxt > r[:6])  # the largest FP32 value not above r
+
+
+def test_golden_select_kcenter():
+    g = golden("select_kcenter.json")
+    W, b = np.array(g["W"], np.float32), np.array(g["b"], np.float32)
+    rows = np.array(g["rows"], np.float32)
+    cert = oracle.certify(W, b, g["sigma"], rows)
+    assert oracle.select_kcenter(rows, cert, 3, 2)["selected"].tolist() == g["budget_3"]
+    assert oracle.select_kcenter(rows, cert, 1, 2)["selected"].tolist() == g["budget_1"]
+    tie = np.array(g["tie_rows"], np.float32)
+    ct = oracle.certify(W, b, g["sigma"], tie)
+    assert oracle.select_kcenter(tie, ct, 2, 2)["selected"].tolist() == g["tie_budget_2"]
+
+
+@pytest.mark.parametrize("seed,C,d,k", [(0, 3, 2, 5), (1, 4, 3, 8), (2, 2, 5, 20)])
+def test_select_kcenter_farthest_point(seed, C, d, k):
+    """Brute force: per class the first centre has the largest radius and
+    every next centre is at least as far from the earlier centres as any
+    other candidate; a class with fewer candidates than the budget keeps all."""
+    rng, W, b, rows = _instance(seed, C, d, 200, 0)
+    cert = oracle.certify(W, b, oracle.sigma_max(W), rows)
+    sel = oracle.select_kcenter(rows, cert, k, C)["selected"]
+    for c in range(C):
+        cand = np.nonzero(cert["accept"] & (cert["label"] == c))[0]
+        mine = [i for i in sel.tolist() if cert["label"][i] == c]
+        assert len(mine) == min(k, len(cand))
+        if not mine:
+            continue
+        assert cert["radius"][mine[0]] == cert["radius"][cand].max()
+        for t in range(1, len(mine)):
+            centres = rows[mine[:t]].astype(np.float64)
+            dmin = lambda i: np.min(np.linalg.norm(centres - rows[i].astype(np.float64), axis=1))
+            others = [i for i in cand if i not in mine[:t]]
+            assert dmin(mine[t]) >= max(dmin(i) for i in others) - 1e-12
