@@ -183,6 +183,7 @@ lipcache_status lipcache_probe(lipcache_t* h, const float* Q, int64_t B, int64_t
 /* Selection strategies S (Algorithm 1, last steps; lipcache_insert_select). */
 #define LIPCACHE_SELECT_ALL 0          /* every certified candidate, in input order (= lipcache_insert) */
 #define LIPCACHE_SELECT_RADIUS_DEDUP 1 /* radius-prioritised de-duplication (Sec. 5.5) */
+#define LIPCACHE_SELECT_KCENTER 2      /* K-center per class (Sec. 5.5) */
 
 /*
  * Algorithm 1 with a selection strategy S: certify the n candidate rows as
@@ -198,6 +199,13 @@ lipcache_status lipcache_probe(lipcache_t* h, const float* Q, int64_t B, int64_t
  *   is the probe's conservative one, so a skipped row is always exactly
  *   covered; a row within ~2e-6 relative of a ball's boundary may be kept
  *   where exact arithmetic would skip it.
+ *   LIPCACHE_SELECT_KCENTER (the alternative Sec. 5.5 names): per class
+ *   (payload label in [0, C); other labels are not selected), Gonzalez's
+ *   farthest-point greedy over the class's certified candidates: first the
+ *   largest radius, then repeatedly the candidate farthest from the centres
+ *   so far (canonical FP32 squared distance; ties to the lower row), up to
+ *   budget_per_class (required > 0; budget_total must be 0). Appended class
+ *   by class in selection order. Cost: centres x class size x d per class.
  *   LIPCACHE_SELECT_ALL: lipcache_insert (budgets must be 0).
  *   budget_total, budget_per_class   <= 0: unlimited
  *   out_index    n int64 (device), nullable: cache index of a kept row, else -1
@@ -206,8 +214,9 @@ lipcache_status lipcache_probe(lipcache_t* h, const float* Q, int64_t B, int64_t
  * Requires the certified radius policy (the coverage test uses the certified
  * balls). Synchronises `stream` (once per 4,096 candidates). All or nothing
  * on capacity: E_FULL, before any work, if size + min(n, budget_total)
- * exceeds it. Errors: those of lipcache_insert and lipcache_probe; E_STATE
- * under an empirical radius policy; E_INVALID for an unknown strategy.
+ * exceeds it (K-center: min(n, C x budget_per_class)). Errors: those of
+ * lipcache_insert and lipcache_probe; E_STATE under an empirical radius
+ * policy; E_INVALID for an unknown strategy or budgets it does not take.
  */
 lipcache_status lipcache_insert_select(lipcache_t* h, const float* H, int64_t n, const int32_t* payload,
                                        int32_t require_consistency, int32_t strategy, int64_t budget_total,

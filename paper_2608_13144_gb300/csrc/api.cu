@@ -291,8 +291,11 @@ LC_API lipcache_status lipcache_insert_select(lipcache_t* h, const float* H, int
   if (n_selected) *n_selected = 0;
   return guarded([&] {
     check_handle(h);
-    LC_REQUIRE(strategy == LIPCACHE_SELECT_ALL || strategy == LIPCACHE_SELECT_RADIUS_DEDUP, LIPCACHE_E_INVALID,
-               "unknown selection strategy");
+    LC_REQUIRE(strategy == LIPCACHE_SELECT_ALL || strategy == LIPCACHE_SELECT_RADIUS_DEDUP ||
+                   strategy == LIPCACHE_SELECT_KCENTER,
+               LIPCACHE_E_INVALID, "unknown selection strategy");
+    LC_REQUIRE(strategy != LIPCACHE_SELECT_KCENTER || (budget_per_class > 0 && budget_total <= 0), LIPCACHE_E_INVALID,
+               "K-center takes a per-class budget and no total budget");
     if (strategy == LIPCACHE_SELECT_ALL) {
       LC_REQUIRE(budget_total <= 0 && budget_per_class <= 0, LIPCACHE_E_INVALID,
                  "LIPCACHE_SELECT_ALL takes no budget");
@@ -308,12 +311,17 @@ LC_API lipcache_status lipcache_insert_select(lipcache_t* h, const float* H, int
     if (n == 0) return;
     LC_REQUIRE(H != nullptr, LIPCACHE_E_INVALID, "H is NULL");
     LC_REQUIRE(((uintptr_t)H & 3) == 0, LIPCACHE_E_INVALID, "H must be 4-byte aligned");
-    const int64_t most = budget_total > 0 && budget_total < n ? budget_total : n;
+    int64_t most = budget_total > 0 && budget_total < n ? budget_total : n;
+    if (strategy == LIPCACHE_SELECT_KCENTER && (int64_t)budget_per_class * h->C < most)
+      most = (int64_t)budget_per_class * h->C;
     LC_REQUIRE(most <= h->capacity - h->size, LIPCACHE_E_FULL, "the selection could exceed the cache capacity");
     use_device(h);
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-    const int64_t kept = lc::select_insert(h, H, n, payload, require_consistency, budget_total, budget_per_class,
-                                           out_index, out_radius, s);
+    const int64_t kept =
+        strategy == LIPCACHE_SELECT_KCENTER
+            ? lc::select_kcenter(h, H, n, payload, require_consistency, budget_per_class, out_index, out_radius, s)
+            : lc::select_insert(h, H, n, payload, require_consistency, budget_total, budget_per_class, out_index,
+                                out_radius, s);
     LC_CUDA(cudaStreamSynchronize(s));
     if (n_selected) *n_selected = kept;
   });

@@ -133,6 +133,8 @@ struct SelectScratch {
   int64_t list_cap = 0;
   int32_t* class_cnt = nullptr;
   int64_t class_cap = 0;
+  float* kc_mind = nullptr;  // K-center: squared distance to the nearest centre
+  int64_t kc_mind_cap = 0;
   int64_t* small = nullptr;       // device: accepted, kept, chunk count
   int64_t* small_host = nullptr;  // pinned
 };
@@ -266,6 +268,9 @@ void certify_rows(lipcache* h, const float* H, int64_t n, const int32_t* payload
 int64_t select_insert(lipcache* h, const float* H, int64_t n, const int32_t* payload, int require_consistency,
                       int64_t budget_total, int budget_per_class, int64_t* out_index, float* out_radius,
                       cudaStream_t s);
+// select.cu: K-center per class (at most budget_per_class centres per class)
+int64_t select_kcenter(lipcache* h, const float* H, int64_t n, const int32_t* payload, int require_consistency,
+                       int budget_per_class, int64_t* out_index, float* out_radius, cudaStream_t s);
 void release_select(lipcache* h);
 // Certified-consistency check: argmax of the head on Q against y^G of the hit
 // entries; counts (hits, consistent, invalid index) land in ins_total[1..3].

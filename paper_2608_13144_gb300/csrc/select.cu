@@ -1,5 +1,6 @@
-// Selection strategy S of Algorithm 1: radius-prioritised de-duplication
-// (the default strategy of Sec. 5.5).
+// Selection strategies S of Algorithm 1 (Sec. 5.5): radius-prioritised
+// de-duplication (the paper's default) and K-center per class (at the end
+// of the file).
 //
 // The candidates that Algorithm 1 accepts are visited in order of decreasing
 // certified radius (the FP32 radius, ties to the lower row). A candidate is
@@ -245,6 +246,162 @@ __global__ void k_copy_f32(const float* __restrict__ s, float* __restrict__ d, i
   if (i < n) d[i] = s[i];
 }
 
+// ---------------------------------------------------------------- K-center
+// Per class (payload label in [0, C)) among the certified candidates:
+// Gonzalez's farthest-point greedy, first centre the largest radius, ties to
+// the lower row, at most budget_per_class centres. The candidates are sorted
+// by (label, row); one block per class walks its segment once per centre
+// (cost: centres x class size x d). Distances are the canonical FP32 squared
+// distance, so near-ties (~1e-6 relative) may resolve differently from an
+// FP64 evaluation.
+// Sort key of the per-class K-center: label, then row; others last.
+__global__ void k_kc_keys(const uint8_t* __restrict__ accept, const int32_t* __restrict__ label, int64_t n,
+                          int64_t npow, int C, unsigned long long* __restrict__ keys, int64_t* __restrict__ n_acc) {
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= npow) return;
+  unsigned long long k = ~0ull;
+  bool in = false;
+  if (i < n && accept[i] && label[i] >= 0 && label[i] < C) {
+    in = true;
+    k = ((unsigned long long)(uint32_t)label[i] << 32) | (unsigned long long)(uint32_t)i;
+  }
+  keys[i] = k;
+  const unsigned m = __ballot_sync(0xffffffffu, in);
+  if ((threadIdx.x & 31) == 0 && m) atomicAdd(reinterpret_cast<unsigned long long*>(n_acc), (unsigned long long)__popc(m));
+}
+
+// Class segments [seg[2c], seg[2c+1]) of the sorted keys (zero-initialised).
+__global__ void k_kc_segments(const unsigned long long* __restrict__ keys, int64_t n_acc, int32_t* __restrict__ seg) {
+  const int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (p >= n_acc) return;
+  const uint32_t c = (uint32_t)(keys[p] >> 32);
+  if (p == 0 || (uint32_t)(keys[p - 1] >> 32) != c) seg[2 * c] = (int32_t)p;
+  if (p == n_acc - 1 || (uint32_t)(keys[p + 1] >> 32) != c) seg[2 * c + 1] = (int32_t)(p + 1);
+}
+
+constexpr int kKcThreads = 256;
+
+__device__ __forceinline__ unsigned long long block_max_u64(unsigned long long v, unsigned long long* red) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const unsigned long long w = __shfl_xor_sync(0xffffffffu, v, o);
+    v = w > v ? w : v;
+  }
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  __syncthreads();
+  if (lane == 0) red[warp] = v;
+  __syncthreads();
+  unsigned long long m = red[0];
+  for (int w = 1; w < kKcThreads / 32; ++w) m = red[w] > m ? red[w] : m;
+  return m;
+}
+
+// Gonzalez's farthest-point greedy for one class per block: first the
+// candidate of largest radius, then repeatedly the one farthest (canonical
+// FP32 squared distance) from the centres so far; ties to the lower row.
+// mind[p] holds each segment member's squared distance to the nearest centre
+// (negative once chosen); the chosen rows go to out[s0 ..] in order.
+__global__ void __launch_bounds__(kKcThreads) k_kcenter(const unsigned long long* __restrict__ keys,
+                                                        const int32_t* __restrict__ seg, const float* __restrict__ H,
+                                                        int d, const float* __restrict__ radius, int budget,
+                                                        float* __restrict__ mind, int32_t* __restrict__ out,
+                                                        int32_t* __restrict__ cnt) {
+  extern __shared__ float zc[];  // the newest centre's features (d)
+  __shared__ unsigned long long red[kKcThreads / 32];
+  const int c = blockIdx.x, tid = threadIdx.x;
+  const int s0 = seg[2 * c], s1 = seg[2 * c + 1];
+  const int nc = s1 - s0;
+  if (nc <= 0) {
+    if (tid == 0) cnt[c] = 0;
+    return;
+  }
+  unsigned long long best = 0ull;
+  for (int p = s0 + tid; p < s1; p += kKcThreads) {
+    const uint32_t row = (uint32_t)(keys[p] & 0xFFFFFFFFull);
+    const unsigned long long k = ((unsigned long long)__float_as_uint(radius[row]) << 32) | (0xFFFFFFFFu - row);
+    best = k > best ? k : best;
+    mind[p] = INFINITY;
+  }
+  best = block_max_u64(best, red);
+  const int want = budget < nc ? budget : nc;
+  for (int t = 0; t < want; ++t) {
+    const uint32_t row = 0xFFFFFFFFu - (uint32_t)(best & 0xFFFFFFFFull);
+    if (tid == 0) out[s0 + t] = (int32_t)row;
+    for (int j = tid; j < d; j += kKcThreads) zc[j] = H[(size_t)row * d + j];
+    __syncthreads();
+    if (t + 1 == want) break;
+    best = 0ull;
+    for (int p = s0 + tid; p < s1; p += kKcThreads) {
+      const uint32_t r = (uint32_t)(keys[p] & 0xFFFFFFFFull);
+      float m = mind[p];
+      if (r == row) m = -1.f;  // chosen
+      if (m >= 0.f) {
+        const float* z = H + (size_t)r * d;
+        float total = 0.f;
+        for (int c0 = 0; c0 < d; c0 += 32) {
+          float q = 0.f;
+          const int ce = c0 + 32 < d ? c0 + 32 : d;
+          for (int j = c0; j < ce; ++j) {
+            const float e = __fsub_rn(z[j], zc[j]);
+            q = __fmaf_rn(e, e, q);
+          }
+          total = __fadd_rn(total, q);
+        }
+        m = fminf(m, total);
+        const unsigned long long k = ((unsigned long long)__float_as_uint(m) << 32) | (0xFFFFFFFFu - r);
+        best = k > best ? k : best;
+      }
+      mind[p] = m;
+    }
+    best = block_max_u64(best, red);
+  }
+  if (tid == 0) cnt[c] = want;
+}
+
+// Append the centres class by class (offsets = exclusive scan of cnt).
+__global__ void k_kc_scatter(const int32_t* __restrict__ seg, const int32_t* __restrict__ cnt,
+                             const int32_t* __restrict__ off, const int32_t* __restrict__ out, const float* __restrict__ H,
+                             int d, int dpad, int64_t size0, const float* __restrict__ rr, const float* __restrict__ tau,
+                             const float* __restrict__ kn, const float* __restrict__ radius,
+                             const int32_t* __restrict__ label, const int32_t* __restrict__ yG, Table t,
+                             int64_t* __restrict__ out_index) {
+  const int c = blockIdx.y;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  for (int q = blockIdx.x * 8 + warp; q < cnt[c]; q += gridDim.x * 8) {
+    const int32_t row = out[seg[2 * c] + q];
+    const int64_t dst = size0 + off[c] + q;
+    float* kd = t.keys + (size_t)dst * dpad;
+    for (int j = lane; j < dpad; j += 32) kd[j] = j < d ? H[(size_t)row * d + j] : 0.f;
+    if (lane == 0) {
+      t.rr[dst] = rr[row];
+      t.tau[dst] = tau[row];
+      t.kn[dst] = kn[row];
+      t.radius[dst] = radius[row];
+      t.label[dst] = label[row];
+      t.yG[dst] = yG[row];
+      if (out_index) out_index[row] = dst;
+    }
+  }
+}
+
+// Exclusive scan of C counts (C <= 1024), total in *total.
+__global__ void __launch_bounds__(1024) k_kc_scan(const int32_t* __restrict__ cnt, int C, int32_t* __restrict__ off,
+                                                  int64_t* __restrict__ total) {
+  __shared__ int32_t buf[1024];
+  const int t = threadIdx.x;
+  const int v = t < C ? cnt[t] : 0;
+  buf[t] = v;
+  __syncthreads();
+  for (int s = 1; s < 1024; s <<= 1) {
+    const int x = t >= s ? buf[t - s] : 0;
+    __syncthreads();
+    buf[t] += x;
+    __syncthreads();
+  }
+  if (t < C) off[t] = buf[t] - v;
+  if (t == 1023) *total = buf[1023];
+}
+
 template <typename T>
 void grow_to(T*& p, int64_t& cap, int64_t n) {
   if (n <= cap) return;
@@ -353,6 +510,67 @@ int64_t select_insert(lipcache* h, const float* H, int64_t n, const int32_t* pay
   return kept;
 }
 
+int64_t select_kcenter(lipcache* h, const float* H, int64_t n, const int32_t* payload, int require_consistency,
+                       int budget_per_class, int64_t* out_index, float* out_radius, cudaStream_t s) {
+  SelectScratch& x = h->sel;
+  const int C = h->C;
+  certify_rows(h, H, n, payload, require_consistency, s);
+  const unsigned nb = (unsigned)((n + 255) / 256);
+  if (out_index) {
+    k_fill_i64<<<nb, 256, 0, s>>>(out_index, n, -1);
+    LC_LAUNCH_CHECK("k_fill_i64");
+  }
+  if (out_radius) {
+    k_copy_f32<<<nb, 256, 0, s>>>(h->ins_radius, out_radius, n);
+    LC_LAUNCH_CHECK("k_copy_f32");
+  }
+  int64_t npow = 1;
+  while (npow < n) npow <<= 1;
+  grow_to(x.keys, x.keys_cap, npow);
+  if (!x.small) {
+    LC_CUDA(cudaMalloc(&x.small, sizeof(int64_t) * 4));
+    LC_CUDA(cudaMallocHost(&x.small_host, sizeof(int64_t) * 4));
+  }
+  LC_CUDA(cudaMemsetAsync(x.small, 0, sizeof(int64_t) * 4, s));
+  const unsigned npb = (unsigned)((npow + 255) / 256);
+  k_kc_keys<<<npb, 256, 0, s>>>(h->ins_accept, h->ins_label, n, npow, C, x.keys, x.small);
+  LC_LAUNCH_CHECK("k_kc_keys");
+  for (int64_t k = 2; k <= npow; k <<= 1)
+    for (int64_t j = k >> 1; j > 0; j >>= 1) {
+      k_bitonic<<<npb, 256, 0, s>>>(x.keys, npow, j, k);
+      LC_LAUNCH_CHECK("k_bitonic");
+    }
+  LC_CUDA(cudaMemcpyAsync(x.small_host, x.small, sizeof(int64_t), cudaMemcpyDeviceToHost, s));
+  LC_CUDA(cudaStreamSynchronize(s));
+  const int64_t n_in = x.small_host[0];
+  if (n_in == 0) return 0;
+  // per-class segments, counts and offsets share one int32 scratch: seg[2C], cnt[C], off[C]
+  grow_to(x.list, x.list_cap, 4 * (int64_t)C + 1);
+  int32_t* seg = x.list;
+  int32_t* cnt = seg + 2 * C;
+  int32_t* off = cnt + C;
+  LC_CUDA(cudaMemsetAsync(seg, 0, sizeof(int32_t) * 2 * C, s));
+  k_kc_segments<<<(unsigned)((n_in + 255) / 256), 256, 0, s>>>(x.keys, n_in, seg);
+  LC_LAUNCH_CHECK("k_kc_segments");
+  grow_to(x.kc_mind, x.kc_mind_cap, n_in);
+  grow_to(x.rows, x.rows_cap, n_in);
+  k_kcenter<<<C, kKcThreads, sizeof(float) * (size_t)h->d, s>>>(x.keys, seg, H, h->d, h->ins_radius, budget_per_class,
+                                                                x.kc_mind, x.rows, cnt);
+  LC_LAUNCH_CHECK("k_kcenter");
+  k_kc_scan<<<1, 1024, 0, s>>>(cnt, C, off, x.small + 1);
+  LC_LAUNCH_CHECK("k_kc_scan");
+  const int per = budget_per_class;
+  k_kc_scatter<<<dim3((unsigned)((per + 7) / 8 < 64 ? (per + 7) / 8 : 64), (unsigned)C), 256, 0, s>>>(
+      seg, cnt, off, x.rows, H, h->d, h->dpad, h->size, h->ins_rr, h->ins_tau, h->ins_kn, h->ins_radius,
+      h->ins_label, h->ins_yG, h->table, out_index);
+  LC_LAUNCH_CHECK("k_kc_scatter");
+  LC_CUDA(cudaMemcpyAsync(x.small_host + 1, x.small + 1, sizeof(int64_t), cudaMemcpyDeviceToHost, s));
+  LC_CUDA(cudaStreamSynchronize(s));
+  const int64_t kept = x.small_host[1];
+  h->size += kept;
+  return kept;
+}
+
 void release_select(lipcache* h) {
   SelectScratch& x = h->sel;
   cudaFree(x.keys);
@@ -362,6 +580,7 @@ void release_select(lipcache* h) {
   cudaFree(x.cov);
   cudaFree(x.list);
   cudaFree(x.class_cnt);
+  cudaFree(x.kc_mind);
   cudaFree(x.small);
   if (x.small_host) cudaFreeHost(x.small_host);
   x = SelectScratch{};

@@ -18,7 +18,7 @@ RADIUS_MODES = {"conservative": _lib.RADIUS_CONSERVATIVE, "tight": _lib.RADIUS_T
 PROBE_PATHS = {"auto": _lib.PROBE_AUTO, "tensor": _lib.PROBE_TENSOR, "exact": _lib.PROBE_EXACT,
                "tensor_single": _lib.PROBE_TENSOR_SINGLE, "tensor_pair": _lib.PROBE_TENSOR_PAIR}
 RADIUS_POLICIES = {"certified": 0, "global": 1, "interclass": 2}
-SELECT_STRATEGIES = {"all": 0, "radius_dedup": 1}
+SELECT_STRATEGIES = {"all": 0, "radius_dedup": 1, "kcenter": 2}
 
 
 def _stream(device: torch.device):
@@ -95,8 +95,9 @@ class LipCache:
     def insert_select(self, H: torch.Tensor, payload: torch.Tensor | None = None, require_consistency: bool = False,
                       strategy: str = "radius_dedup", budget_total: int = 0, budget_per_class: int = 0):
         """Algorithm 1 with a selection strategy S ("radius_dedup": radius-
-        prioritised de-duplication; "all": insert). Returns (index, radius,
-        n_selected); index[i] is the cache index of row i or -1."""
+        prioritised de-duplication; "kcenter": K-center per class; "all":
+        insert). Returns (index, radius, n_selected); index[i] is the cache
+        index of row i or -1."""
         H = self._dev(H, torch.float32, "H")
         n = H.shape[0]
         if H.dim() != 2 or (n and H.shape[1] != self.d):

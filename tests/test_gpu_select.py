@@ -189,3 +189,82 @@ def test_select_errors_and_all(dev):
     assert n1 == n2 and torch.equal(i1, i2) and torch.equal(r1, r2)
     c1.close()
     c2.close()
+
+
+# ---------------------------------------------------------------- K-center
+def test_golden_kcenter(dev):
+    g = golden("select_kcenter.json")
+    W, b = np.array(g["W"], np.float32), np.array(g["b"], np.float32)
+    rows = np.array(g["rows"], np.float32)
+    for k, key in ((3, "budget_3"), (1, "budget_1")):
+        cache = make_cache(dev, W, b, 16)
+        idx, _, n = cache.insert_select(T(rows, dev), strategy="kcenter", budget_per_class=k)
+        assert kept_in_order(idx.cpu().numpy()).tolist() == g[key] and n == len(g[key])
+        cache.close()
+    tie = np.array(g["tie_rows"], np.float32)
+    cache = make_cache(dev, W, b, 16)
+    idx, _, n = cache.insert_select(T(tie, dev), strategy="kcenter", budget_per_class=2)
+    assert kept_in_order(idx.cpu().numpy()).tolist() == g["tie_budget_2"]
+    cache.close()
+
+
+@pytest.mark.parametrize("name,n,k", [("tiny", 1024, 20), ("cifar10", 6000, 50), ("cifar100", 5000, 10),
+                                      ("tinyimagenet", 4000, 5)])
+def test_kcenter_workload(dev, name, n, k):
+    """Per class the GPU's centres are a farthest-point sequence (each at
+    least (1 - 1e-5) as far from the earlier centres as any other candidate,
+    FP64), the first has the class's largest radius, and the whole selection
+    equals the oracle's whenever no step was a near-tie."""
+    w = synth.WORKLOADS[name]
+    W, b = synth.head(w)
+    rows = _pool(w, n, 11)
+    cert = oracle.certify(W, b, oracle.sigma_max(W), rows)
+    cache = make_cache(dev, W, b, n)
+    idx, rad, got = cache.insert_select(T(rows, dev), strategy="kcenter", budget_per_class=k)
+    idx = idx.cpu().numpy()
+    sel = kept_in_order(idx)
+    assert got == len(sel)
+    ref = oracle.select_kcenter(rows, cert, k, w.C)
+    for c in range(w.C):
+        cand = np.nonzero(cert["accept"] & (cert["label"] == c))[0]
+        mine = [i for i in sel.tolist() if cert["label"][i] == c]
+        assert len(mine) == min(k, len(cand))
+        if not mine:
+            continue
+        assert cert["radius"][mine[0]] >= cert["radius"][cand].max() * (1 - 1e-6)
+        Z = rows[cand].astype(np.float64)
+        mind = np.full(len(cand), np.inf)
+        pos = {r: j for j, r in enumerate(cand.tolist())}
+        for t, r in enumerate(mine):
+            if t:
+                avail = np.ones(len(cand), bool)
+                avail[[pos[x] for x in mine[:t]]] = False
+                assert mind[pos[r]] >= mind[avail].max() * (1 - 1e-5)
+            mind = np.minimum(mind, np.linalg.norm(Z - Z[pos[r]], axis=1))
+    # classes come out in ascending order
+    labs = cert["label"][sel]
+    assert np.all(np.diff(labs) >= 0)
+    if len(ref["gaps"]) == 0 or ref["gaps"].min() > 1e-5:
+        np.testing.assert_array_equal(sel, ref["selected"])
+    # the kept entries carry their certified radii
+    gi, _, gd = cache.probe(T(rows[sel], dev))
+    assert np.array_equal(gi.cpu().numpy(), idx[sel]) or np.all(gd.cpu().numpy() == 0)
+    cache.close()
+
+
+def test_kcenter_errors(dev):
+    from paper_2608_13144_gb300._lib import LipCacheError
+    w = synth.WORKLOADS["tiny"]
+    W, b = synth.head(w)
+    rows = synth.cache_rows(w)[:100]
+    cache = make_cache(dev, W, b, 1000)
+    for kw in ({}, {"budget_per_class": 0}, {"budget_per_class": 2, "budget_total": 5}):
+        with pytest.raises(LipCacheError) as e:
+            cache.insert_select(T(rows, dev), strategy="kcenter", **kw)
+        assert e.value.status == 1
+    small = make_cache(dev, W, b, 15)
+    with pytest.raises(LipCacheError) as e:
+        small.insert_select(T(rows, dev), strategy="kcenter", budget_per_class=2)  # 10 classes x 2 > 15
+    assert e.value.status == 4
+    cache.close()
+    small.close()
