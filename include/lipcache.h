@@ -241,7 +241,9 @@ lipcache_status lipcache_insert_select(lipcache_t* h, const float* H, int64_t n,
  *   n_inserted    host, nullable: number of entries appended
  * Synchronises `stream`. All or nothing: if size + B > capacity nothing is
  * probed or written and E_FULL is returned (the number of misses is not known
- * in advance). Errors: those of lipcache_probe and lipcache_insert.
+ * in advance). Errors: those of lipcache_probe and lipcache_insert;
+ * E_DEVICE if a bounded wait of the probe kernel expired (the probe outputs
+ * then report misses and nothing is written back).
  */
 lipcache_status lipcache_probe_writeback(lipcache_t* h, const float* Q, int64_t B, const int32_t* payload,
                                          int32_t require_consistency, int64_t* out_index, int32_t* out_label,
@@ -297,10 +299,25 @@ lipcache_status lipcache_set_radius_policy(lipcache_t* h, int32_t policy, double
                                            lipcache_stream_t stream);
 
 /*
+ * Test hooks for failure detection. LIPCACHE_DEBUG_STALL_PROBE makes the MMA
+ * issuer of the tensor probe kernels first wait on an mbarrier that nothing
+ * arrives on: the bounded wait (~2^31 cycles, about a second) expires, the
+ * kernel takes its abort path (no trap, no hang), the batch's queries come
+ * back as misses, lipcache_info.device_errors counts the aborted CTAs, and
+ * the synchronous entry points (lipcache_probe_host, _probe_writeback)
+ * return LIPCACHE_E_DEVICE. The exact kernel has no waits and is unaffected.
+ * flags = 0 restores normal operation. Errors: E_INVALID (unknown bits).
+ */
+#define LIPCACHE_DEBUG_STALL_PROBE 1
+lipcache_status lipcache_set_debug(lipcache_t* h, int32_t flags);
+
+/*
  * lipcache_probe for callers holding HOST buffers: copies Q to the device,
  * probes, copies the results back and synchronises `stream`.
  *   Q_host     B x d FP32 (host; pinned memory gives asynchronous copies)
  *   out_*_host host, same meaning as lipcache_probe (out_label/out_dist nullable)
+ * Returns LIPCACHE_E_DEVICE (outputs written: all misses) if a bounded wait
+ * of the probe kernel expired during the call.
  */
 lipcache_status lipcache_probe_host(lipcache_t* h, const float* Q_host, int64_t B, int64_t* out_index_host,
                                     int32_t* out_label_host, float* out_dist_host, lipcache_stream_t stream);

@@ -138,6 +138,14 @@ void lc::harvest_timing(lipcache* h, bool all) {
   }
 }
 
+// After a synchronised probe: E_DEVICE if a bounded wait of the kernel expired.
+static void require_no_abort(lipcache* h, cudaStream_t s) {
+  LC_CUDA(cudaMemcpyAsync(h->stats_host, h->stats, sizeof(lc::DevStats), cudaMemcpyDeviceToHost, s));
+  LC_CUDA(cudaStreamSynchronize(s));
+  LC_REQUIRE(h->stats_host->abort_flag == 0, LIPCACHE_E_DEVICE,
+             "a bounded wait of the probe kernel expired; the batch's queries were reported as misses");
+}
+
 LC_API const char* lipcache_last_error(void) { return g_err.c_str(); }
 
 LC_API lipcache_status lipcache_create(int32_t d, int32_t C, int64_t capacity, int32_t radius_mode,
@@ -343,6 +351,7 @@ LC_API lipcache_status lipcache_probe_writeback(lipcache_t* h, const float* Q, i
     use_device(h);
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     lc::probe(h, Q, B, out_index, out_label, out_dist, s);
+    require_no_abort(h, s);  // an aborted probe reports misses: write nothing back
     lc::certify_insert(h, Q, B, payload, require_consistency, out_inserted, nullptr, s, out_index);
     LC_CUDA(cudaMemcpyAsync(h->ins_total_host, h->ins_total, sizeof(int64_t), cudaMemcpyDeviceToHost, s));
     LC_CUDA(cudaStreamSynchronize(s));
@@ -398,6 +407,14 @@ LC_API lipcache_status lipcache_set_radius_policy(lipcache_t* h, int32_t policy,
   });
 }
 
+LC_API lipcache_status lipcache_set_debug(lipcache_t* h, int32_t flags) {
+  return guarded([&] {
+    check_handle(h);
+    LC_REQUIRE((flags & ~LIPCACHE_DEBUG_STALL_PROBE) == 0, LIPCACHE_E_INVALID, "unknown debug flags");
+    h->debug_flags = flags;
+  });
+}
+
 LC_API lipcache_status lipcache_probe_host(lipcache_t* h, const float* Q_host, int64_t B, int64_t* out_index_host,
                                            int32_t* out_label_host, float* out_dist_host, lipcache_stream_t stream) {
   return guarded([&] {
@@ -427,7 +444,7 @@ LC_API lipcache_status lipcache_probe_host(lipcache_t* h, const float* Q_host, i
       LC_CUDA(cudaMemcpyAsync(out_label_host, h->hlabel, sizeof(int32_t) * (size_t)B, cudaMemcpyDeviceToHost, s));
     if (out_dist_host)
       LC_CUDA(cudaMemcpyAsync(out_dist_host, h->hdist, sizeof(float) * (size_t)B, cudaMemcpyDeviceToHost, s));
-    LC_CUDA(cudaStreamSynchronize(s));
+    require_no_abort(h, s);
   });
 }
 

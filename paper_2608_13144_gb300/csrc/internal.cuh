@@ -227,6 +227,7 @@ struct lipcache {
   double eps_rc = 0.0, c_scr = 0.0;
   lc::EncodeTiledFn encode = nullptr;
   int pair_clusters = -1;  // resident clusters of the pair probe kernel (-1: not yet queried)
+  int debug_flags = 0;     // LIPCACHE_DEBUG_* test hooks
   lc::SelectScratch sel;
 
   // radius policy (Sec. 5.4): the probe reads rr_emp / tau_emp instead of

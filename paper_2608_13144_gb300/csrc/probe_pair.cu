@@ -71,6 +71,7 @@ struct PairArgs {
   const float* rr;
   unsigned long long* best;
   DevStats* stats;
+  int debug_stall;  // test hook: the MMA issuer first waits on a barrier nothing arrives on
 };
 
 struct PairLayout {
@@ -201,7 +202,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       int qs = 0;
       uint32_t qph = 0;
       int t = 0, i = 0;
-      bool ok = true;
+      // failure-detection test: no arrival ever completes this phase, so the
+      // bounded wait expires and the kernel takes its abort path
+      bool ok = !a.debug_stall || ptx::mbar_wait(drain, 0, abort_s, kWaitLimit);
       for (int u = cluster_id; u < a.n_units && ok; u += n_clusters, ++i) {
         int kt, qt0, qt1;
         unit_range(a, u, pair, kt, qt0, qt1);
@@ -456,6 +459,7 @@ void launch_probe_pair(lipcache* h, int64_t B, const float* qpad, const float* k
   a.rr = h->probe_rr();
   a.best = best;
   a.stats = h->stats;
+  a.debug_stall = (h->debug_flags & LIPCACHE_DEBUG_STALL_PROBE) ? 1 : 0;
   const int smem = PairLayout{a.nch, a.nst}.total() + 1024;
   LC_CUDA(cudaFuncSetAttribute(k_probe_pair, cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
   cudaLaunchAttribute attr[1];

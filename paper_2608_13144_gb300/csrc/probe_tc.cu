@@ -74,6 +74,7 @@ struct TcArgs {
   const float* rr;
   unsigned long long* best;
   DevStats* stats;
+  int debug_stall;  // test hook: the MMA issuer first waits on a barrier nothing arrives on
 };
 
 template <int BN>
@@ -229,7 +230,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       int qs = 0;
       uint32_t qph = 0;
       int t = 0, i = 0;
-      bool ok = true;
+      // failure-detection test: no arrival ever completes this phase, so the
+      // bounded wait expires and the kernel takes its abort path
+      bool ok = !a.debug_stall || ptx::mbar_wait(drain, 0, abort_s, kWaitLimit);
       for (int u = cluster_id; u < a.n_units && ok; u += n_clusters, ++i) {
         int kt, qt0, qt1;
         unit_range(a, u, rank, kt, qt0, qt1);
@@ -450,6 +453,7 @@ void launch(lipcache* h, int64_t B, const float* qpad, const float* kappa, unsig
   a.rr = h->probe_rr();
   a.best = best;
   a.stats = h->stats;
+  a.debug_stall = (h->debug_flags & LIPCACHE_DEBUG_STALL_PROBE) ? 1 : 0;
   const Layout<BN> L{a.nch, a.nst};
   const int smem = L.total() + 1024;
   LC_CUDA(cudaFuncSetAttribute(k_probe_tc<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem));

@@ -202,6 +202,10 @@ class LipCache:
                                                 rho.ctypes.data, _stream(self.device)))
         return rho
 
+    def set_debug(self, flags: int):
+        """Failure-detection test hooks (LIPCACHE_DEBUG_*; 0 = off)."""
+        check(self.L.lipcache_set_debug(self._h, int(flags)))
+
     def set_radius_scale(self, kappa: float):
         check(self.L.lipcache_set_radius_scale(self._h, float(kappa)))
 

@@ -69,6 +69,7 @@ def test_null_handle_calls(lib):
     assert lib.lipcache_insert_select(None, None, 0, None, 0, 1, 0, 0, None, None, C.byref(ns), None) == 1
     assert ns.value == 0
     assert lib.lipcache_set_radius_policy(None, 1, 1.0, None, None) == 1
+    assert lib.lipcache_set_debug(None, 0) == 1
 
 
 def test_create_without_gpu_fails_cleanly(lib):
