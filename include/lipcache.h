@@ -58,6 +58,15 @@ typedef enum lipcache_status {
 #define LIPCACHE_RADIUS_CONSERVATIVE 0 /* r  = m / (sigma_max(W) sqrt 2), Eq. 21 */
 #define LIPCACHE_RADIUS_TIGHT 1        /* r* = min_j (s_y - s_j) / ||W_y - W_j||, Eq. 29 */
 
+/* Certify kernels (lipcache_info.last_insert_kernel). WIDE_TILE: head resident
+ * in shared memory, 128-row tiles, logits in registers (conservative radius,
+ * d % 4 == 0, head small enough). TILE64: head resident, 64-row tiles, logits
+ * in shared memory (also the tight radius). STREAMED: head read from L2
+ * (large heads). All three compute the same values. */
+#define LIPCACHE_INSERT_WIDE_TILE 1
+#define LIPCACHE_INSERT_TILE64 2
+#define LIPCACHE_INSERT_STREAMED 3
+
 /* Radius policies of the probe (lipcache_set_radius_policy). */
 #define LIPCACHE_POLICY_CERTIFIED 0  /* per-entry certified radius (Eq. 21 or Eq. 29) */
 #define LIPCACHE_POLICY_GLOBAL 1     /* one global nearest-neighbour threshold (Sec. 5.4) */
@@ -102,7 +111,7 @@ typedef struct lipcache_info {
   int32_t last_grid;        /* CTAs launched by the last probe's main kernel */
   int32_t last_cluster;     /* CTAs per cluster of that launch (1 = no cluster) */
   int32_t radius_policy;    /* LIPCACHE_POLICY_* the probe uses */
-  int32_t reserved;
+  int32_t last_insert_kernel; /* kernel that certified the last insert: LIPCACHE_INSERT_* (0 before any) */
   double policy_param;      /* tau (GLOBAL) or beta (INTERCLASS); 0 for CERTIFIED */
 } lipcache_info;
 
@@ -299,6 +308,19 @@ lipcache_status lipcache_set_radius_policy(lipcache_t* h, int32_t policy, double
                                            lipcache_stream_t stream);
 
 /*
+ * Read back cache entries [first, first + n) (insertion order), e.g. to
+ * inspect a cache or to persist it: re-inserting the returned keys with their
+ * labels as payload into a cache with the same head rebuilds the same entries.
+ *   keys_host    n x d FP32 (host), nullable
+ *   radius_host  n FP32 (host), nullable: the reported radius r of each entry
+ *   label_host   n int32 (host), nullable: payload
+ *   yG_host      n int32 (host), nullable: GuardNet label of the key
+ * Synchronises `stream`. Errors: E_INVALID (range outside [0, size)), E_CUDA.
+ */
+lipcache_status lipcache_read_entries(lipcache_t* h, int64_t first, int64_t n, float* keys_host, float* radius_host,
+                                      int32_t* label_host, int32_t* yG_host, lipcache_stream_t stream);
+
+/*
  * Test hooks for failure detection. LIPCACHE_DEBUG_STALL_PROBE makes the MMA
  * issuer of the tensor probe kernels first wait on an mbarrier that nothing
  * arrives on: the bounded wait (~2^31 cycles, about a second) expires, the
@@ -309,6 +331,9 @@ lipcache_status lipcache_set_radius_policy(lipcache_t* h, int32_t policy, double
  * flags = 0 restores normal operation. Errors: E_INVALID (unknown bits).
  */
 #define LIPCACHE_DEBUG_STALL_PROBE 1
+/* Certify inserted rows with the 64-row-tile kernel where the wide-tile one
+ * would run; both compute the same values, so tests compare them bit for bit. */
+#define LIPCACHE_DEBUG_INSERT_TILE64 2
 lipcache_status lipcache_set_debug(lipcache_t* h, int32_t flags);
 
 /*

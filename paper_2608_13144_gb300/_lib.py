@@ -21,7 +21,7 @@ PROBE_AUTO, PROBE_TENSOR, PROBE_EXACT, PROBE_TENSOR_SINGLE, PROBE_TENSOR_PAIR = 
 # Every symbol the header declares; tests check the library exports them all.
 EXPORTS = ["lipcache_create", "lipcache_set_head", "lipcache_insert", "lipcache_probe", "lipcache_probe_host",
            "lipcache_probe_noalloc", "lipcache_probe_writeback", "lipcache_consistency",
-           "lipcache_set_radius_policy", "lipcache_insert_select", "lipcache_set_debug",
+           "lipcache_set_radius_policy", "lipcache_insert_select", "lipcache_set_debug", "lipcache_read_entries",
            "lipcache_set_probe_path", "lipcache_set_radius_scale", "lipcache_set_spectral_options",
            "lipcache_reserve", "lipcache_enable_timing", "lipcache_get_info", "lipcache_reset_stats",
            "lipcache_size", "lipcache_destroy", "lipcache_last_error"]
@@ -35,7 +35,7 @@ class Info(C.Structure):
                 ("candidates", C.c_int64), ("device_errors", C.c_int64), ("probe_path", C.c_int32),
                 ("last_probe_path", C.c_int32), ("last_probe_ms", C.c_float), ("num_sms", C.c_int32),
                 ("kernel_ms_total", C.c_double), ("kernel_launches", C.c_int64), ("last_grid", C.c_int32),
-                ("last_cluster", C.c_int32), ("radius_policy", C.c_int32), ("reserved", C.c_int32),
+                ("last_cluster", C.c_int32), ("radius_policy", C.c_int32), ("last_insert_kernel", C.c_int32),
                 ("policy_param", C.c_double)]
 
 
@@ -69,6 +69,7 @@ def load(path: str = LIB_PATH):
         "lipcache_set_radius_policy": ([vp, i32, f64, vp, vp], C.c_int),
         "lipcache_insert_select": ([vp, vp, i64, vp, i32, i32, i64, i32, vp, vp, C.POINTER(i64), vp], C.c_int),
         "lipcache_set_debug": ([vp, i32], C.c_int),
+        "lipcache_read_entries": ([vp, i64, i64, vp, vp, vp, vp, vp], C.c_int),
         "lipcache_set_probe_path": ([vp, i32], C.c_int),
         "lipcache_set_radius_scale": ([vp, f64], C.c_int),
         "lipcache_set_spectral_options": ([vp, i32, i32], C.c_int),

@@ -56,6 +56,7 @@ void release(lipcache* h) {
   if (!h) return;
   cudaSetDevice(h->device);
   dev_free(h->W);
+  dev_free(h->wt_prep);
   dev_free(h->b);
   dev_free(h->Wnorm);
   dev_free(h->Wnorm32);
@@ -231,6 +232,7 @@ LC_API lipcache_status lipcache_set_head(lipcache_t* h, const float* W, const fl
     use_device(h);
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     h->head_set = false;
+    h->wt_prep_ncg = 0;
     LC_CUDA(cudaMemcpyAsync(h->W, W, sizeof(float) * (size_t)h->C * h->d, cudaMemcpyDeviceToDevice, s));
     LC_CUDA(cudaMemcpyAsync(h->b, b, sizeof(float) * (size_t)h->C, cudaMemcpyDeviceToDevice, s));
     lc::spectral_norm(h, s);
@@ -407,10 +409,36 @@ LC_API lipcache_status lipcache_set_radius_policy(lipcache_t* h, int32_t policy,
   });
 }
 
+LC_API lipcache_status lipcache_read_entries(lipcache_t* h, int64_t first, int64_t n, float* keys_host,
+                                             float* radius_host, int32_t* label_host, int32_t* yG_host,
+                                             lipcache_stream_t stream) {
+  return guarded([&] {
+    check_handle(h);
+    LC_REQUIRE(first >= 0 && n >= 0 && first + n <= h->size, LIPCACHE_E_INVALID, "entries outside [0, size)");
+    if (n == 0) return;
+    use_device(h);
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    if (keys_host)
+      LC_CUDA(cudaMemcpy2DAsync(keys_host, sizeof(float) * (size_t)h->d, h->table.keys + (size_t)first * h->dpad,
+                                sizeof(float) * (size_t)h->dpad, sizeof(float) * (size_t)h->d, (size_t)n,
+                                cudaMemcpyDeviceToHost, s));
+    if (radius_host)
+      LC_CUDA(cudaMemcpyAsync(radius_host, h->table.radius + first, sizeof(float) * (size_t)n, cudaMemcpyDeviceToHost,
+                              s));
+    if (label_host)
+      LC_CUDA(cudaMemcpyAsync(label_host, h->table.label + first, sizeof(int32_t) * (size_t)n,
+                              cudaMemcpyDeviceToHost, s));
+    if (yG_host)
+      LC_CUDA(cudaMemcpyAsync(yG_host, h->table.yG + first, sizeof(int32_t) * (size_t)n, cudaMemcpyDeviceToHost, s));
+    LC_CUDA(cudaStreamSynchronize(s));
+  });
+}
+
 LC_API lipcache_status lipcache_set_debug(lipcache_t* h, int32_t flags) {
   return guarded([&] {
     check_handle(h);
-    LC_REQUIRE((flags & ~LIPCACHE_DEBUG_STALL_PROBE) == 0, LIPCACHE_E_INVALID, "unknown debug flags");
+    LC_REQUIRE((flags & ~(LIPCACHE_DEBUG_STALL_PROBE | LIPCACHE_DEBUG_INSERT_TILE64)) == 0, LIPCACHE_E_INVALID,
+               "unknown debug flags");
     h->debug_flags = flags;
   });
 }
@@ -540,7 +568,7 @@ LC_API lipcache_status lipcache_get_info(lipcache_t* h, lipcache_info* info) {
     info->last_grid = h->last_grid;
     info->last_cluster = h->last_cluster;
     info->radius_policy = h->policy;
-    info->reserved = 0;
+    info->last_insert_kernel = h->last_insert_kernel;
     info->policy_param = h->policy_param;
   });
 }

@@ -821,6 +821,442 @@ __global__ void __launch_bounds__(kThreads, 1) k_certify_wres(CertArgs a, int Cp
   }
 }
 
+// ---------------------------------------------------------------- k_certify_wt
+// Certified insertion, conservative radius, head resident in shared memory,
+// tiles of 128 rows (persistent CTAs of 8 warps; C <= 256, d % 4 == 0):
+//  1. Load: warp w takes feature quarter w % 4 of rows 64 (w / 4) .. + 63,
+//     lane = row; the rows are transposed into shared memory (h^T) and the
+//     quarter sums of ||z||^2 are formed on the way, in feature order.
+//  2. FP32 logits: each thread keeps a register tile of 8 rows x NCG classes
+//     (16 row groups x 16 class groups; packed FP32x2 FMAs on class pairs, one
+//     FMA chain per (row, class) in k order). Per feature it reads 8 + NCG
+//     shared floats for 8 NCG FMAs, so at NCG = 13 the FP32 pipe (every
+//     sub-partition equally loaded), not shared memory, bounds the product.
+//  3. From the registers: interval lower ends, each row's second-largest
+//     lower end L2 (butterfly over the 16 lanes that share the rows), and the
+//     candidate classes (upper end >= L2) into per-row slots and a pair list.
+//  4. Pair refinement (8 lanes a pair, compensated dot product), per-row
+//     selection and FP64 finals, rows with more than kMaxCand candidates by
+//     warp_row_refine, 32-row ranks and counts.
+// Logits, candidate sets, refined pairs and finals are the values
+// k_certify_wres computes, bit for bit. W^T holds class g NCG + j at column
+// g GS + j (GS even, GS = 2 mod 4), so the 16 class groups' 64-bit weight
+// loads fall on distinct banks.
+constexpr int kWtRows = 128;        // rows per tile
+constexpr int kWtHst = kWtRows + 4;  // h^T row stride (floats): 16-byte aligned, banks spread
+
+struct WtTile {
+  float knp[4][kWtRows];  // quarter sums of ||z||^2
+  float hn[kWtRows];      // upper bound of ||z||
+  int ncand[kWtRows];
+  uint8_t cls[kWtRows][kMaxCand];
+  float rh[kWtRows][kMaxCand], rl[kWtRows][kMaxCand], re[kWtRows][kMaxCand];
+  int pairs[kWtRows * kMaxCand];  // r | slot << 8 | class << 16; after the refinement, per-warp logit rows
+  int ovf[kWtRows];
+  int npairs, novf, pad[2];
+  uint8_t acc_flag[kWtRows];
+};
+
+struct WtLayout {
+  int NCG, GS, wst;
+  uint32_t off_h, off_e, off_tile, total;
+};
+
+template <int NCG>
+__global__ void __launch_bounds__(kThreads, 1) k_certify_wt(CertArgs a, WtLayout L, const float* __restrict__ prep,
+                                                             int64_t nb32) {
+  extern __shared__ __align__(16) unsigned char smem[];
+  constexpr int NPR = NCG / 2;  // class pairs per thread
+  constexpr bool kOdd = (NCG & 1) != 0;
+  const int d = a.d, C = a.C, GS = L.GS, wst = L.wst;
+  float* wT = reinterpret_cast<float*>(smem);
+  float* hT = reinterpret_cast<float*>(smem + L.off_h);  // d x kWtHst
+  float* eA = reinterpret_cast<float*>(smem + L.off_e);  // 16 GS each, grouped columns
+  float* eB = eA + 16 * GS;
+  float* bp = eB + 16 * GS;
+  float* wn_s = bp + 16 * GS;  // C each, by class
+  float* b_s = wn_s + C;
+  WtTile& ts = *reinterpret_cast<WtTile*>(smem + L.off_tile);
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  {
+    // the prepared head: L.off_h bytes, 128-bit loads, eight in flight
+    const float4* src = reinterpret_cast<const float4*>(prep);
+    float4* dst = reinterpret_cast<float4*>(smem);
+    const int n4 = (int)(L.off_h / 16);
+    constexpr int kB = 8;
+    for (int i0 = tid; i0 < n4; i0 += kB * kThreads) {
+      float4 v[kB];
+#pragma unroll
+      for (int u = 0; u < kB; ++u) {
+        const int i = i0 + u * kThreads;
+        if (i < n4) v[u] = __ldg(src + i);
+      }
+#pragma unroll
+      for (int u = 0; u < kB; ++u) {
+        const int i = i0 + u * kThreads;
+        if (i < n4) dst[i] = v[u];
+      }
+    }
+  }
+  const int cg = lane & 15, rg = warp * 2 + (lane >> 4);  // product: rows 8 rg .. 8 rg + 7, classes cg NCG ..
+  const float* wp = wT + cg * GS;
+  const int g8 = tid / kGroup, sub = tid % kGroup;  // refinement groups
+  const int q = warp & 3, dq = (d + 3) / 4, k_lo = q * dq, k_hi = min(d, k_lo + dq);  // load quarter
+  // this CTA's rows: a contiguous range of whole 32-row blocks (balanced over
+  // the grid), in chunks of up to kWtRows rows
+  const int64_t b_lo = (int64_t)blockIdx.x * nb32 / gridDim.x, b_hi = ((int64_t)blockIdx.x + 1) * nb32 / gridDim.x;
+  const int64_t row_hi = b_hi * 32 < a.n ? b_hi * 32 : a.n;
+  if (tid == 0 && b_lo * 32 < row_hi)
+    prefetch_l2_bulk(a.H + (size_t)(b_lo * 32) * d,
+                     (uint32_t)((row_hi - b_lo * 32 < kWtRows ? row_hi - b_lo * 32 : kWtRows) * d * sizeof(float)));
+
+  for (int64_t row0 = b_lo * 32; row0 < row_hi; row0 += kWtRows) {
+    const int nrows = (int)(row_hi - row0 < kWtRows ? row_hi - row0 : kWtRows);
+    __syncthreads();  // the previous chunk is done with h^T and the lists (W^T written on the first pass)
+    // the next chunk's rows start moving into L2
+    if (tid == 0 && row0 + kWtRows < row_hi) {
+      const int64_t r1 = row0 + kWtRows;
+      const int64_t n1 = row_hi - r1 < kWtRows ? row_hi - r1 : kWtRows;
+      prefetch_l2_bulk(a.H + (size_t)r1 * d, (uint32_t)(n1 * d * sizeof(float)));
+    }
+    // 1. load, transpose, quarter sums (32-row blocks past nrows are skipped;
+    //    rows past nrows are never selected)
+    for (int half = 0; half < 2; ++half) {
+      const int rb = (warp >> 2) * 64 + half * 32;
+      if (rb >= nrows) continue;
+      const int r = rb + lane;
+      const bool live = r < nrows;
+      const float* src = a.H + (size_t)(row0 + (live ? r : 0)) * d;
+      float p = 0.f;
+      if ((dq & 3) == 0) {
+        constexpr int kB = 8;
+        for (int k0 = k_lo; k0 < k_hi; k0 += 4 * kB) {
+          float4 v[kB];
+#pragma unroll
+          for (int u = 0; u < kB; ++u) {
+            const int k = k0 + 4 * u;
+            v[u] = (live && k < k_hi) ? __ldg(reinterpret_cast<const float4*>(src + k))
+                                      : make_float4(0.f, 0.f, 0.f, 0.f);
+          }
+#pragma unroll
+          for (int u = 0; u < kB; ++u) {
+            const int k = k0 + 4 * u;
+            if (k < k_hi) {
+              p = fmaf(v[u].x, v[u].x, p);
+              p = fmaf(v[u].y, v[u].y, p);
+              p = fmaf(v[u].z, v[u].z, p);
+              p = fmaf(v[u].w, v[u].w, p);
+              float* dst = hT + (size_t)k * kWtHst + r;
+              dst[0] = v[u].x;
+              dst[kWtHst] = v[u].y;
+              dst[2 * kWtHst] = v[u].z;
+              dst[3 * kWtHst] = v[u].w;
+            }
+          }
+        }
+      } else {
+        for (int k = k_lo; k < k_hi; ++k) {
+          const float x = live ? __ldg(src + k) : 0.f;
+          p = fmaf(x, x, p);
+          hT[(size_t)k * kWtHst + r] = x;
+        }
+      }
+      ts.knp[q][r] = p;
+    }
+    if (tid < kWtRows) {
+      ts.ncand[tid] = 0;
+      ts.acc_flag[tid] = 0;
+    }
+    if (tid == 0) {
+      ts.npairs = 0;
+      ts.novf = 0;
+    }
+    __syncthreads();
+    if (16 * warp < nrows) {  // this warp's 16 rows hold at least one live row
+      // 2. FP32 logits of rows 8 rg .. 8 rg + 7 and classes cg NCG .. cg NCG + NCG - 1
+      uint64_t accp[8][NPR > 0 ? NPR : 1];
+      float accs[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+#pragma unroll
+        for (int m = 0; m < NPR; ++m) accp[i][m] = 0ull;
+        accs[i] = 0.f;
+      }
+      {
+        const float* hb = hT + 8 * rg;
+#pragma unroll 2
+        for (int k = 0; k < d; ++k) {
+          const float4 x0 = *reinterpret_cast<const float4*>(hb + (size_t)k * kWtHst);
+          const float4 x1 = *reinterpret_cast<const float4*>(hb + (size_t)k * kWtHst + 4);
+          const float hv[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
+          const float* wk = wp + (size_t)k * wst;
+          uint64_t wv[NPR > 0 ? NPR : 1];
+#pragma unroll
+          for (int m = 0; m < NPR; ++m) wv[m] = *reinterpret_cast<const uint64_t*>(wk + 2 * m);
+          const float w1 = kOdd ? wk[NCG - 1] : 0.f;
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            const uint32_t hb32 = __float_as_uint(hv[i]);
+            const uint64_t hh = ptx::pack_f32x2(hb32, hb32);
+#pragma unroll
+            for (int m = 0; m < NPR; ++m) accp[i][m] = ptx::fma_f32x2(wv[m], hh, accp[i][m]);
+            if (kOdd) accs[i] = __fmaf_rn(w1, hv[i], accs[i]);
+          }
+        }
+      }
+      // 3. interval lower ends, each row's L2, candidates, two rows at a time.
+      // The loop stays rolled (its body runs once per chunk and would not stay
+      // in the instruction cache unrolled); rows i, i + 1 are always in
+      // accp[0..1], the rest shift down. Branch-free over the classes (a
+      // divergent branch per class would serialise them): dead classes get
+      // -inf lower ends and no candidacy.
+#pragma unroll 1
+      for (int i = 0; i < 8; i += 2) {
+        float sv[2][NCG], E[2][NCG], l1[2], l2[2], hn[2];
+        int r[2];
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+          r[u] = 8 * rg + i + u;
+          const float kn = (ts.knp[0][r[u]] + ts.knp[1][r[u]]) + (ts.knp[2][r[u]] + ts.knp[3][r[u]]);
+          hn[u] = norm_upper(kn);
+#pragma unroll
+          for (int m = 0; m < NPR; ++m) {
+            sv[u][2 * m] = __fadd_rn(__uint_as_float((uint32_t)accp[u][m]), bp[cg * GS + 2 * m]);
+            sv[u][2 * m + 1] = __fadd_rn(__uint_as_float((uint32_t)(accp[u][m] >> 32)), bp[cg * GS + 2 * m + 1]);
+          }
+          if (kOdd) sv[u][NCG - 1] = __fadd_rn(accs[u], bp[cg * GS + NCG - 1]);
+        }
+#pragma unroll
+        for (int ii = 0; ii < 6; ++ii) {
+#pragma unroll
+          for (int m = 0; m < NPR; ++m) accp[ii][m] = accp[ii + 2][m];
+          accs[ii] = accs[ii + 2];
+        }
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+          l1[u] = -INFINITY;
+          l2[u] = -INFINITY;
+#pragma unroll
+          for (int jc = 0; jc < NCG; ++jc) {
+            E[u][jc] = __fmaf_ru(eA[cg * GS + jc], hn[u], __fmaf_ru(fabsf(sv[u][jc]), 2.3841858e-07f, eB[cg * GS + jc]));
+            float lo = __fsub_rd(sv[u][jc], E[u][jc]);
+            lo = (lo == lo && cg * NCG + jc < C) ? lo : -INFINITY;
+            l2[u] = fmaxf(l2[u], fminf(l1[u], lo));
+            l1[u] = fmaxf(l1[u], lo);
+          }
+        }
+#pragma unroll
+        for (int o = 1; o < 16; o <<= 1) {
+#pragma unroll
+          for (int u = 0; u < 2; ++u) {
+            const float o1 = __shfl_xor_sync(kFull, l1[u], o), o2 = __shfl_xor_sync(kFull, l2[u], o);
+            l2[u] = fmaxf(l2[u], fminf(l1[u], o1));
+            l1[u] = fmaxf(l1[u], o1);
+            l2[u] = fmaxf(l2[u], fminf(l1[u], o2));
+            l1[u] = fmaxf(l1[u], o2);
+          }
+        }
+        unsigned cm[2];  // candidate bits of this lane's classes
+        int incl[2], mine[2];
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+          cm[u] = 0;
+#pragma unroll
+          for (int jc = 0; jc < NCG; ++jc)
+            cm[u] |= (unsigned)(cg * NCG + jc < C && __fadd_ru(sv[u][jc], E[u][jc]) >= l2[u]) << jc;
+          cm[u] = r[u] < nrows ? cm[u] : 0u;
+          mine[u] = __popc(cm[u]);
+          incl[u] = mine[u];
+        }
+        // slots of each row: the 16 lanes of this half-warp own it; prefix
+        // sum of their candidate counts
+#pragma unroll
+        for (int o = 1; o < 16; o <<= 1) {
+#pragma unroll
+          for (int u = 0; u < 2; ++u) {
+            const int t = __shfl_up_sync(kFull, incl[u], o, 16);
+            if (cg >= o) incl[u] += t;
+          }
+        }
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+          int slot = incl[u] - mine[u];
+          unsigned m = cm[u];
+          while (m) {
+            const int jc = __ffs(m) - 1;
+            m &= m - 1;
+            if (slot < kMaxCand) ts.cls[r[u]][slot] = (uint8_t)(cg * NCG + jc);
+            ++slot;
+          }
+          if (cg == 15) {
+            ts.ncand[r[u]] = incl[u];
+            ts.hn[r[u]] = hn[u];
+          }
+        }
+      }
+    }
+    // this warp's 16 rows into the pair list: one reservation per warp
+    __syncwarp();
+    {
+      const int R = 8 * (2 * warp + ((lane >> 3) & 1)) + (lane & 7);
+      const int n = lane < 16 ? min(ts.ncand[R], kMaxCand) : 0;
+      int incl = n;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int t = __shfl_up_sync(kFull, incl, o);
+        if (lane >= o) incl += t;
+      }
+      const int total = __shfl_sync(kFull, incl, 31);
+      int base = 0;
+      if (lane == 0 && total) base = atomicAdd(&ts.npairs, total);
+      base = __shfl_sync(kFull, base, 0) + incl - n;
+      for (int sl = 0; sl < n; ++sl) ts.pairs[base + sl] = R | (sl << 8) | ((int)ts.cls[R][sl] << 16);
+    }
+    __syncthreads();
+    // 4. refine the pairs, kGroup lanes a pair, two pairs a group at a time
+    constexpr int kGroups = kThreads / kGroup;
+    const int np = ts.npairs;
+    for (int base = 0; base < np; base += 2 * kGroups) {
+      int pi[2], r[2], slot[2], c[2], col[2];
+      float p[2] = {0.f, 0.f}, cc[2] = {0.f, 0.f};
+#pragma unroll
+      for (int u = 0; u < 2; ++u) {
+        pi[u] = base + u * kGroups + g8;
+        const int pk = ts.pairs[pi[u] < np ? pi[u] : 0];
+        r[u] = pk & 0xff;
+        slot[u] = (pk >> 8) & 0xff;
+        c[u] = pk >> 16;
+        col[u] = (c[u] / NCG) * GS + (c[u] % NCG);
+      }
+      for (int k = sub; k < d; k += kGroup) {
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+          const float w = wT[(size_t)k * wst + col[u]], x = hT[(size_t)k * kWtHst + r[u]];
+          const float pr = __fmul_rn(w, x);
+          const float er = __fmaf_rn(w, x, -pr);
+          float t, qq;
+          two_sum(p[u], pr, t, qq);
+          p[u] = t;
+          cc[u] = __fadd_rn(cc[u], __fadd_rn(qq, er));
+        }
+      }
+#pragma unroll
+      for (int o = kGroup / 2; o > 0; o >>= 1) {
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+          const float pb = __shfl_xor_sync(kFull, p[u], o), cb = __shfl_xor_sync(kFull, cc[u], o);
+          float t, qq;
+          two_sum(p[u], pb, t, qq);
+          p[u] = t;
+          cc[u] = __fadd_rn(__fadd_rn(cc[u], cb), qq);
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < 2; ++u) {
+        if (pi[u] < np && sub == 0) {
+          float t, qq, hi, lo;
+          two_sum(p[u], b_s[c[u]], t, qq);
+          two_sum(t, __fadd_rn(cc[u], qq), hi, lo);
+          ts.rh[r[u]][slot[u]] = hi;
+          ts.rl[r[u]][slot[u]] = lo;
+          ts.re[r[u]][slot[u]] = refined_err(a.g2f, wn_s[c[u]], ts.hn[r[u]], b_s[c[u]]);
+        }
+      }
+    }
+    __syncthreads();
+    if (tid < nrows) {
+      const int r = tid, n = ts.ncand[r];
+      if (n > kMaxCand) {
+        ts.ovf[atomicAdd(&ts.novf, 1)] = r;
+      } else {
+        const float kn = (ts.knp[0][r] + ts.knp[1][r]) + (ts.knp[2][r] + ts.knp[3][r]);
+        Top2 t;
+        for (int sl = 0; sl < n; ++sl) t.push(ts.cls[r][sl], ts.rh[r][sl], ts.rl[r][sl], ts.re[r][sl]);
+        row_finals(a, row0 + r, t.result(kn), &ts.acc_flag[r]);
+      }
+    }
+    __syncthreads();
+    // rows with more than kMaxCand candidates: FP32 logits again (the same
+    // FMA chains, into this warp's share of the dead pair list), then the
+    // one-warp refinement
+    for (int i = warp; i < ts.novf; i += kWarps) {
+      const int r = ts.ovf[i];
+      float* lrow = reinterpret_cast<float*>(ts.pairs) + (size_t)warp * C;
+      for (int c = lane; c < C; c += 32) {
+        const int col = (c / NCG) * GS + (c % NCG);
+        float v = 0.f;
+        for (int k = 0; k < d; ++k) v = __fmaf_rn(wT[(size_t)k * wst + col], hT[(size_t)k * kWtHst + r], v);
+        lrow[c] = __fadd_rn(v, b_s[c]);
+      }
+      __syncwarp();
+      const RowVals v = warp_row_refine(a, hT + r, kWtHst, lrow, a.W, d, 1, a.Wnorm32, a.b, lane);
+      if (lane == 0) row_finals(a, row0 + r, v, &ts.acc_flag[r]);
+      __syncwarp();
+    }
+    __syncthreads();
+    if (warp < kWtRows / 32 && warp * 32 < nrows) {
+      const int s0 = warp * 32;
+      const int nsub = nrows - s0 < 32 ? nrows - s0 : 32;
+      const bool f = lane < nsub && ts.acc_flag[s0 + lane];
+      const unsigned m = __ballot_sync(kFull, f);
+      if (lane < nsub) a.rank[row0 + s0 + lane] = __popc(m & ((1u << lane) - 1u));
+      if (lane == 0) a.bcount[(row0 + s0) / 32] = __popc(m);
+    }
+  }
+}
+
+WtLayout wt_layout(int d, int C, int NCG) {
+  WtLayout L;
+  L.NCG = NCG;
+  L.GS = NCG + (NCG & 1);
+  if (L.GS % 4 == 0) L.GS += 2;
+  L.wst = ((16 * L.GS - 4 + 31) / 32) * 32 + 4;
+  auto al = [](size_t x) { return (uint32_t)((x + 15) / 16 * 16); };
+  L.off_e = al(sizeof(float) * (size_t)d * L.wst);
+  L.off_h = al(L.off_e + sizeof(float) * (3 * 16 * (size_t)L.GS + 2 * (size_t)C));
+  L.off_tile = al(L.off_h + sizeof(float) * (size_t)d * kWtHst);
+  L.total = L.off_tile + (uint32_t)sizeof(WtTile);
+  return L;
+}
+
+// The head in k_certify_wt's shared-memory layout (its first L.off_h bytes):
+// W^T in grouped columns (class g NCG + j at column g GS + j, zero padded),
+// then the per-column error terms eA = g32f ||W_c|| and eB = g32f |b_c| +
+// tiny (rounded up) and biases, then ||W_c|| and b_c by class.
+__global__ void k_wt_prepare(CertArgs a, WtLayout L, float* __restrict__ out) {
+  const int d = a.d, C = a.C, NCG = L.NCG, GS = L.GS, wst = L.wst;
+  float* eA = out + L.off_e / sizeof(float);
+  float* eB = eA + 16 * GS;
+  float* bp = eB + 16 * GS;
+  float* wn_s = bp + 16 * GS;
+  float* b_s = wn_s + C;
+  const int stride = gridDim.x * blockDim.x;
+  for (int idx = blockIdx.x * blockDim.x + threadIdx.x; idx < d * wst; idx += stride) {
+    const int k = idx / wst, col = idx - k * wst;
+    const int g = col / GS, j = col - g * GS, c = g * NCG + j;
+    out[idx] = (col < 16 * GS && j < NCG && c < C) ? a.W[(size_t)c * d + k] : 0.f;
+  }
+  for (int col = blockIdx.x * blockDim.x + threadIdx.x; col < 16 * GS; col += stride) {
+    const int g = col / GS, j = col - g * GS, c = g * NCG + j;
+    const bool live = j < NCG && c < C;
+    const float wn = live ? a.Wnorm32[c] : 0.f, bc = live ? a.b[c] : 0.f;
+    eA[col] = __fmul_ru(a.g32f, wn);
+    eB[col] = __fmaf_ru(a.g32f, fabsf(bc), kTinyF);
+    bp[col] = bc;
+  }
+  for (int c = blockIdx.x * blockDim.x + threadIdx.x; c < C; c += stride) {
+    wn_s[c] = a.Wnorm32[c];
+    b_s[c] = a.b[c];
+  }
+}
+
+// Smallest compiled per-thread class count covering C classes in 16 groups.
+int wt_ncg(int C) {
+  const int need = (C + 15) / 16;
+  return need <= 1 ? 1 : need <= 4 ? 4 : need <= 7 ? 7 : need <= 13 ? 13 : need <= 16 ? 16 : 0;
+}
+
 // Exclusive scan of the per-block accepted counts (one block).
 __global__ void __launch_bounds__(1024) k_scan(const int32_t* __restrict__ cnt, int32_t* __restrict__ off, int nb,
                                                int64_t* __restrict__ total) {
@@ -1037,18 +1473,47 @@ void launch_certify(lipcache* h, const float* H, int64_t n, const int32_t* paylo
   const size_t smem_wres = sizeof(float) * ((size_t)h->dpad * Cp + (size_t)h->dpad * kHStride +
                                             (size_t)kWTile * a.lstride + 1 + 4 * (size_t)h->C) +
                            sizeof(double) * 2 * kWarps * (size_t)(a.tight ? h->C : 0) + sizeof(TileSmem);
-  if (h->C <= 256 && smem_wres <= 220 * 1024) {
+  const int ncg = wt_ncg(h->C);
+  const bool vec16 = h->d % 4 == 0 && ((uintptr_t)H & 15) == 0;
+  const WtLayout L = wt_layout(h->d, h->C, ncg > 0 ? ncg : 1);
+  if (!a.tight && vec16 && ncg > 0 && L.total <= 227 * 1024 && !(h->debug_flags & LIPCACHE_DEBUG_INSERT_TILE64)) {
+    const int64_t nb32 = (n + 31) / 32;
+    const int grid = nb32 < h->num_sms ? (int)nb32 : h->num_sms;
+    if (h->wt_prep_ncg != ncg) {
+      if (h->wt_prep_cap < L.off_h) {
+        if (h->wt_prep) cudaFree(h->wt_prep);
+        h->wt_prep = nullptr;
+        h->wt_prep_cap = 0;
+        LC_CUDA(cudaMalloc(&h->wt_prep, L.off_h));
+        h->wt_prep_cap = L.off_h;
+      }
+      k_wt_prepare<<<64, 256, 0, s>>>(a, L, h->wt_prep);
+      LC_LAUNCH_CHECK("k_wt_prepare");
+      h->wt_prep_ncg = ncg;
+    }
+    void (*kern)(CertArgs, WtLayout, const float*, int64_t) = ncg == 1    ? k_certify_wt<1>
+                                            : ncg == 4  ? k_certify_wt<4>
+                                            : ncg == 7  ? k_certify_wt<7>
+                                            : ncg == 13 ? k_certify_wt<13>
+                                                        : k_certify_wt<16>;
+    LC_CUDA(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)L.total));
+    kern<<<grid, kThreads, L.total, s>>>(a, L, h->wt_prep, nb32);
+    LC_LAUNCH_CHECK("k_certify_wt");
+    h->last_insert_kernel = LIPCACHE_INSERT_WIDE_TILE;
+  } else if (h->C <= 256 && smem_wres <= 220 * 1024) {
     const int n_tiles = (int)((n + kWTile - 1) / kWTile);
     const int grid = n_tiles < h->num_sms ? n_tiles : h->num_sms;
     LC_CUDA(cudaFuncSetAttribute(k_certify_wres, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_wres));
     const int vec = (h->d % 4 == 0 && ((uintptr_t)H & 15) == 0) ? 1 : 0;
     k_certify_wres<<<grid, kThreads, smem_wres, s>>>(a, Cp, h->dpad, n_tiles, vec);
     LC_LAUNCH_CHECK("k_certify_wres");
+    h->last_insert_kernel = LIPCACHE_INSERT_TILE64;
   } else {
     const size_t smem = certify_smem_bytes(h->d, h->C);
     LC_CUDA(cudaFuncSetAttribute(k_certify, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
     k_certify<<<nb, kThreads, smem, s>>>(a);
     LC_LAUNCH_CHECK("k_certify");
+    h->last_insert_kernel = LIPCACHE_INSERT_STREAMED;
   }
 }
 

@@ -228,6 +228,10 @@ struct lipcache {
   lc::EncodeTiledFn encode = nullptr;
   int pair_clusters = -1;  // resident clusters of the pair probe kernel (-1: not yet queried)
   int debug_flags = 0;     // LIPCACHE_DEBUG_* test hooks
+  int last_insert_kernel = 0;  // LIPCACHE_INSERT_*
+  float* wt_prep = nullptr;    // the head in the wide-tile certify kernel's shared-memory layout
+  size_t wt_prep_cap = 0;      // bytes allocated
+  int wt_prep_ncg = 0;         // classes per thread it was laid out for (0: stale)
   lc::SelectScratch sel;
 
   // radius policy (Sec. 5.4): the probe reads rr_emp / tau_emp instead of

@@ -202,6 +202,19 @@ class LipCache:
                                                 rho.ctypes.data, _stream(self.device)))
         return rho
 
+    def entries(self, first: int = 0, n: int | None = None) -> dict:
+        """Cache entries [first, first + n) as numpy arrays: keys (n x d),
+        radius, label (payload) and yG, in insertion order."""
+        size = self.size
+        n = size - first if n is None else n
+        keys = np.empty((n, self.d), dtype=np.float32)
+        radius = np.empty(n, dtype=np.float32)
+        label = np.empty(n, dtype=np.int32)
+        yG = np.empty(n, dtype=np.int32)
+        check(self.L.lipcache_read_entries(self._h, int(first), int(n), keys.ctypes.data, radius.ctypes.data,
+                                           label.ctypes.data, yG.ctypes.data, _stream(self.device)))
+        return {"keys": keys, "radius": radius, "label": label, "yG": yG}
+
     def set_debug(self, flags: int):
         """Failure-detection test hooks (LIPCACHE_DEBUG_*; 0 = off)."""
         check(self.L.lipcache_set_debug(self._h, int(flags)))

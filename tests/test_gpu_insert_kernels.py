@@ -1,0 +1,140 @@
+"""The wide-tile certify kernel (128-row tiles, logits in registers) against
+the 64-row-tile kernel and the FP64 oracle (pytest -m gpu). Both form the same
+FP32 logit chains, candidate sets, compensated refinements and FP64 finals,
+so their outputs agree bit for bit; the oracle pins the values."""
+import numpy as np
+import pytest
+
+import oracle
+import synth
+from parity_utils import check_insert
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+WIDE_TILE, TILE64, STREAMED = 1, 2, 3
+DEBUG_INSERT_TILE64 = 2
+
+
+@pytest.fixture(scope="module")
+def dev():
+    if not torch.cuda.is_available():
+        pytest.skip("no GPU")
+    import __graft_entry__
+    __graft_entry__.build()
+    return torch.device("cuda", 0)
+
+
+def T(x, dev):
+    return torch.from_numpy(np.ascontiguousarray(x)).to(dev)
+
+
+def build(dev, W, b, rows, batch, tile64, payload=None, consistency=False):
+    from paper_2608_13144_gb300.lipcache import LipCache
+    c = LipCache(W.shape[1], W.shape[0], len(rows), device=dev)
+    c.set_head(T(W, dev), T(b, dev))
+    if tile64:
+        c.set_debug(DEBUG_INSERT_TILE64)
+    idx, rad, n = [], [], 0
+    for s, e in synth.batches(len(rows), batch):
+        p = None if payload is None else T(payload[s:e], dev)
+        i, r, k = c.insert(T(rows[s:e], dev), p, consistency)
+        idx.append(i.cpu().numpy())
+        rad.append(r.cpu().numpy())
+        n += k
+    return c, np.concatenate(idx), np.concatenate(rad), n
+
+
+def same_bits(x, y):
+    x, y = np.asarray(x), np.asarray(y)
+    if x.dtype == np.float32:
+        x, y = x.view(np.uint32), y.view(np.uint32)
+    return x.shape == y.shape and np.array_equal(x, y)
+
+
+# (d, C, rows, insert batch): every compiled per-thread class count (1, 4, 7,
+# 13, 16), ragged last tiles, several tiles per CTA, one-tile batches
+SHAPES = [(16, 10, 1000, 1000), (64, 10, 20000, 20000), (128, 100, 30001, 30001), (128, 200, 40000, 16384),
+          (96, 250, 3000, 3000), (20, 40, 777, 100), (8, 3, 65, 65), (128, 200, 200, 64)]
+
+
+@pytest.mark.parametrize("d,C,N,batch", SHAPES)
+def test_wide_tile_bit_identical_and_oracle(dev, d, C, N, batch):
+    w = synth.WORKLOADS["cifar100"].scaled(d=d, C=C, components=C, N=N, n_queries=512, sphere_radius=4.0)
+    W, b = synth.head(w)
+    rows = synth.cache_rows(w)
+    Q, _ = synth.queries(w, rows)
+    a, ia, ra, na = build(dev, W, b, rows, batch, False)
+    assert a.info()["last_insert_kernel"] == WIDE_TILE
+    s, is_, rs, ns = build(dev, W, b, rows, batch, True)
+    assert s.info()["last_insert_kernel"] == TILE64
+    assert na == ns and same_bits(ia, is_) and same_bits(ra, rs)
+    ea, es = a.entries(), s.entries()
+    for k in ("keys", "radius", "label", "yG"):
+        assert same_bits(ea[k], es[k]), k
+    # the probe thresholds (not exported) agree through every probe result
+    for path in ("exact", "tensor"):
+        a.set_probe_path(path)
+        s.set_probe_path(path)
+        for x, y in zip(a.probe(T(Q, dev)), s.probe(T(Q, dev))):
+            assert same_bits(x.cpu().numpy(), y.cpu().numpy()), path
+    ref = oracle.build_cache(W, b, oracle.sigma_max(W), rows)
+    check_insert(ia, ra, na, ref, (W, b, rows, 1.0))
+    a.close()
+    s.close()
+
+
+def test_wide_tile_overflow_rows(dev):
+    """More candidate classes per row than the per-row slots (19 identical
+    head rows): the kernel recomputes those rows' logits and hands them to the
+    one-warp refinement; identical to the 64-row-tile kernel."""
+    rng = np.random.default_rng(21)
+    d, C = 32, 24
+    W = (rng.standard_normal((C, d)) / np.sqrt(d)).astype(np.float32)
+    W[1:20] = W[1]
+    b = (0.1 * rng.standard_normal(C)).astype(np.float32)
+    b[1:20] = b[1]
+    rows = np.concatenate([3 * W[0] + 0.3 * rng.standard_normal((700, d)),
+                           3 * W[1] + 0.3 * rng.standard_normal((700, d)),
+                           rng.standard_normal((600, d))]).astype(np.float32)
+    a, ia, ra, na = build(dev, W, b, rows, len(rows), False)
+    s, is_, rs, ns = build(dev, W, b, rows, len(rows), True)
+    assert a.info()["last_insert_kernel"] == WIDE_TILE
+    assert na == ns and same_bits(ia, is_) and same_bits(ra, rs)
+    ref = oracle.build_cache(W, b, oracle.sigma_max(W), rows)
+    check_insert(ia, ra, na, ref, (W, b, rows, 1.0))
+    a.close()
+    s.close()
+
+
+def test_wide_tile_payload_and_consistency(dev):
+    """Payload labels and the consistency flag go through the same finals."""
+    w = synth.WORKLOADS["cifar10"].scaled(N=6000)
+    W, b = synth.head(w)
+    rows = synth.cache_rows(w)
+    payload = (np.arange(len(rows)) % w.C).astype(np.int32)
+    a, ia, ra, na = build(dev, W, b, rows, 4096, False, payload, True)
+    s, is_, rs, ns = build(dev, W, b, rows, 4096, True, payload, True)
+    assert na == ns and same_bits(ia, is_) and same_bits(ra, rs)
+    ref = oracle.build_cache(W, b, oracle.sigma_max(W), rows, payload=payload, require_consistency=True)
+    check_insert(ia, ra, na, ref, (W, b, rows, 1.0))
+    a.close()
+    s.close()
+
+
+def test_kernel_choice(dev):
+    """Shapes outside the wide-tile kernel's limits take the other
+    kernels: the tight radius, d % 4 != 0, and heads too large for shared
+    memory."""
+    from paper_2608_13144_gb300.lipcache import LipCache
+    cases = [((64, 10), "tight", TILE64), ((33, 10), "conservative", TILE64),
+             ((256, 200), "conservative", STREAMED), ((128, 300), "conservative", STREAMED)]
+    rng = np.random.default_rng(5)
+    for (d, C), mode, kernel in cases:
+        W = (rng.standard_normal((C, d)) / np.sqrt(d)).astype(np.float32)
+        b = np.zeros(C, np.float32)
+        c = LipCache(d, C, 100, mode, device=dev)
+        c.set_head(T(W, dev), T(b, dev))
+        c.insert(T(rng.standard_normal((100, d)).astype(np.float32), dev))
+        assert c.info()["last_insert_kernel"] == kernel, (d, C, mode)
+        c.close()

@@ -206,3 +206,37 @@ def test_consistency_workload(dev, name):
     assert nh == orc["n_hits"]
     assert abs(nc - orc["n_consistent"]) <= int((~clear).sum())
     cache.close()
+
+
+def test_read_entries_roundtrip(dev):
+    """Entries read back equal the accepted rows, their radii and labels; a
+    cache rebuilt from them (keys + labels as payload) answers identically."""
+    w = synth.WORKLOADS["cifar10"]
+    W, b = synth.head(w)
+    rows = synth.cache_rows(w)[:3000]
+    Q, _ = synth.queries(w, rows)
+    Q = Q[:1000]
+    payload = (np.arange(len(rows)) % 7).astype(np.int32)
+    cache, _ = make_cache(dev, W, b, 4000)
+    idx, rad, n = cache.insert(T(rows, dev), T(payload, dev))
+    idx, rad = idx.cpu().numpy(), rad.cpu().numpy()
+    e = cache.entries()
+    acc = idx >= 0
+    np.testing.assert_array_equal(e["keys"], rows[acc])
+    np.testing.assert_array_equal(e["radius"], rad[acc])
+    np.testing.assert_array_equal(e["label"], payload[acc])
+    ref = oracle.certify(W, b, oracle.sigma_max(W), rows)
+    np.testing.assert_array_equal(e["yG"], ref["yG"][acc])
+    part = cache.entries(10, 5)
+    np.testing.assert_array_equal(part["keys"], e["keys"][10:15])
+    from paper_2608_13144_gb300._lib import LipCacheError
+    with pytest.raises(LipCacheError):
+        cache.entries(n - 2, 5)
+    again, _ = make_cache(dev, W, b, 4000)
+    again.insert(T(e["keys"], dev), T(e["label"], dev))
+    a = [t.cpu().numpy() for t in cache.probe(T(Q, dev))]
+    c = [t.cpu().numpy() for t in again.probe(T(Q, dev))]
+    for x, y in zip(a, c):
+        np.testing.assert_array_equal(x, y)
+    cache.close()
+    again.close()
