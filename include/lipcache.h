@@ -113,6 +113,8 @@ typedef struct lipcache_info {
   int32_t radius_policy;    /* LIPCACHE_POLICY_* the probe uses */
   int32_t last_insert_kernel; /* kernel that certified the last insert: LIPCACHE_INSERT_* (0 before any) */
   double policy_param;      /* tau (GLOBAL) or beta (INTERCLASS); 0 for CERTIFIED */
+  double insert_kernel_ms_total; /* summed certify-kernel time of timed inserts since the last reset */
+  int64_t insert_kernel_launches; /* number of timed certify kernels in insert_kernel_ms_total */
 } lipcache_info;
 
 /*

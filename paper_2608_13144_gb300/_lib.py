@@ -36,7 +36,8 @@ class Info(C.Structure):
                 ("last_probe_path", C.c_int32), ("last_probe_ms", C.c_float), ("num_sms", C.c_int32),
                 ("kernel_ms_total", C.c_double), ("kernel_launches", C.c_int64), ("last_grid", C.c_int32),
                 ("last_cluster", C.c_int32), ("radius_policy", C.c_int32), ("last_insert_kernel", C.c_int32),
-                ("policy_param", C.c_double)]
+                ("policy_param", C.c_double), ("insert_kernel_ms_total", C.c_double),
+                ("insert_kernel_launches", C.c_int64)]
 
 
 class LipCacheError(RuntimeError):

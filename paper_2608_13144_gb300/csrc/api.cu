@@ -132,9 +132,14 @@ void lc::harvest_timing(lipcache* h, bool all) {
     LC_CUDA(cudaEventSynchronize(h->tev1[slot]));
     float ms = 0.f;
     LC_CUDA(cudaEventElapsedTime(&ms, h->tev0[slot], h->tev1[slot]));
-    h->last_ms = ms;
-    h->t_ms_total += ms;
-    ++h->t_count;
+    if (h->t_kind[slot]) {
+      h->ti_ms_total += ms;
+      ++h->ti_count;
+    } else {
+      h->last_ms = ms;
+      h->t_ms_total += ms;
+      ++h->t_count;
+    }
     ++h->t_harvested;
   }
 }
@@ -530,6 +535,8 @@ LC_API lipcache_status lipcache_reset_stats(lipcache_t* h) {
     lc::harvest_timing(h, true);
     h->t_ms_total = 0.0;
     h->t_count = 0;
+    h->ti_ms_total = 0.0;
+    h->ti_count = 0;
     LC_CUDA(cudaMemset(h->stats, 0, sizeof(lc::DevStats)));
     LC_CUDA(cudaDeviceSynchronize());
   });
@@ -568,6 +575,8 @@ LC_API lipcache_status lipcache_get_info(lipcache_t* h, lipcache_info* info) {
     info->last_grid = h->last_grid;
     info->last_cluster = h->last_cluster;
     info->radius_policy = h->policy;
+    info->insert_kernel_ms_total = h->ti_ms_total;
+    info->insert_kernel_launches = h->ti_count;
     info->last_insert_kernel = h->last_insert_kernel;
     info->policy_param = h->policy_param;
   });

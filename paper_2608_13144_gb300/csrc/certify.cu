@@ -1421,6 +1421,17 @@ size_t certify_smem_bytes(int d, int C) {
 
 namespace {
 
+// With timing enabled: a slot of the event ring for a certify kernel, its
+// start recorded on `s` (-1 when timing is off).
+int timing_begin(lipcache* h, cudaStream_t s) {
+  if (!h->timing) return -1;
+  if (h->t_issued - h->t_harvested >= lipcache::kTimingRing) harvest_timing(h, false);
+  const int slot = (int)(h->t_issued % lipcache::kTimingRing);
+  h->t_kind[slot] = 1;
+  LC_CUDA(cudaEventRecord(h->tev0[slot], s));
+  return slot;
+}
+
 // Per-row certification of H (n rows) into the insert scratch: accept, y^G,
 // label, radius, probe thresholds, per-32-row ranks and counts.
 void launch_certify(lipcache* h, const float* H, int64_t n, const int32_t* payload, int require_consistency,
@@ -1473,6 +1484,7 @@ void launch_certify(lipcache* h, const float* H, int64_t n, const int32_t* paylo
   const size_t smem_wres = sizeof(float) * ((size_t)h->dpad * Cp + (size_t)h->dpad * kHStride +
                                             (size_t)kWTile * a.lstride + 1 + 4 * (size_t)h->C) +
                            sizeof(double) * 2 * kWarps * (size_t)(a.tight ? h->C : 0) + sizeof(TileSmem);
+  int slot = -1;
   const int ncg = wt_ncg(h->C);
   const bool vec16 = h->d % 4 == 0 && ((uintptr_t)H & 15) == 0;
   const WtLayout L = wt_layout(h->d, h->C, ncg > 0 ? ncg : 1);
@@ -1497,6 +1509,7 @@ void launch_certify(lipcache* h, const float* H, int64_t n, const int32_t* paylo
                                             : ncg == 13 ? k_certify_wt<13>
                                                         : k_certify_wt<16>;
     LC_CUDA(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)L.total));
+    slot = timing_begin(h, s);
     kern<<<grid, kThreads, L.total, s>>>(a, L, h->wt_prep, nb32);
     LC_LAUNCH_CHECK("k_certify_wt");
     h->last_insert_kernel = LIPCACHE_INSERT_WIDE_TILE;
@@ -1505,15 +1518,21 @@ void launch_certify(lipcache* h, const float* H, int64_t n, const int32_t* paylo
     const int grid = n_tiles < h->num_sms ? n_tiles : h->num_sms;
     LC_CUDA(cudaFuncSetAttribute(k_certify_wres, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_wres));
     const int vec = (h->d % 4 == 0 && ((uintptr_t)H & 15) == 0) ? 1 : 0;
+    slot = timing_begin(h, s);
     k_certify_wres<<<grid, kThreads, smem_wres, s>>>(a, Cp, h->dpad, n_tiles, vec);
     LC_LAUNCH_CHECK("k_certify_wres");
     h->last_insert_kernel = LIPCACHE_INSERT_TILE64;
   } else {
     const size_t smem = certify_smem_bytes(h->d, h->C);
     LC_CUDA(cudaFuncSetAttribute(k_certify, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+    slot = timing_begin(h, s);
     k_certify<<<nb, kThreads, smem, s>>>(a);
     LC_LAUNCH_CHECK("k_certify");
     h->last_insert_kernel = LIPCACHE_INSERT_STREAMED;
+  }
+  if (slot >= 0) {
+    LC_CUDA(cudaEventRecord(h->tev1[slot], s));
+    ++h->t_issued;
   }
 }
 

@@ -222,6 +222,9 @@ struct lipcache {
   int64_t t_issued = 0, t_harvested = 0;
   double t_ms_total = 0.0;
   int64_t t_count = 0;
+  uint8_t t_kind[kTimingRing] = {};  // per slot: 0 probe main kernel, 1 certify kernel
+  double ti_ms_total = 0.0;          // certify kernels
+  int64_t ti_count = 0;
   float last_ms = 0.f;
 
   double eps_rc = 0.0, c_scr = 0.0;

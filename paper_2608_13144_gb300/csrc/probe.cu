@@ -186,6 +186,7 @@ void probe(lipcache* h, const float* Q, int64_t B, int64_t* out_index, int32_t* 
     if (h->timing) {
       if (h->t_issued - h->t_harvested >= lipcache::kTimingRing) harvest_timing(h, false);
       slot = (int)(h->t_issued % lipcache::kTimingRing);
+      h->t_kind[slot] = 0;
       LC_CUDA(cudaEventRecord(h->tev0[slot], s));
     }
     if (path != LIPCACHE_PROBE_EXACT) {

@@ -61,8 +61,12 @@ def test_insert_roofline_arithmetic():
     import bench
     import synth
     w = synth.WORKLOADS["scale"]
-    r = bench.insert_summary(w, w.N, 20.0, 152, {"sm_max_mhz": 2070})
+    r = bench.insert_summary(w, w.N, 20.0, 152, {"sm_max_mhz": 2070}, kernel=("k_certify_wt", 8.0, 62))
     assert r["rows_per_s"] == w.N / 0.02
-    assert abs(r["roofline"]["achieved"] - 2 * w.N * w.C * w.d / 0.02 / 1e12) < 1e-9
+    assert abs(r["e2e"]["achieved"] - 2 * w.N * w.C * w.d / 0.02 / 1e12) < 1e-9
+    assert abs(r["roofline"]["achieved"] - 2 * w.N * w.C * w.d / 0.008 / 1e12) < 1e-9
     assert abs(r["roofline"]["peak"] - 152 * 128 * 2 * 2070e6 / 1e12) < 1e-9
-    assert r["roofline"]["bound"] == "alu" and 0 < r["roofline"]["frac"] < 1
+    assert r["roofline"]["bound"] == "alu" and 0 < r["e2e"]["frac"] < r["roofline"]["frac"] < 1
+    assert r["kernel"] == "k_certify_wt" and abs(r["kernel_ms"] - 8.0 / 62) < 1e-12
+    r = bench.insert_summary(w, w.N, 20.0, 152, {"sm_max_mhz": 2070})
+    assert r["roofline"]["achieved"] == r["e2e"]["achieved"]
