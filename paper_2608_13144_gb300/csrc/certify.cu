@@ -862,6 +862,168 @@ struct WtLayout {
   uint32_t off_h, off_e, off_tile, total;
 };
 
+// Steps 2-3 of k_certify_wt for one chunk, with ROWS rows per thread (8 for
+// chunks of more than 64 rows, 4 otherwise, so that a short chunk still keeps
+// two warps on every sub-partition): the FP32 logits, the interval pass, the
+// candidate slots and this warp's share of the pair list.
+template <int NCG, int ROWS>
+__device__ __forceinline__ void wt_chunk_logits(const CertArgs& a, const float* __restrict__ wT,
+                                                const float* __restrict__ hT, const float* __restrict__ eA,
+                                                const float* __restrict__ eB, const float* __restrict__ bp, WtTile& ts,
+                                                int GS, int wst, int nrows, int warp, int lane) {
+  constexpr int NPR = NCG / 2;  // class pairs per thread
+  constexpr bool kOdd = (NCG & 1) != 0;
+  const int d = a.d, C = a.C;
+  const int cg = lane & 15, rg = warp * 2 + (lane >> 4);  // rows ROWS rg .. ROWS rg + ROWS - 1, classes cg NCG ..
+  const float* wp = wT + cg * GS;
+  if (2 * ROWS * warp < nrows) {  // this warp's 2 ROWS rows hold at least one live row
+    // 2. FP32 logits of rows ROWS rg .. ROWS rg + ROWS - 1 and classes cg NCG .. cg NCG + NCG - 1
+    uint64_t accp[ROWS][NPR > 0 ? NPR : 1];
+    float accs[ROWS];
+#pragma unroll
+    for (int i = 0; i < ROWS; ++i) {
+#pragma unroll
+      for (int m = 0; m < NPR; ++m) accp[i][m] = 0ull;
+      accs[i] = 0.f;
+    }
+    {
+      const float* hb = hT + ROWS * rg;
+#pragma unroll 2
+      for (int k = 0; k < d; ++k) {
+        float hv[ROWS];
+#pragma unroll
+        for (int v4 = 0; v4 < ROWS / 4; ++v4) {
+          const float4 x = *reinterpret_cast<const float4*>(hb + (size_t)k * kWtHst + 4 * v4);
+          hv[4 * v4] = x.x;
+          hv[4 * v4 + 1] = x.y;
+          hv[4 * v4 + 2] = x.z;
+          hv[4 * v4 + 3] = x.w;
+        }
+        const float* wk = wp + (size_t)k * wst;
+        uint64_t wv[NPR > 0 ? NPR : 1];
+#pragma unroll
+        for (int m = 0; m < NPR; ++m) wv[m] = *reinterpret_cast<const uint64_t*>(wk + 2 * m);
+        const float w1 = kOdd ? wk[NCG - 1] : 0.f;
+#pragma unroll
+        for (int i = 0; i < ROWS; ++i) {
+          const uint32_t hb32 = __float_as_uint(hv[i]);
+          const uint64_t hh = ptx::pack_f32x2(hb32, hb32);
+#pragma unroll
+          for (int m = 0; m < NPR; ++m) accp[i][m] = ptx::fma_f32x2(wv[m], hh, accp[i][m]);
+          if (kOdd) accs[i] = __fmaf_rn(w1, hv[i], accs[i]);
+        }
+      }
+    }
+    // 3. interval lower ends, each row's L2, candidates, two rows at a time.
+    // The loop stays rolled (its body runs once per chunk and would not stay
+    // in the instruction cache unrolled); rows i, i + 1 are always in
+    // accp[0..1], the rest shift down. Branch-free over the classes (a
+    // divergent branch per class would serialise them): dead classes get
+    // -inf lower ends and no candidacy.
+#pragma unroll 1
+    for (int i = 0; i < ROWS; i += 2) {
+      float sv[2][NCG], E[2][NCG], l1[2], l2[2], hn[2];
+      int r[2];
+#pragma unroll
+      for (int u = 0; u < 2; ++u) {
+        r[u] = ROWS * rg + i + u;
+        const float kn = (ts.knp[0][r[u]] + ts.knp[1][r[u]]) + (ts.knp[2][r[u]] + ts.knp[3][r[u]]);
+        hn[u] = norm_upper(kn);
+#pragma unroll
+        for (int m = 0; m < NPR; ++m) {
+          sv[u][2 * m] = __fadd_rn(__uint_as_float((uint32_t)accp[u][m]), bp[cg * GS + 2 * m]);
+          sv[u][2 * m + 1] = __fadd_rn(__uint_as_float((uint32_t)(accp[u][m] >> 32)), bp[cg * GS + 2 * m + 1]);
+        }
+        if (kOdd) sv[u][NCG - 1] = __fadd_rn(accs[u], bp[cg * GS + NCG - 1]);
+      }
+#pragma unroll
+      for (int ii = 0; ii < ROWS - 2; ++ii) {
+#pragma unroll
+        for (int m = 0; m < NPR; ++m) accp[ii][m] = accp[ii + 2][m];
+        accs[ii] = accs[ii + 2];
+      }
+#pragma unroll
+      for (int u = 0; u < 2; ++u) {
+        l1[u] = -INFINITY;
+        l2[u] = -INFINITY;
+#pragma unroll
+        for (int jc = 0; jc < NCG; ++jc) {
+          E[u][jc] = __fmaf_ru(eA[cg * GS + jc], hn[u], __fmaf_ru(fabsf(sv[u][jc]), 2.3841858e-07f, eB[cg * GS + jc]));
+          float lo = __fsub_rd(sv[u][jc], E[u][jc]);
+          lo = (lo == lo && cg * NCG + jc < C) ? lo : -INFINITY;
+          l2[u] = fmaxf(l2[u], fminf(l1[u], lo));
+          l1[u] = fmaxf(l1[u], lo);
+        }
+      }
+#pragma unroll
+      for (int o = 1; o < 16; o <<= 1) {
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+          const float o1 = __shfl_xor_sync(kFull, l1[u], o), o2 = __shfl_xor_sync(kFull, l2[u], o);
+          l2[u] = fmaxf(l2[u], fminf(l1[u], o1));
+          l1[u] = fmaxf(l1[u], o1);
+          l2[u] = fmaxf(l2[u], fminf(l1[u], o2));
+          l1[u] = fmaxf(l1[u], o2);
+        }
+      }
+      unsigned cm[2];  // candidate bits of this lane's classes
+      int incl[2], mine[2];
+#pragma unroll
+      for (int u = 0; u < 2; ++u) {
+        cm[u] = 0;
+#pragma unroll
+        for (int jc = 0; jc < NCG; ++jc)
+          cm[u] |= (unsigned)(cg * NCG + jc < C && __fadd_ru(sv[u][jc], E[u][jc]) >= l2[u]) << jc;
+        cm[u] = r[u] < nrows ? cm[u] : 0u;
+        mine[u] = __popc(cm[u]);
+        incl[u] = mine[u];
+      }
+      // slots of each row: the 16 lanes of this half-warp own it; prefix
+      // sum of their candidate counts
+#pragma unroll
+      for (int o = 1; o < 16; o <<= 1) {
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+          const int t = __shfl_up_sync(kFull, incl[u], o, 16);
+          if (cg >= o) incl[u] += t;
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < 2; ++u) {
+        int slot = incl[u] - mine[u];
+        unsigned m = cm[u];
+        while (m) {
+          const int jc = __ffs(m) - 1;
+          m &= m - 1;
+          if (slot < kMaxCand) ts.cls[r[u]][slot] = (uint8_t)(cg * NCG + jc);
+          ++slot;
+        }
+        if (cg == 15) {
+          ts.ncand[r[u]] = incl[u];
+          ts.hn[r[u]] = hn[u];
+        }
+      }
+    }
+  }
+  // this warp's 2 ROWS rows into the pair list: one reservation per warp
+  __syncwarp();
+  {
+    const int R = ROWS * (2 * warp + lane / ROWS) + lane % ROWS;
+    const int n = lane < 2 * ROWS ? min(ts.ncand[R], kMaxCand) : 0;
+    int incl = n;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int t = __shfl_up_sync(kFull, incl, o);
+      if (lane >= o) incl += t;
+    }
+    const int total = __shfl_sync(kFull, incl, 31);
+    int base = 0;
+    if (lane == 0 && total) base = atomicAdd(&ts.npairs, total);
+    base = __shfl_sync(kFull, base, 0) + incl - n;
+    for (int sl = 0; sl < n; ++sl) ts.pairs[base + sl] = R | (sl << 8) | ((int)ts.cls[R][sl] << 16);
+  }
+}
+
 template <int NCG>
 __global__ void __launch_bounds__(kThreads, 1) k_certify_wt(CertArgs a, WtLayout L, const float* __restrict__ prep,
                                                              int64_t nb32) {
@@ -899,8 +1061,6 @@ __global__ void __launch_bounds__(kThreads, 1) k_certify_wt(CertArgs a, WtLayout
       }
     }
   }
-  const int cg = lane & 15, rg = warp * 2 + (lane >> 4);  // product: rows 8 rg .. 8 rg + 7, classes cg NCG ..
-  const float* wp = wT + cg * GS;
   const int g8 = tid / kGroup, sub = tid % kGroup;  // refinement groups
   const int q = warp & 3, dq = (d + 3) / 4, k_lo = q * dq, k_hi = min(d, k_lo + dq);  // load quarter
   // this CTA's rows: a contiguous range of whole 32-row blocks (balanced over
@@ -973,146 +1133,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_certify_wt(CertArgs a, WtLayout
       ts.novf = 0;
     }
     __syncthreads();
-    if (16 * warp < nrows) {  // this warp's 16 rows hold at least one live row
-      // 2. FP32 logits of rows 8 rg .. 8 rg + 7 and classes cg NCG .. cg NCG + NCG - 1
-      uint64_t accp[8][NPR > 0 ? NPR : 1];
-      float accs[8];
-#pragma unroll
-      for (int i = 0; i < 8; ++i) {
-#pragma unroll
-        for (int m = 0; m < NPR; ++m) accp[i][m] = 0ull;
-        accs[i] = 0.f;
-      }
-      {
-        const float* hb = hT + 8 * rg;
-#pragma unroll 2
-        for (int k = 0; k < d; ++k) {
-          const float4 x0 = *reinterpret_cast<const float4*>(hb + (size_t)k * kWtHst);
-          const float4 x1 = *reinterpret_cast<const float4*>(hb + (size_t)k * kWtHst + 4);
-          const float hv[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
-          const float* wk = wp + (size_t)k * wst;
-          uint64_t wv[NPR > 0 ? NPR : 1];
-#pragma unroll
-          for (int m = 0; m < NPR; ++m) wv[m] = *reinterpret_cast<const uint64_t*>(wk + 2 * m);
-          const float w1 = kOdd ? wk[NCG - 1] : 0.f;
-#pragma unroll
-          for (int i = 0; i < 8; ++i) {
-            const uint32_t hb32 = __float_as_uint(hv[i]);
-            const uint64_t hh = ptx::pack_f32x2(hb32, hb32);
-#pragma unroll
-            for (int m = 0; m < NPR; ++m) accp[i][m] = ptx::fma_f32x2(wv[m], hh, accp[i][m]);
-            if (kOdd) accs[i] = __fmaf_rn(w1, hv[i], accs[i]);
-          }
-        }
-      }
-      // 3. interval lower ends, each row's L2, candidates, two rows at a time.
-      // The loop stays rolled (its body runs once per chunk and would not stay
-      // in the instruction cache unrolled); rows i, i + 1 are always in
-      // accp[0..1], the rest shift down. Branch-free over the classes (a
-      // divergent branch per class would serialise them): dead classes get
-      // -inf lower ends and no candidacy.
-#pragma unroll 1
-      for (int i = 0; i < 8; i += 2) {
-        float sv[2][NCG], E[2][NCG], l1[2], l2[2], hn[2];
-        int r[2];
-#pragma unroll
-        for (int u = 0; u < 2; ++u) {
-          r[u] = 8 * rg + i + u;
-          const float kn = (ts.knp[0][r[u]] + ts.knp[1][r[u]]) + (ts.knp[2][r[u]] + ts.knp[3][r[u]]);
-          hn[u] = norm_upper(kn);
-#pragma unroll
-          for (int m = 0; m < NPR; ++m) {
-            sv[u][2 * m] = __fadd_rn(__uint_as_float((uint32_t)accp[u][m]), bp[cg * GS + 2 * m]);
-            sv[u][2 * m + 1] = __fadd_rn(__uint_as_float((uint32_t)(accp[u][m] >> 32)), bp[cg * GS + 2 * m + 1]);
-          }
-          if (kOdd) sv[u][NCG - 1] = __fadd_rn(accs[u], bp[cg * GS + NCG - 1]);
-        }
-#pragma unroll
-        for (int ii = 0; ii < 6; ++ii) {
-#pragma unroll
-          for (int m = 0; m < NPR; ++m) accp[ii][m] = accp[ii + 2][m];
-          accs[ii] = accs[ii + 2];
-        }
-#pragma unroll
-        for (int u = 0; u < 2; ++u) {
-          l1[u] = -INFINITY;
-          l2[u] = -INFINITY;
-#pragma unroll
-          for (int jc = 0; jc < NCG; ++jc) {
-            E[u][jc] = __fmaf_ru(eA[cg * GS + jc], hn[u], __fmaf_ru(fabsf(sv[u][jc]), 2.3841858e-07f, eB[cg * GS + jc]));
-            float lo = __fsub_rd(sv[u][jc], E[u][jc]);
-            lo = (lo == lo && cg * NCG + jc < C) ? lo : -INFINITY;
-            l2[u] = fmaxf(l2[u], fminf(l1[u], lo));
-            l1[u] = fmaxf(l1[u], lo);
-          }
-        }
-#pragma unroll
-        for (int o = 1; o < 16; o <<= 1) {
-#pragma unroll
-          for (int u = 0; u < 2; ++u) {
-            const float o1 = __shfl_xor_sync(kFull, l1[u], o), o2 = __shfl_xor_sync(kFull, l2[u], o);
-            l2[u] = fmaxf(l2[u], fminf(l1[u], o1));
-            l1[u] = fmaxf(l1[u], o1);
-            l2[u] = fmaxf(l2[u], fminf(l1[u], o2));
-            l1[u] = fmaxf(l1[u], o2);
-          }
-        }
-        unsigned cm[2];  // candidate bits of this lane's classes
-        int incl[2], mine[2];
-#pragma unroll
-        for (int u = 0; u < 2; ++u) {
-          cm[u] = 0;
-#pragma unroll
-          for (int jc = 0; jc < NCG; ++jc)
-            cm[u] |= (unsigned)(cg * NCG + jc < C && __fadd_ru(sv[u][jc], E[u][jc]) >= l2[u]) << jc;
-          cm[u] = r[u] < nrows ? cm[u] : 0u;
-          mine[u] = __popc(cm[u]);
-          incl[u] = mine[u];
-        }
-        // slots of each row: the 16 lanes of this half-warp own it; prefix
-        // sum of their candidate counts
-#pragma unroll
-        for (int o = 1; o < 16; o <<= 1) {
-#pragma unroll
-          for (int u = 0; u < 2; ++u) {
-            const int t = __shfl_up_sync(kFull, incl[u], o, 16);
-            if (cg >= o) incl[u] += t;
-          }
-        }
-#pragma unroll
-        for (int u = 0; u < 2; ++u) {
-          int slot = incl[u] - mine[u];
-          unsigned m = cm[u];
-          while (m) {
-            const int jc = __ffs(m) - 1;
-            m &= m - 1;
-            if (slot < kMaxCand) ts.cls[r[u]][slot] = (uint8_t)(cg * NCG + jc);
-            ++slot;
-          }
-          if (cg == 15) {
-            ts.ncand[r[u]] = incl[u];
-            ts.hn[r[u]] = hn[u];
-          }
-        }
-      }
-    }
-    // this warp's 16 rows into the pair list: one reservation per warp
-    __syncwarp();
-    {
-      const int R = 8 * (2 * warp + ((lane >> 3) & 1)) + (lane & 7);
-      const int n = lane < 16 ? min(ts.ncand[R], kMaxCand) : 0;
-      int incl = n;
-#pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        const int t = __shfl_up_sync(kFull, incl, o);
-        if (lane >= o) incl += t;
-      }
-      const int total = __shfl_sync(kFull, incl, 31);
-      int base = 0;
-      if (lane == 0 && total) base = atomicAdd(&ts.npairs, total);
-      base = __shfl_sync(kFull, base, 0) + incl - n;
-      for (int sl = 0; sl < n; ++sl) ts.pairs[base + sl] = R | (sl << 8) | ((int)ts.cls[R][sl] << 16);
-    }
+    if (nrows > 64)
+      wt_chunk_logits<NCG, 8>(a, wT, hT, eA, eB, bp, ts, GS, wst, nrows, warp, lane);
+    else
+      wt_chunk_logits<NCG, 4>(a, wT, hT, eA, eB, bp, ts, GS, wst, nrows, warp, lane);
     __syncthreads();
     // 4. refine the pairs, kGroup lanes a pair, two pairs a group at a time
     constexpr int kGroups = kThreads / kGroup;
