@@ -323,6 +323,17 @@ lipcache_status lipcache_read_entries(lipcache_t* h, int64_t first, int64_t n, f
                                       int32_t* label_host, int32_t* yG_host, lipcache_stream_t stream);
 
 /*
+ * Copy the head set by lipcache_set_head back to the host (with
+ * lipcache_read_entries, what a checkpoint needs: a cache is restored by
+ * set_head and re-inserting the entries' keys with their labels as payload,
+ * which re-certifies them to the same radii).
+ *   W_host  C x d FP32 row-major (host), nullable
+ *   b_host  C FP32 (host), nullable
+ * Synchronises `stream`. Errors: E_STATE (no head), E_CUDA.
+ */
+lipcache_status lipcache_read_head(lipcache_t* h, float* W_host, float* b_host, lipcache_stream_t stream);
+
+/*
  * Test hooks for failure detection. LIPCACHE_DEBUG_STALL_PROBE makes the MMA
  * issuer of the tensor probe kernels first wait on an mbarrier that nothing
  * arrives on: the bounded wait (~2^31 cycles, about a second) expires, the

@@ -21,7 +21,7 @@ PROBE_AUTO, PROBE_TENSOR, PROBE_EXACT, PROBE_TENSOR_SINGLE, PROBE_TENSOR_PAIR = 
 # Every symbol the header declares; tests check the library exports them all.
 EXPORTS = ["lipcache_create", "lipcache_set_head", "lipcache_insert", "lipcache_probe", "lipcache_probe_host",
            "lipcache_probe_noalloc", "lipcache_probe_writeback", "lipcache_consistency",
-           "lipcache_set_radius_policy", "lipcache_insert_select", "lipcache_set_debug", "lipcache_read_entries",
+           "lipcache_set_radius_policy", "lipcache_insert_select", "lipcache_set_debug", "lipcache_read_entries", "lipcache_read_head",
            "lipcache_set_probe_path", "lipcache_set_radius_scale", "lipcache_set_spectral_options",
            "lipcache_reserve", "lipcache_enable_timing", "lipcache_get_info", "lipcache_reset_stats",
            "lipcache_size", "lipcache_destroy", "lipcache_last_error"]
@@ -71,6 +71,7 @@ def load(path: str = LIB_PATH):
         "lipcache_insert_select": ([vp, vp, i64, vp, i32, i32, i64, i32, vp, vp, C.POINTER(i64), vp], C.c_int),
         "lipcache_set_debug": ([vp, i32], C.c_int),
         "lipcache_read_entries": ([vp, i64, i64, vp, vp, vp, vp, vp], C.c_int),
+        "lipcache_read_head": ([vp, vp, vp, vp], C.c_int),
         "lipcache_set_probe_path": ([vp, i32], C.c_int),
         "lipcache_set_radius_scale": ([vp, f64], C.c_int),
         "lipcache_set_spectral_options": ([vp, i32, i32], C.c_int),

@@ -1,6 +1,8 @@
 // C ABI of the certified cache lookup: argument checks, ownership of the
 // cache table and scratch memory, and kernel launches on the caller's stream.
 // Declarations and contracts: include/lipcache.h.
+#include <nvtx3/nvToolsExt.h>
+
 #include <cstdio>
 #include <cstring>
 #include <string>
@@ -17,6 +19,13 @@ void reserve_probe(lipcache* h, int64_t max_batch);
 namespace {
 
 thread_local std::string g_err;
+
+// An NVTX range around an entry point (a no-op unless a profiler is attached),
+// so that `ncu --nvtx` can select a call's kernels.
+struct Range {
+  explicit Range(const char* name) { nvtxRangePushA(name); }
+  ~Range() { nvtxRangePop(); }
+};
 
 template <typename F>
 lipcache_status guarded(F&& f) {
@@ -231,6 +240,7 @@ LC_API int64_t lipcache_size(const lipcache_t* h) { return h ? h->size : 0; }
 LC_API lipcache_status lipcache_set_head(lipcache_t* h, const float* W, const float* b, double* sigma_out,
                                          lipcache_stream_t stream) {
   return guarded([&] {
+    Range nvtx_range("lipcache_set_head");
     check_handle(h);
     LC_REQUIRE(W != nullptr && b != nullptr, LIPCACHE_E_INVALID, "W and b must be device pointers");
     LC_REQUIRE(h->size == 0, LIPCACHE_E_STATE, "set_head requires an empty cache (radii depend on W)");
@@ -262,6 +272,7 @@ LC_API lipcache_status lipcache_insert(lipcache_t* h, const float* H, int64_t n,
                                        int64_t* n_accepted, lipcache_stream_t stream) {
   if (n_accepted) *n_accepted = 0;
   return guarded([&] {
+    Range nvtx_range("lipcache_insert");
     check_handle(h);
     LC_REQUIRE(h->head_set, LIPCACHE_E_STATE, "insert before set_head");
     LC_REQUIRE(n >= 0, LIPCACHE_E_INVALID, "n must be >= 0");
@@ -288,6 +299,7 @@ LC_API lipcache_status lipcache_insert(lipcache_t* h, const float* H, int64_t n,
 LC_API lipcache_status lipcache_probe(lipcache_t* h, const float* Q, int64_t B, int64_t* out_index,
                                       int32_t* out_label, float* out_dist, lipcache_stream_t stream) {
   return guarded([&] {
+    Range nvtx_range("lipcache_probe");
     check_handle(h);
     LC_REQUIRE(h->head_set, LIPCACHE_E_STATE, "probe before set_head");
     LC_REQUIRE(B >= 0 && B <= (1LL << 22), LIPCACHE_E_INVALID, "B must be in [0, 2^22]");
@@ -305,6 +317,7 @@ LC_API lipcache_status lipcache_insert_select(lipcache_t* h, const float* H, int
                                               int64_t* n_selected, lipcache_stream_t stream) {
   if (n_selected) *n_selected = 0;
   return guarded([&] {
+    Range nvtx_range("lipcache_insert_select");
     check_handle(h);
     LC_REQUIRE(strategy == LIPCACHE_SELECT_ALL || strategy == LIPCACHE_SELECT_RADIUS_DEDUP ||
                    strategy == LIPCACHE_SELECT_KCENTER,
@@ -348,6 +361,7 @@ LC_API lipcache_status lipcache_probe_writeback(lipcache_t* h, const float* Q, i
                                                 lipcache_stream_t stream) {
   if (n_inserted) *n_inserted = 0;
   return guarded([&] {
+    Range nvtx_range("lipcache_probe_writeback");
     check_handle(h);
     LC_REQUIRE(h->head_set, LIPCACHE_E_STATE, "probe before set_head");
     LC_REQUIRE(B >= 0 && B <= (1LL << 22), LIPCACHE_E_INVALID, "B must be in [0, 2^22]");
@@ -379,6 +393,7 @@ LC_API lipcache_status lipcache_consistency(lipcache_t* h, const float* Q, int64
   if (n_hits) *n_hits = 0;
   if (n_consistent) *n_consistent = 0;
   return guarded([&] {
+    Range nvtx_range("lipcache_consistency");
     check_handle(h);
     LC_REQUIRE(h->head_set, LIPCACHE_E_STATE, "consistency check before set_head");
     LC_REQUIRE(B >= 0 && B <= (1LL << 22), LIPCACHE_E_INVALID, "B must be in [0, 2^22]");
@@ -399,6 +414,7 @@ LC_API lipcache_status lipcache_consistency(lipcache_t* h, const float* Q, int64
 LC_API lipcache_status lipcache_set_radius_policy(lipcache_t* h, int32_t policy, double param, double* rho_out,
                                                   lipcache_stream_t stream) {
   return guarded([&] {
+    Range nvtx_range("lipcache_set_radius_policy");
     check_handle(h);
     LC_REQUIRE(h->head_set, LIPCACHE_E_STATE, "set_radius_policy before set_head");
     LC_REQUIRE(policy == LIPCACHE_POLICY_CERTIFIED || policy == LIPCACHE_POLICY_GLOBAL ||
@@ -418,6 +434,7 @@ LC_API lipcache_status lipcache_read_entries(lipcache_t* h, int64_t first, int64
                                              float* radius_host, int32_t* label_host, int32_t* yG_host,
                                              lipcache_stream_t stream) {
   return guarded([&] {
+    Range nvtx_range("lipcache_read_entries");
     check_handle(h);
     LC_REQUIRE(first >= 0 && n >= 0 && first + n <= h->size, LIPCACHE_E_INVALID, "entries outside [0, size)");
     if (n == 0) return;
@@ -439,6 +456,19 @@ LC_API lipcache_status lipcache_read_entries(lipcache_t* h, int64_t first, int64
   });
 }
 
+LC_API lipcache_status lipcache_read_head(lipcache_t* h, float* W_host, float* b_host, lipcache_stream_t stream) {
+  return guarded([&] {
+    check_handle(h);
+    LC_REQUIRE(h->head_set, LIPCACHE_E_STATE, "read_head before set_head");
+    use_device(h);
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    if (W_host)
+      LC_CUDA(cudaMemcpyAsync(W_host, h->W, sizeof(float) * (size_t)h->C * h->d, cudaMemcpyDeviceToHost, s));
+    if (b_host) LC_CUDA(cudaMemcpyAsync(b_host, h->b, sizeof(float) * (size_t)h->C, cudaMemcpyDeviceToHost, s));
+    LC_CUDA(cudaStreamSynchronize(s));
+  });
+}
+
 LC_API lipcache_status lipcache_set_debug(lipcache_t* h, int32_t flags) {
   return guarded([&] {
     check_handle(h);
@@ -451,6 +481,7 @@ LC_API lipcache_status lipcache_set_debug(lipcache_t* h, int32_t flags) {
 LC_API lipcache_status lipcache_probe_host(lipcache_t* h, const float* Q_host, int64_t B, int64_t* out_index_host,
                                            int32_t* out_label_host, float* out_dist_host, lipcache_stream_t stream) {
   return guarded([&] {
+    Range nvtx_range("lipcache_probe_host");
     check_handle(h);
     LC_REQUIRE(h->head_set, LIPCACHE_E_STATE, "probe before set_head");
     LC_REQUIRE(B >= 0 && B <= (1LL << 22), LIPCACHE_E_INVALID, "B must be in [0, 2^22]");

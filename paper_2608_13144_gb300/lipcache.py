@@ -215,6 +215,53 @@ class LipCache:
                                            label.ctypes.data, yG.ctypes.data, _stream(self.device)))
         return {"keys": keys, "radius": radius, "label": label, "yG": yG}
 
+    def head(self) -> tuple[np.ndarray, np.ndarray]:
+        """The head (W, b) set by set_head, as numpy arrays."""
+        W = np.empty((self.C, self.d), dtype=np.float32)
+        b = np.empty(self.C, dtype=np.float32)
+        check(self.L.lipcache_read_head(self._h, W.ctypes.data, b.ctypes.data, _stream(self.device)))
+        return W, b
+
+    def save(self, path: str):
+        """Checkpoint: the configuration, the head and the entries' keys and
+        labels (numpy .npz). LipCache.load re-certifies the keys under the
+        head, which gives the same radii; radii are stored only to check it."""
+        inf = self.info()
+        W, b = self.head()
+        e = self.entries()
+        mode = {v: k for k, v in RADIUS_MODES.items()}[inf["radius_mode"]]
+        path_name = {v: k for k, v in PROBE_PATHS.items()}.get(inf["probe_path"], "auto")
+        policy = {v: k for k, v in RADIUS_POLICIES.items()}[inf["radius_policy"]]
+        np.savez(path, d=self.d, C=self.C, capacity=inf["capacity"], radius_mode=mode,
+                 radius_scale=inf["radius_scale"], probe_path=path_name, radius_policy=policy,
+                 policy_param=inf["policy_param"], sigma=inf["sigma"], W=W, b=b, keys=e["keys"],
+                 label=e["label"], radius=e["radius"])
+
+    @classmethod
+    def load(cls, path: str, device: int | torch.device | None = None, batch: int = 65536) -> "LipCache":
+        """Restore a checkpoint written by save: create, set_head, re-insert
+        the keys with their labels as payload (Algorithm 1 again), restore
+        the probe path and radius policy. Raises if sigma or a radius
+        differs from the saved one."""
+        z = np.load(path if str(path).endswith(".npz") else str(path) + ".npz")
+        c = cls(int(z["d"]), int(z["C"]), int(z["capacity"]), str(z["radius_mode"]), device=device)
+        c.set_radius_scale(float(z["radius_scale"]))
+        sigma = c.set_head(torch.from_numpy(z["W"]).to(c.device), torch.from_numpy(z["b"]).to(c.device))
+        if sigma != float(z["sigma"]):
+            raise ValueError(f"sigma of the restored head {sigma!r} differs from the saved {float(z['sigma'])!r}")
+        keys, label = z["keys"], z["label"]
+        for s in range(0, len(keys), batch):
+            idx, _, n = c.insert(torch.from_numpy(keys[s:s + batch]).to(c.device),
+                                 torch.from_numpy(label[s:s + batch]).to(c.device))
+            if n != len(keys[s:s + batch]):
+                raise ValueError("a saved entry was not re-certified")
+        if not np.array_equal(c.entries()["radius"].view(np.uint32), z["radius"].view(np.uint32)):
+            raise ValueError("re-certified radii differ from the saved ones")
+        c.set_probe_path(str(z["probe_path"]))
+        if str(z["radius_policy"]) != "certified":
+            c.set_radius_policy(str(z["radius_policy"]), float(z["policy_param"]))
+        return c
+
     def set_debug(self, flags: int):
         """Failure-detection test hooks (LIPCACHE_DEBUG_*; 0 = off)."""
         check(self.L.lipcache_set_debug(self._h, int(flags)))

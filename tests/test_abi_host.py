@@ -71,6 +71,7 @@ def test_null_handle_calls(lib):
     assert lib.lipcache_set_radius_policy(None, 1, 1.0, None, None) == 1
     assert lib.lipcache_set_debug(None, 0) == 1
     assert lib.lipcache_read_entries(None, 0, 0, None, None, None, None, None) == 1
+    assert lib.lipcache_read_head(None, None, None, None) == 1
 
 
 def test_create_without_gpu_fails_cleanly(lib):

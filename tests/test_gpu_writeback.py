@@ -240,3 +240,40 @@ def test_read_entries_roundtrip(dev):
         np.testing.assert_array_equal(x, y)
     cache.close()
     again.close()
+
+
+@pytest.mark.parametrize("mode,policy", [("conservative", "certified"), ("tight", "interclass")])
+def test_checkpoint_roundtrip(dev, tmp_path, mode, policy):
+    """save / load: the restored cache has the same head, entries (keys,
+    radii re-certified to the same bits, labels, y^G), probe path and radius
+    policy, and answers every probe identically."""
+    from paper_2608_13144_gb300.lipcache import LipCache
+    w = synth.WORKLOADS["cifar10"]
+    W, b = synth.head(w)
+    rows = synth.cache_rows(w)[:5000]
+    Q, _ = synth.queries(w, rows)
+    Q = Q[:1500]
+    cache = LipCache(w.d, w.C, 6000, mode, device=dev)
+    cache.set_radius_scale(0.9)
+    cache.set_head(T(W, dev), T(b, dev))
+    cache.insert(T(rows, dev), T((np.arange(len(rows)) % 3).astype(np.int32), dev))
+    cache.set_probe_path("exact")
+    if policy != "certified":
+        cache.set_radius_policy(policy, 0.8)
+    path = str(tmp_path / "cache.npz")
+    cache.save(path)
+    again = LipCache.load(path, device=dev)
+    a, c = cache.info(), again.info()
+    for k in ("d", "C", "capacity", "size", "radius_mode", "radius_scale", "sigma", "probe_path", "radius_policy",
+              "policy_param"):
+        assert a[k] == c[k], k
+    Wa, ba = again.head()
+    np.testing.assert_array_equal(Wa, W)
+    np.testing.assert_array_equal(ba, b)
+    ea, ec = cache.entries(), again.entries()
+    for k in ("keys", "radius", "label", "yG"):
+        np.testing.assert_array_equal(ea[k], ec[k])
+    for x, y in zip(cache.probe(T(Q, dev)), again.probe(T(Q, dev))):
+        np.testing.assert_array_equal(x.cpu().numpy(), y.cpu().numpy())
+    cache.close()
+    again.close()
