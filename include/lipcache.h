@@ -73,7 +73,7 @@ typedef enum lipcache_status {
 #define LIPCACHE_POLICY_INTERCLASS 2 /* radius from inter-class centroid distances (Sec. 5.4) */
 
 /* Probe kernels. All return identical results; they differ in speed. */
-#define LIPCACHE_PROBE_AUTO 0          /* tensor path when supported (d <= 256), else exact */
+#define LIPCACHE_PROBE_AUTO 0          /* tensor path when supported (d <= 256) and B N d_pad >= 2^24, else exact */
 #define LIPCACHE_PROBE_TENSOR 1        /* tcgen05 TF32 screen, then exact FP32 recheck of candidates;
                                           the kernel is chosen by shape: TENSOR_SINGLE for
                                           d_pad <= 128, TENSOR_PAIR above (when clusters of four fit) */

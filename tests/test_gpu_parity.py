@@ -391,3 +391,24 @@ def test_large_dim_exact_path(dev):
     gi, gl, gd = run_probe(cache, Q, dev, 64, "exact")
     check_probe(gi, gl, gd, ref, Q, oracle.probe(ref["keys"], ref["radius"], ref["label"], Q))
     cache.close()
+
+
+def test_auto_path_choice(dev):
+    """"auto" takes the exact kernel below 2^24 multiply-adds per batch (its
+    fixed cost is smaller) and the tensor kernel above; both give the same
+    bits."""
+    for name, N, B, expect in [("tiny", 1024, 256, 2), ("cifar10", 5000, 256, 3)]:
+        w = synth.WORKLOADS[name].scaled(N=N, n_queries=B)
+        W, b = synth.head(w)
+        rows = synth.cache_rows(w)
+        Q, _ = synth.queries(w, rows)
+        cache, _ = make_cache(dev, W, b, N)
+        cache.insert(T(rows, dev))
+        cache.set_probe_path("auto")
+        a = [t.cpu().numpy() for t in cache.probe(T(Q, dev))]
+        assert cache.info()["last_probe_path"] == expect, name
+        cache.set_probe_path("tensor" if expect == 2 else "exact")
+        c = [t.cpu().numpy() for t in cache.probe(T(Q, dev))]
+        for x, y in zip(a, c):
+            assert np.array_equal(x.view(np.uint8), y.view(np.uint8))
+        cache.close()
