@@ -1028,8 +1028,6 @@ template <int NCG>
 __global__ void __launch_bounds__(kThreads, 1) k_certify_wt(CertArgs a, WtLayout L, const float* __restrict__ prep,
                                                              int64_t nb32) {
   extern __shared__ __align__(16) unsigned char smem[];
-  constexpr int NPR = NCG / 2;  // class pairs per thread
-  constexpr bool kOdd = (NCG & 1) != 0;
   const int d = a.d, C = a.C, GS = L.GS, wst = L.wst;
   float* wT = reinterpret_cast<float*>(smem);
   float* hT = reinterpret_cast<float*>(smem + L.off_h);  // d x kWtHst
