@@ -138,3 +138,43 @@ def test_kernel_choice(dev):
         c.insert(T(rng.standard_normal((100, d)).astype(np.float32), dev))
         assert c.info()["last_insert_kernel"] == kernel, (d, C, mode)
         c.close()
+
+
+def _near_ties(W, b, n, rng, k):
+    """Rows whose top k logits agree to about 1e-6 relative: random points
+    moved onto the set where classes a_1..a_k tie (least-squares step in the
+    span of W_{a_i} - W_{a_1}), then perturbed slightly."""
+    d = W.shape[1]
+    W64, b64 = W.astype(np.float64), b.astype(np.float64)
+    out = []
+    for _ in range(n):
+        z = rng.standard_normal(d) * 2.0
+        s = W64 @ z + b64
+        top = np.argsort(-s)[:k]
+        D = W64[top[1:]] - W64[top[0]]              # (k-1) x d
+        g = -(s[top[1:]] - s[top[0]])               # logit differences to cancel
+        z = z + D.T @ np.linalg.lstsq(D @ D.T, g, rcond=None)[0]
+        z = z + rng.standard_normal(d) * 1e-5 * np.linalg.norm(z) / np.sqrt(d)
+        out.append(z)
+    return np.asarray(out, dtype=np.float32)
+
+
+@pytest.mark.parametrize("d,C", [(16, 10), (64, 40), (128, 100), (128, 200), (96, 250)])
+def test_wide_tile_near_ties(dev, d, C):
+    """Rows on two- and three-way logit ties: several candidate classes per
+    row, refinement deciding the order, margins near zero (some rows
+    rejected). Bit-identical to the 64-row-tile kernel and within the
+    refinement bound of the oracle."""
+    rng = np.random.default_rng(d * 1000 + C)
+    W = (rng.standard_normal((C, d)) / np.sqrt(d)).astype(np.float32)
+    b = (0.1 * rng.standard_normal(C)).astype(np.float32)
+    rows = np.concatenate([_near_ties(W, b, 600, rng, 2), _near_ties(W, b, 600, rng, 3),
+                           rng.standard_normal((400, d)).astype(np.float32)])
+    a, ia, ra, na = build(dev, W, b, rows, len(rows), False)
+    s, is_, rs, ns = build(dev, W, b, rows, len(rows), True)
+    assert a.info()["last_insert_kernel"] == WIDE_TILE
+    assert na == ns and same_bits(ia, is_) and same_bits(ra, rs)
+    ref = oracle.build_cache(W, b, oracle.sigma_max(W), rows)
+    check_insert(ia, ra, na, ref, (W, b, rows, 1.0))
+    a.close()
+    s.close()
