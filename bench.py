@@ -262,25 +262,37 @@ def run_ours(args, dist: Dist):
     W, b, rows, Q = workload_data(w)
     stream = torch.cuda.current_stream(dev)
 
-    cache = LipCache(w.d, w.C, w.N, device=dev)
-    sigma = cache.set_head(torch.from_numpy(W).to(dev), torch.from_numpy(b).to(dev))
-    # certified insertion (Algorithm 1), timed separately
     rows_d = torch.from_numpy(rows).to(dev)
-    torch.cuda.synchronize(dev)
-    cache.enable_timing(True)  # CUDA events around each certify kernel, inside the library
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    n_acc = 0
-    for s, e in synth.batches(w.N, w.insert_batch):
-        n_acc += cache.insert(rows_d[s:e])[2]
-    e1.record(stream)
-    torch.cuda.synchronize(dev)
-    insert_ms = e0.elapsed_time(e1)
-    ins_info = cache.info()
-    cache.enable_timing(False)
-    insert_kernel = (INSERT_KERNELS.get(ins_info["last_insert_kernel"], "?"), ins_info["insert_kernel_ms_total"],
-                     ins_info["insert_kernel_launches"])
+
+    def build(mode):
+        """Certified insertion (Algorithm 1) of every row, timed separately:
+        CUDA events around the insert calls, and the library's events around
+        each certify kernel."""
+        c = LipCache(w.d, w.C, w.N, mode, device=dev)
+        sig = c.set_head(torch.from_numpy(W).to(dev), torch.from_numpy(b).to(dev))
+        torch.cuda.synchronize(dev)
+        c.enable_timing(True)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        acc = 0
+        for s, e in synth.batches(w.N, w.insert_batch):
+            acc += c.insert(rows_d[s:e])[2]
+        e1.record(stream)
+        torch.cuda.synchronize(dev)
+        inf = c.info()
+        c.enable_timing(False)
+        kern = (INSERT_KERNELS.get(inf["last_insert_kernel"], "?"), inf["insert_kernel_ms_total"],
+                inf["insert_kernel_launches"])
+        return c, sig, acc, e0.elapsed_time(e1), kern
+
+    # the tight radius (Eq. 29, Sec. 5.6) on the same rows, then the
+    # conservative radius (Eq. 21) whose cache the probe uses
+    tcache, _, n_acc_t, insert_ms_t, insert_kernel_t = build("tight")
+    tcache.close()
+    del tcache
+    cache, sigma, n_acc, insert_ms, insert_kernel = build("conservative")
     del rows_d
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     cache.set_probe_path(args.path)
     cache.reserve(w.batch)
     N = cache.size
@@ -360,6 +372,9 @@ def run_ours(args, dist: Dist):
         "clocks": clocks,
         "insert": insert_summary(w, n_acc, insert_ms, torch.cuda.get_device_properties(dev).multi_processor_count,
                                  clocks, kernel=insert_kernel),
+        "insert_tight": insert_summary(w, n_acc_t, insert_ms_t,
+                                       torch.cuda.get_device_properties(dev).multi_processor_count, clocks,
+                                       kernel=insert_kernel_t),
         "stats": {"sigma": sigma, "hit_rate": hit_rate,
                   "candidates_per_query": info["candidates"] / max(1, args.steps * B),
                   "device_errors": info["device_errors"], "kernel_ms": kernel_ms,

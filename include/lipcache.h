@@ -59,10 +59,12 @@ typedef enum lipcache_status {
 #define LIPCACHE_RADIUS_TIGHT 1        /* r* = min_j (s_y - s_j) / ||W_y - W_j||, Eq. 29 */
 
 /* Certify kernels (lipcache_info.last_insert_kernel). WIDE_TILE: head resident
- * in shared memory, 128-row tiles, logits in registers (conservative radius,
- * d % 4 == 0, head small enough). TILE64: head resident, 64-row tiles, logits
- * in shared memory (also the tight radius). STREAMED: head read from L2
- * (large heads). All three compute the same values. */
+ * in shared memory, 128-row tiles, logits in registers (d % 4 == 0, head small
+ * enough; both radii, the tight one refining only the classes that can be its
+ * minimiser). TILE64: head resident, 64-row tiles, logits in shared memory.
+ * STREAMED: head read from L2 (large heads). For the conservative radius all
+ * three compute the same values; for the tight radius the last two refine
+ * every class in FP64 and agree with WIDE_TILE within the refinement bound. */
 #define LIPCACHE_INSERT_WIDE_TILE 1
 #define LIPCACHE_INSERT_TILE64 2
 #define LIPCACHE_INSERT_STREAMED 3

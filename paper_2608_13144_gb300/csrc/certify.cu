@@ -60,6 +60,8 @@ struct CertArgs {
   ThreshConsts tc;       // constants of the probe thresholds
   const int64_t* miss_of;      // nullable: row accepted only if miss_of[row] < 0 (write-back)
   const double* inv_pairnorm;  // 1 / ||W_y - W_j|| (tight mode)
+  const float* ipn_up32;       // FP32 brackets of 1 / ||W_y - W_j|| (tight mode; +inf where the rows coincide)
+  const float* ipn_dn32;
   double tight_f;              // 1 - gamma_{d+8} (FP64)
   uint8_t* accept;
   int32_t* yG;
@@ -849,6 +851,7 @@ struct WtTile {
   float knp[4][kWtRows];  // quarter sums of ||z||^2
   float hn[kWtRows];      // upper bound of ||z||
   int ncand[kWtRows];
+  int yq[kWtRows];        // tight radius: y^G of the row, known from the FP32 intervals
   uint8_t cls[kWtRows][kMaxCand];
   float rh[kWtRows][kMaxCand], rl[kWtRows][kMaxCand], re[kWtRows][kMaxCand];
   int pairs[kWtRows * kMaxCand];  // r | slot << 8 | class << 16; after the refinement, per-warp logit rows
@@ -861,6 +864,231 @@ struct WtLayout {
   int NCG, GS, wst;
   uint32_t off_h, off_e, off_tile, total;
 };
+
+// E_c of an FP32 logit s~_c, rounded up, from the per-column terms
+// eA = g32f ||W_c|| and eB = g32f |b_c| + tiny (both rounded up) and the
+// bound hn of ||z||: gamma_{d+2} (||W_c|| ||z|| + |b_c|) + 2^-22 |s~_c| + tiny.
+__device__ __forceinline__ float logit_bound(float eA, float eB, float hn, float sv) {
+  return __fmaf_ru(eA, hn, __fmaf_ru(fabsf(sv), 2.3841858e-07f /* 2^-22 */, eB));
+}
+
+// Tight radius (Eq. 29) candidates of one row from the FP32 logit intervals
+// of this lane's classes (the 16 lanes of a half-warp hold the row). y^G is
+// certain when exactly one class's upper end reaches the largest lower end l1
+// (then every other interval lies below y's). For each other class j, u_j and
+// l_j bracket (s_y - s_j) / ||W_y - W_j|| (outward rounding, FP32 brackets of
+// the reciprocal norm); with U = min_j u_j, the minimiser of Eq. 29 is among
+// {j : l_j <= U}, since its l_j <= r* <= U. Returns this lane's candidate bits
+// (y and those classes) for refinement; `fallback` marks rows the intervals
+// cannot settle (several possible y^G, or a NaN logit), `y` the certain y^G.
+template <int NCG>
+__device__ __forceinline__ unsigned tight_candidates(const CertArgs& a, const float (&sv)[NCG], const float* eA,
+                                                     const float* eB, float hn, float l1, int cg, int lane,
+                                                     bool live_row, int& y, bool& fallback) {
+  const int C = a.C;
+  const unsigned half = 0xffffu << (lane & 16);
+  unsigned t1 = 0;
+  bool nan_l = false;
+  int myjc = -1;
+  float mlo = 0.f, mhi = 0.f;
+#pragma unroll
+  for (int jc = 0; jc < NCG; ++jc) {
+    const bool live = cg * NCG + jc < C;
+    const float E = logit_bound(eA[jc], eB[jc], hn, sv[jc]);
+    const float hi = __fadd_ru(sv[jc], E), lo = __fsub_rd(sv[jc], E);
+    nan_l |= live && !(sv[jc] == sv[jc]);
+    const bool top = live && hi >= l1;
+    const bool first = top && myjc < 0;
+    myjc = first ? jc : myjc;
+    mlo = first ? lo : mlo;
+    mhi = first ? hi : mhi;
+    t1 |= (unsigned)top << jc;
+  }
+  int cnt = __popc(t1);
+#pragma unroll
+  for (int o = 1; o < 16; o <<= 1) cnt += __shfl_xor_sync(kFull, cnt, o);
+  const unsigned nanb = __ballot_sync(kFull, nan_l) & half;
+  const unsigned hasb = __ballot_sync(kFull, t1 != 0u) & half;
+  const int src = hasb ? __ffs((int)hasb) - 1 : lane;
+  const int jy = __shfl_sync(kFull, myjc, src);
+  const float loy = __shfl_sync(kFull, mlo, src), hiy = __shfl_sync(kFull, mhi, src);
+  const bool certain = live_row && cnt == 1 && nanb == 0u;
+  const int yc = (src & 15) * NCG + jy;
+  float ub = INFINITY;
+#pragma unroll
+  for (int jc = 0; jc < NCG; ++jc) {
+    const int j = cg * NCG + jc;
+    const bool live = certain && j < C && j != yc;
+    const float iu = live ? __ldg(a.ipn_up32 + (size_t)yc * C + j) : INFINITY;
+    const float uj = __fmul_ru(__fsub_ru(hiy, __fsub_rd(sv[jc], logit_bound(eA[jc], eB[jc], hn, sv[jc]))), iu);
+    ub = fminf(ub, live ? uj : INFINITY);
+  }
+#pragma unroll
+  for (int o = 1; o < 16; o <<= 1) ub = fminf(ub, __shfl_xor_sync(kFull, ub, o));
+  unsigned c = 0;
+#pragma unroll
+  for (int jc = 0; jc < NCG; ++jc) {
+    const int j = cg * NCG + jc;
+    const bool live = certain && j < C && j != yc;
+    const float il = live ? __ldg(a.ipn_dn32 + (size_t)yc * C + j) : INFINITY;
+    const float lj = __fmul_rd(__fsub_rd(loy, __fadd_ru(sv[jc], logit_bound(eA[jc], eB[jc], hn, sv[jc]))), il);
+    c |= (unsigned)(certain && j < C && (j == yc || lj <= ub)) << jc;
+  }
+  y = certain ? yc : -1;
+  fallback = live_row && !certain;
+  return c;
+}
+
+// FP64 tight radius (Eq. 29) of one row from its refined candidates (y^G and
+// every class that can be the minimiser), with the certified lower bound and
+// the probe thresholds; the skip rules of Algorithm 1.
+__device__ void row_finals_tight(const CertArgs& a, int64_t row, int y, int n, const uint8_t* cls, const float* rh,
+                                 const float* rl, const float* re, float kn, uint8_t* acc_slot) {
+  const int C = a.C;
+  double vy = NAN, ey = 0.0;
+  for (int sl = 0; sl < n; ++sl)
+    if (cls[sl] == y) {
+      vy = (double)rh[sl] + (double)rl[sl];
+      ey = (double)re[sl];
+    }
+  double rmin = INFINITY, smin = INFINITY;
+  bool any_nan = !(vy == vy);
+  for (int sl = 0; sl < n; ++sl) {
+    const int j = cls[sl];
+    if (j == y) continue;
+    const double vj = (double)rh[sl] + (double)rl[sl], ej = (double)re[sl];
+    if (!(vj == vj)) any_nan = true;
+    const double pn = a.pairnorm[(size_t)y * C + j];
+    if (!(pn > 0.0)) continue;
+    const double ipn = a.inv_pairnorm[(size_t)y * C + j];
+    rmin = fmin(rmin, (vy - vj) * ipn);
+    const double num = __dsub_rd(__dsub_rd(vy, ey), __dadd_ru(vj, ej));
+    smin = fmin(smin, __dmul_rd(__dmul_rd(num, ipn), a.tight_f));
+  }
+  const double r64 = any_nan ? NAN : a.kappa * rmin;
+  const double rs = (smin > 0.0 && !any_nan) ? __dmul_rd(a.kappa, smin) : 0.0;
+  const int32_t lab = a.payload ? a.payload[row] : y;
+  const bool acc = !(a.require_consistency && lab != y) && (r64 > 0.0) && !(a.miss_of && a.miss_of[row] >= 0);
+  float rr, tau;
+  thresholds(__double2float_rd(rs), kn, a.tc, rr, tau);
+  a.accept[row] = acc ? 1 : 0;
+  a.yG[row] = y;
+  a.label[row] = lab;
+  a.radius[row] = __double2float_rz(r64);
+  a.rr[row] = rr;
+  a.kn[row] = kn;
+  a.tau[row] = tau;
+  *acc_slot = acc ? 1 : 0;
+}
+
+// One row of the tight radius on one warp, for rows the FP32 intervals cannot
+// settle (several classes may be y^G, a NaN logit, or more candidates than
+// slots): every class refined with the compensated dot product (lane = class,
+// features in order; the same error bound as the 8-lane refinement), y^G the
+// largest refined logit (lowest class on ties), then Eq. 29 over every other
+// class in FP64, as row_finals_tight. FP64 stays out of the per-feature work,
+// which runs at a small fraction of the FP32 rate on this GPU.
+template <int NCG>
+__device__ void wt_tight_row_warp(const CertArgs& a, int64_t row, int r, const float* __restrict__ wT, int wst,
+                                  int GS, const float* __restrict__ hT, const float* __restrict__ wn_s,
+                                  const float* __restrict__ b_s, float kn, int lane, uint8_t* acc_slot) {
+  constexpr int kPer = 8;  // classes per lane (C <= 256)
+  const int d = a.d, C = a.C;
+  const float hn = norm_upper(kn);
+  float vh[kPer], vl[kPer], ve[kPer];
+  float bh = -INFINITY, bl = 0.f;
+  int by = -1;
+  bool nan_any = false;
+#pragma unroll
+  for (int t = 0; t < kPer; ++t) {
+    const int c = lane + 32 * t;
+    vh[t] = NAN;
+    vl[t] = 0.f;
+    ve[t] = 0.f;
+    if (c < C) {
+      const int col = (c / NCG) * GS + (c % NCG);
+      float p = 0.f, cc = 0.f;
+      for (int k = 0; k < d; ++k) {
+        const float w = wT[(size_t)k * wst + col], x = hT[(size_t)k * kWtHst + r];
+        const float pr = __fmul_rn(w, x);
+        const float er = __fmaf_rn(w, x, -pr);
+        float s1, q;
+        two_sum(p, pr, s1, q);
+        p = s1;
+        cc = __fadd_rn(cc, __fadd_rn(q, er));
+      }
+      float s1, q, hi, lo;
+      two_sum(p, b_s[c], s1, q);
+      two_sum(s1, __fadd_rn(cc, q), hi, lo);
+      vh[t] = hi;
+      vl[t] = lo;
+      ve[t] = refined_err(a.g2f, wn_s[c], hn, b_s[c]);
+      nan_any |= !(hi == hi && lo == lo);
+      if (pair_gt(hi, lo, bh, bl)) {  // ascending classes: ties keep the lowest
+        bh = hi;
+        bl = lo;
+        by = c;
+      }
+    }
+  }
+  // warp argmax, ties to the lowest class (a total order on non-NaN pairs)
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float oh = __shfl_xor_sync(kFull, bh, o), ol = __shfl_xor_sync(kFull, bl, o);
+    const int oy = __shfl_xor_sync(kFull, by, o);
+    const bool eq = oh == bh && ol == bl;
+    if (oy >= 0 && (by < 0 || pair_gt(oh, ol, bh, bl) || (eq && oy < by))) {
+      bh = oh;
+      bl = ol;
+      by = oy;
+    }
+  }
+  nan_any = __any_sync(kFull, nan_any);
+  const int y = by < 0 ? 0 : by;
+  float myh = 0.f, myl = 0.f, mye = 0.f;
+#pragma unroll
+  for (int t = 0; t < kPer; ++t)
+    if (lane + 32 * t == y) {
+      myh = vh[t];
+      myl = vl[t];
+      mye = ve[t];
+    }
+  const int owner = y & 31;
+  const double vy = (double)__shfl_sync(kFull, myh, owner) + (double)__shfl_sync(kFull, myl, owner);
+  const double ey = (double)__shfl_sync(kFull, mye, owner);
+  double rmin = INFINITY, smin = INFINITY;
+#pragma unroll
+  for (int t = 0; t < kPer; ++t) {
+    const int j = lane + 32 * t;
+    if (j >= C || j == y) continue;
+    const double pn = a.pairnorm[(size_t)y * C + j];
+    if (!(pn > 0.0)) continue;
+    const double ipn = a.inv_pairnorm[(size_t)y * C + j];
+    const double vj = (double)vh[t] + (double)vl[t], ej = (double)ve[t];
+    rmin = fmin(rmin, (vy - vj) * ipn);
+    const double num = __dsub_rd(__dsub_rd(vy, ey), __dadd_ru(vj, ej));
+    smin = fmin(smin, __dmul_rd(__dmul_rd(num, ipn), a.tight_f));
+  }
+  rmin = warp_min_d(rmin);
+  smin = warp_min_d(smin);
+  if (lane == 0) {
+    const double r64 = nan_any ? NAN : a.kappa * rmin;
+    const double rs = (smin > 0.0 && !nan_any) ? __dmul_rd(a.kappa, smin) : 0.0;
+    const int32_t lab = a.payload ? a.payload[row] : y;
+    const bool acc = !(a.require_consistency && lab != y) && (r64 > 0.0) && !(a.miss_of && a.miss_of[row] >= 0);
+    float rr, tau;
+    thresholds(__double2float_rd(rs), kn, a.tc, rr, tau);
+    a.accept[row] = acc ? 1 : 0;
+    a.yG[row] = y;
+    a.label[row] = lab;
+    a.radius[row] = __double2float_rz(r64);
+    a.rr[row] = rr;
+    a.kn[row] = kn;
+    a.tau[row] = tau;
+    *acc_slot = acc ? 1 : 0;
+  }
+  __syncwarp();
+}
 
 // Steps 2-3 of k_certify_wt for one chunk, with ROWS rows per thread (8 for
 // chunks of more than 64 rows, 4 otherwise, so that a short chunk still keeps
@@ -922,7 +1150,7 @@ __device__ __forceinline__ void wt_chunk_logits(const CertArgs& a, const float* 
     // -inf lower ends and no candidacy.
 #pragma unroll 1
     for (int i = 0; i < ROWS; i += 2) {
-      float sv[2][NCG], E[2][NCG], l1[2], l2[2], hn[2];
+      float sv[2][NCG], l1[2], l2[2], hn[2];
       int r[2];
 #pragma unroll
       for (int u = 0; u < 2; ++u) {
@@ -948,8 +1176,8 @@ __device__ __forceinline__ void wt_chunk_logits(const CertArgs& a, const float* 
         l2[u] = -INFINITY;
 #pragma unroll
         for (int jc = 0; jc < NCG; ++jc) {
-          E[u][jc] = __fmaf_ru(eA[cg * GS + jc], hn[u], __fmaf_ru(fabsf(sv[u][jc]), 2.3841858e-07f, eB[cg * GS + jc]));
-          float lo = __fsub_rd(sv[u][jc], E[u][jc]);
+          const float E = logit_bound(eA[cg * GS + jc], eB[cg * GS + jc], hn[u], sv[u][jc]);
+          float lo = __fsub_rd(sv[u][jc], E);
           lo = (lo == lo && cg * NCG + jc < C) ? lo : -INFINITY;
           l2[u] = fmaxf(l2[u], fminf(l1[u], lo));
           l1[u] = fmaxf(l1[u], lo);
@@ -967,13 +1195,24 @@ __device__ __forceinline__ void wt_chunk_logits(const CertArgs& a, const float* 
         }
       }
       unsigned cm[2];  // candidate bits of this lane's classes
-      int incl[2], mine[2];
+      int incl[2], mine[2], yv[2];
+      bool fallback[2];
 #pragma unroll
       for (int u = 0; u < 2; ++u) {
         cm[u] = 0;
+        yv[u] = -1;
+        fallback[u] = false;
+        if (!a.tight) {
 #pragma unroll
-        for (int jc = 0; jc < NCG; ++jc)
-          cm[u] |= (unsigned)(cg * NCG + jc < C && __fadd_ru(sv[u][jc], E[u][jc]) >= l2[u]) << jc;
+          for (int jc = 0; jc < NCG; ++jc)
+            cm[u] |= (unsigned)(cg * NCG + jc < C &&
+                                __fadd_ru(sv[u][jc], logit_bound(eA[cg * GS + jc], eB[cg * GS + jc], hn[u], sv[u][jc])) >=
+                                    l2[u])
+                     << jc;
+        } else {
+          cm[u] = tight_candidates<NCG>(a, sv[u], eA + cg * GS, eB + cg * GS, hn[u], l1[u], cg, lane, r[u] < nrows,
+                                        yv[u], fallback[u]);
+        }
         cm[u] = r[u] < nrows ? cm[u] : 0u;
         mine[u] = __popc(cm[u]);
         incl[u] = mine[u];
@@ -999,8 +1238,9 @@ __device__ __forceinline__ void wt_chunk_logits(const CertArgs& a, const float* 
           ++slot;
         }
         if (cg == 15) {
-          ts.ncand[r[u]] = incl[u];
+          ts.ncand[r[u]] = fallback[u] ? kMaxCand + 1 : incl[u];
           ts.hn[r[u]] = hn[u];
+          ts.yq[r[u]] = yv[u];
         }
       }
     }
@@ -1193,17 +1433,28 @@ __global__ void __launch_bounds__(kThreads, 1) k_certify_wt(CertArgs a, WtLayout
         ts.ovf[atomicAdd(&ts.novf, 1)] = r;
       } else {
         const float kn = (ts.knp[0][r] + ts.knp[1][r]) + (ts.knp[2][r] + ts.knp[3][r]);
-        Top2 t;
-        for (int sl = 0; sl < n; ++sl) t.push(ts.cls[r][sl], ts.rh[r][sl], ts.rl[r][sl], ts.re[r][sl]);
-        row_finals(a, row0 + r, t.result(kn), &ts.acc_flag[r]);
+        if (a.tight) {
+          row_finals_tight(a, row0 + r, ts.yq[r], n, ts.cls[r], ts.rh[r], ts.rl[r], ts.re[r], kn, &ts.acc_flag[r]);
+        } else {
+          Top2 t;
+          for (int sl = 0; sl < n; ++sl) t.push(ts.cls[r][sl], ts.rh[r][sl], ts.rl[r][sl], ts.re[r][sl]);
+          row_finals(a, row0 + r, t.result(kn), &ts.acc_flag[r]);
+        }
       }
     }
     __syncthreads();
     // rows with more than kMaxCand candidates: FP32 logits again (the same
     // FMA chains, into this warp's share of the dead pair list), then the
     // one-warp refinement
+    // (tight radius: the rows the intervals could not settle, all classes
+    // refined on one warp by wt_tight_row_warp)
     for (int i = warp; i < ts.novf; i += kWarps) {
       const int r = ts.ovf[i];
+      if (a.tight) {
+        const float kn = (ts.knp[0][r] + ts.knp[1][r]) + (ts.knp[2][r] + ts.knp[3][r]);
+        wt_tight_row_warp<NCG>(a, row0 + r, r, wT, wst, GS, hT, wn_s, b_s, kn, lane, &ts.acc_flag[r]);
+        continue;
+      }
       float* lrow = reinterpret_cast<float*>(ts.pairs) + (size_t)warp * C;
       for (int c = lane; c < C; c += 32) {
         const int col = (c / NCG) * GS + (c % NCG);
@@ -1489,6 +1740,8 @@ void launch_certify(lipcache* h, const float* H, int64_t n, const int32_t* paylo
   a.tc = thresh_consts(h->dpad);
   a.miss_of = miss_of;
   a.inv_pairnorm = h->inv_pairnorm;
+  a.ipn_up32 = h->ipn_up32;
+  a.ipn_dn32 = h->ipn_dn32;
   a.tight_f = 1.0 - gamma64(h->d + 8);
   a.inv_denom = h->radius_scale / (h->sigma * 1.4142135623730951);
   a.inv_denom_safe = h->radius_scale * (1.0 - 8 * kU64) / (h->sigma * (1.0 + kSigmaSlack) * 1.4142135623730951);
@@ -1510,7 +1763,8 @@ void launch_certify(lipcache* h, const float* H, int64_t n, const int32_t* paylo
   const int ncg = wt_ncg(h->C);
   const bool vec16 = h->d % 4 == 0 && ((uintptr_t)H & 15) == 0;
   const WtLayout L = wt_layout(h->d, h->C, ncg > 0 ? ncg : 1);
-  if (!a.tight && vec16 && ncg > 0 && L.total <= 227 * 1024 && !(h->debug_flags & LIPCACHE_DEBUG_INSERT_TILE64)) {
+  if ((!a.tight || h->ipn_up32) && vec16 && ncg > 0 && L.total <= 227 * 1024 &&
+      !(h->debug_flags & LIPCACHE_DEBUG_INSERT_TILE64)) {
     const int64_t nb32 = (n + 31) / 32;
     const int grid = nb32 < h->num_sms ? (int)nb32 : h->num_sms;
     if (h->wt_prep_ncg != ncg) {

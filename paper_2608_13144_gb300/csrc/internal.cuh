@@ -179,6 +179,8 @@ struct lipcache {
   float* Wnorm32 = nullptr;  // C, ||W_c|| rounded up to FP32
   double* pairnorm = nullptr;  // C x C (tight mode)
   double* inv_pairnorm = nullptr;  // C x C: 1 / pairnorm (0 where pairnorm is 0)
+  float* ipn_up32 = nullptr;       // C x C: FP32 upper bound of 1 / ||W_y - W_j|| (+inf where it is 0)
+  float* ipn_dn32 = nullptr;       // C x C: FP32 lower bound (+inf where ||W_y - W_j|| is 0)
   double* gram[2] = {nullptr, nullptr};  // d x d FP64
   lc::SpecResult* spec = nullptr;        // device
   lc::SpecResult* spec_host = nullptr;   // pinned

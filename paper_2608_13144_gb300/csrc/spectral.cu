@@ -174,10 +174,14 @@ __global__ void __launch_bounds__(kPowerThreads) k_power(const float* __restrict
 }
 
 // ||W_c|| for every class and, for the tight radius, ||W_y - W_j|| for every
-// pair (FP64).
+// pair (FP64; the differences of FP32 weights are exact, the sum of d squares
+// is within gamma_d of the exact one) with its reciprocal, and FP32 brackets
+// of the reciprocal (the FP64 value widened by 1e-12, far above its error,
+// then rounded outward; +inf for coinciding rows, which the tight radius skips).
 __global__ void k_row_norms(const float* __restrict__ W, int C, int d, double* __restrict__ Wnorm,
                             float* __restrict__ Wnorm32, double* __restrict__ pairnorm,
-                            double* __restrict__ inv_pairnorm) {
+                            double* __restrict__ inv_pairnorm, float* __restrict__ ipn_up32,
+                            float* __restrict__ ipn_dn32) {
   const int y = blockIdx.y;
   const int j = blockIdx.x * blockDim.x + threadIdx.x;
   if (j >= C) return;
@@ -188,7 +192,10 @@ __global__ void k_row_norms(const float* __restrict__ W, int C, int d, double* _
       acc = fma(e, e, acc);
     }
     pairnorm[(size_t)y * C + j] = sqrt(acc);
-    inv_pairnorm[(size_t)y * C + j] = acc > 0.0 ? 1.0 / sqrt(acc) : 0.0;
+    const double ipn = acc > 0.0 ? 1.0 / sqrt(acc) : 0.0;
+    inv_pairnorm[(size_t)y * C + j] = ipn;
+    ipn_up32[(size_t)y * C + j] = acc > 0.0 ? __double2float_ru(ipn * (1.0 + 1e-12)) : INFINITY;
+    ipn_dn32[(size_t)y * C + j] = acc > 0.0 ? __double2float_rd(ipn * (1.0 - 1e-12)) : INFINITY;
   }
   if (j == y) {
     double n2 = 0.0;
@@ -221,7 +228,8 @@ void spectral_norm(lipcache* h, cudaStream_t s) {
   dim3 rb(128), rg((C + 127) / 128, C);
   const bool tight = h->radius_mode == LIPCACHE_RADIUS_TIGHT;
   k_row_norms<<<rg, rb, 0, s>>>(h->W, C, d, h->Wnorm, h->Wnorm32, tight ? h->pairnorm : nullptr,
-                                tight ? h->inv_pairnorm : nullptr);
+                                tight ? h->inv_pairnorm : nullptr, tight ? h->ipn_up32 : nullptr,
+                                tight ? h->ipn_dn32 : nullptr);
   LC_LAUNCH_CHECK("k_row_norms");
 }
 

@@ -28,11 +28,28 @@ def refine_slack(W, b, rows, kappa=1.0):
     return kappa * 4 * g * g * scale / (oracle.sigma_max(W) * np.sqrt(2.0)) * (1 + 1e-6)
 
 
+def refine_slack_tight(W, b, rows, kappa=1.0):
+    """The same for the tight radius (Eq. 29) computed from compensated FP32
+    refinements: r* = kappa (s_y - s_j) / ||W_y - W_j|| with both logits
+    within 2 gamma_{d+40}^2 (||W_c|| ||z|| + |b_c|) of the exact ones."""
+    W64 = np.asarray(W, np.float64)
+    d = W64.shape[1]
+    u = 2.0 ** -24
+    g = (d + 40) * u / (1 - (d + 40) * u)
+    scale = np.linalg.norm(W64, axis=1).max() * np.linalg.norm(np.asarray(rows, np.float64), axis=1)
+    scale += np.abs(np.asarray(b, np.float64)).max()
+    pn = np.linalg.norm(W64[:, None, :] - W64[None, :, :], axis=2)
+    pmin = pn[pn > 0].min() if np.any(pn > 0) else 1.0
+    return kappa * 4 * g * g * scale / pmin * (1 + 1e-6)
+
+
 def check_insert(g_index, g_radius, n_acc, ref, head=None):
-    """head = (W, b, rows, kappa) for the conservative radius: the reported
-    radius (the refined margin's value, rounded toward zero) must then not
-    exceed the exact one by more than the refinement's error bound. Without
-    it (tight radius, FP64 refinement) the bound is 1e-12 relative."""
+    """head = (W, b, rows, kappa) for the conservative radius and
+    ("tight", W, b, rows, kappa) for the tight radius from compensated FP32
+    refinements: the reported radius (the refined value, rounded toward zero)
+    must then not exceed the exact one by more than the refinement's error
+    bound. Without it (tight radius, FP64 refinement of every class) the bound
+    is 1e-12 relative."""
     cert = ref["cert"]
     assert n_acc == int(cert["accept"].sum())
     bad = np.nonzero(g_index != ref["index"])[0]
@@ -40,7 +57,12 @@ def check_insert(g_index, g_radius, n_acc, ref, head=None):
     r = cert["radius"]
     m = np.isfinite(r) & (r > 0)
     np.testing.assert_allclose(g_radius[m], r[m], rtol=RTOL)
-    slack = r * 1e-12 if head is None else refine_slack(*head)
+    if head is None:
+        slack = r * 1e-12
+    elif isinstance(head[0], str) and head[0] == "tight":
+        slack = r * 1e-12 + refine_slack_tight(*head[1:])
+    else:
+        slack = refine_slack(*head)
     assert np.all(g_radius[m].astype(np.float64) <= r[m] + slack[m])
 
 

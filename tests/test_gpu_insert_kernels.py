@@ -7,7 +7,7 @@ import pytest
 
 import oracle
 import synth
-from parity_utils import check_insert
+from parity_utils import check_insert, refine_slack_tight
 
 torch = pytest.importorskip("torch")
 pytestmark = pytest.mark.gpu
@@ -124,10 +124,9 @@ def test_wide_tile_payload_and_consistency(dev):
 
 def test_kernel_choice(dev):
     """Shapes outside the wide-tile kernel's limits take the other
-    kernels: the tight radius, d % 4 != 0, and heads too large for shared
-    memory."""
+    kernels: d % 4 != 0, and heads too large for shared memory."""
     from paper_2608_13144_gb300.lipcache import LipCache
-    cases = [((64, 10), "tight", TILE64), ((33, 10), "conservative", TILE64),
+    cases = [((64, 10), "tight", WIDE_TILE), ((33, 10), "tight", TILE64), ((33, 10), "conservative", TILE64),
              ((256, 200), "conservative", STREAMED), ((128, 300), "conservative", STREAMED)]
     rng = np.random.default_rng(5)
     for (d, C), mode, kernel in cases:
@@ -178,3 +177,63 @@ def test_wide_tile_near_ties(dev, d, C):
     check_insert(ia, ra, na, ref, (W, b, rows, 1.0))
     a.close()
     s.close()
+
+
+def build_tight(dev, W, b, rows, tile64, kappa=1.0):
+    from paper_2608_13144_gb300.lipcache import LipCache
+    c = LipCache(W.shape[1], W.shape[0], len(rows), "tight", device=dev)
+    c.set_radius_scale(kappa)
+    c.set_head(T(W, dev), T(b, dev))
+    if tile64:
+        c.set_debug(DEBUG_INSERT_TILE64)
+    i, r, n = c.insert(T(rows, dev))
+    return c, i.cpu().numpy(), r.cpu().numpy(), n
+
+
+@pytest.mark.parametrize("d,C,kappa", [(16, 10, 1.0), (64, 40, 0.8), (128, 100, 1.0), (128, 200, 1.0),
+                                       (96, 250, 0.9)])
+def test_wide_tile_tight_radius(dev, d, C, kappa):
+    """Tight radius (Eq. 29) on the wide-tile kernel: y^G settled by the FP32
+    intervals, the minimiser among the classes whose bracket of
+    (s_y - s_j) / ||W_y - W_j|| can reach the smallest upper bracket, refined
+    with the compensated dot product; rows the intervals cannot settle (ties
+    among the top classes) on one warp. Against the oracle and the kernels
+    that refine every class in FP64 (64-row or streamed): the same acceptance
+    and y^G, radii within the refinement bound."""
+    rng = np.random.default_rng(d * 7 + C)
+    W = (rng.standard_normal((C, d)) / np.sqrt(d)).astype(np.float32)
+    b = (0.1 * rng.standard_normal(C)).astype(np.float32)
+    rows = np.concatenate([rng.standard_normal((3000, d)).astype(np.float32) * 2,
+                           _near_ties(W, b, 300, rng, 2), _near_ties(W, b, 300, rng, 3)])
+    a, ia, ra, na = build_tight(dev, W, b, rows, False, kappa)
+    assert a.info()["last_insert_kernel"] == WIDE_TILE
+    s, is_, rs, ns = build_tight(dev, W, b, rows, True, kappa)
+    assert s.info()["last_insert_kernel"] in (TILE64, STREAMED)  # FP64 refinement of every class
+    ref = oracle.build_cache(W, b, oracle.sigma_max(W), rows, radius_mode=oracle.RADIUS_TIGHT, scale=kappa)
+    check_insert(ia, ra, na, ref, ("tight", W, b, rows, kappa))
+    assert na == ns and np.array_equal(ia, is_)
+    np.testing.assert_array_equal(a.entries()["yG"], s.entries()["yG"])
+    m = np.isfinite(rs) & (rs > 0)
+    slack = refine_slack_tight(W, b, rows, kappa)  # each kernel's own refinement error
+    assert np.all(np.abs(ra[m].astype(np.float64) - rs[m]) <= 1e-6 * rs[m] + 2 * slack[m])
+    a.close()
+    s.close()
+
+
+def test_wide_tile_tight_tied_head_rows(dev):
+    """Identical head rows (||W_y - W_j|| = 0, skipped by Eq. 29) and rows won
+    by the tied group (several possible y^G: the FP64 row path)."""
+    rng = np.random.default_rng(21)
+    d, C = 32, 24
+    W = (rng.standard_normal((C, d)) / np.sqrt(d)).astype(np.float32)
+    W[1:20] = W[1]
+    b = (0.1 * rng.standard_normal(C)).astype(np.float32)
+    b[1:20] = b[1]
+    rows = np.concatenate([3 * W[0] + 0.3 * rng.standard_normal((700, d)),
+                           3 * W[1] + 0.3 * rng.standard_normal((700, d)),
+                           rng.standard_normal((600, d))]).astype(np.float32)
+    a, ia, ra, na = build_tight(dev, W, b, rows, False)
+    assert a.info()["last_insert_kernel"] == WIDE_TILE
+    ref = oracle.build_cache(W, b, oracle.sigma_max(W), rows, radius_mode=oracle.RADIUS_TIGHT)
+    check_insert(ia, ra, na, ref, ("tight", W, b, rows, 1.0))
+    a.close()

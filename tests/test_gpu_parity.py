@@ -240,7 +240,7 @@ def test_tensor_equals_exact(built, dev, name):
 @pytest.mark.parametrize("name", ["tiny", "cifar100"])
 def test_tight_radius_parity(built, dev, name):
     s = built(name, "tight")
-    check_insert(s["g_index"], s["g_radius"], s["n_acc"], s["ref"])
+    check_insert(s["g_index"], s["g_radius"], s["n_acc"], s["ref"], ("tight", s["W"], s["b"], s["rows"], 1.0))
     for path in PATHS:
         gi, gl, gd = run_probe(s["cache"], s["Q"], dev, s["w"].batch, path)
         check_probe(gi, gl, gd, s["ref"], s["Q"], s["orc"])
@@ -366,7 +366,8 @@ def test_many_tied_runners_up(dev, mode):
     ref = oracle.build_cache(W, b, oracle.sigma_max(W), rows, radius_mode=int(mode == "tight"))
     cache, _ = make_cache(dev, W, b, len(rows), mode)
     idx, rad, n = cache.insert(T(rows, dev))
-    check_insert(idx.cpu().numpy(), rad.cpu().numpy(), n, ref, None if mode == "tight" else (W, b, rows, 1.0))
+    check_insert(idx.cpu().numpy(), rad.cpu().numpy(), n, ref,
+                 ("tight", W, b, rows, 1.0) if mode == "tight" else (W, b, rows, 1.0))
     assert n > 100
     if mode == "conservative":
         assert n < len(rows)  # rows won by the tied group are skipped
