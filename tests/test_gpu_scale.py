@@ -96,3 +96,28 @@ def test_scale_tensor_equals_exact(scale):
         for x, y in zip(outs["exact"], outs[path]):
             assert np.array_equal(x.view(np.uint8) if x.dtype == np.float32 else x,
                                   y.view(np.uint8) if y.dtype == np.float32 else y), path
+
+
+def test_scale_tight_radius_rows(scale):
+    """The tight radius (Eq. 29) on 262,144 rows of the 4M-entry workload
+    (four 65,536-row launches, the benchmark's batch): acceptance and indices
+    bit-exact, radii within the compensated refinement's bound of the oracle's
+    FP64 tight radius."""
+    from paper_2608_13144_gb300.lipcache import LipCache
+    from parity_utils import check_insert
+    s = scale
+    w = s["w"]
+    rows = s["rows"][:262144]
+    c = LipCache(w.d, w.C, len(rows), "tight", device=s["dev"])
+    c.set_head(torch.from_numpy(s["W"]).to(s["dev"]), torch.from_numpy(s["b"]).to(s["dev"]))
+    rd = torch.from_numpy(rows).to(s["dev"])
+    idx, rad, n = [], [], 0
+    for a, e in synth.batches(len(rows), w.insert_batch):
+        i, r, k = c.insert(rd[a:e])
+        idx.append(i.cpu().numpy())
+        rad.append(r.cpu().numpy())
+        n += k
+    assert c.info()["last_insert_kernel"] == 1
+    ref = oracle.build_cache(s["W"], s["b"], oracle.sigma_max(s["W"]), rows, radius_mode=oracle.RADIUS_TIGHT)
+    check_insert(np.concatenate(idx), np.concatenate(rad), n, ref, ("tight", s["W"], s["b"], rows, 1.0))
+    c.close()
