@@ -237,3 +237,20 @@ def test_wide_tile_tight_tied_head_rows(dev):
     ref = oracle.build_cache(W, b, oracle.sigma_max(W), rows, radius_mode=oracle.RADIUS_TIGHT)
     check_insert(ia, ra, na, ref, ("tight", W, b, rows, 1.0))
     a.close()
+
+
+@pytest.mark.parametrize("d,C,kernel", [(33, 7, TILE64), (21, 40, TILE64), (256, 200, STREAMED), (128, 300, STREAMED)])
+def test_tight_radius_other_kernels(dev, d, C, kernel):
+    """The tight radius on the kernels that refine every class in FP64
+    (d % 4 != 0; heads too large for shared memory) against the oracle,
+    rows on logit ties included."""
+    rng = np.random.default_rng(d * 13 + C)
+    W = (rng.standard_normal((C, d)) / np.sqrt(d)).astype(np.float32)
+    b = (0.1 * rng.standard_normal(C)).astype(np.float32)
+    rows = np.concatenate([rng.standard_normal((800, d)).astype(np.float32) * 2,
+                           _near_ties(W, b, 100, rng, 2), _near_ties(W, b, 100, rng, 3)])
+    c, i, r, n = build_tight(dev, W, b, rows, False)
+    assert c.info()["last_insert_kernel"] == kernel
+    ref = oracle.build_cache(W, b, oracle.sigma_max(W), rows, radius_mode=oracle.RADIUS_TIGHT)
+    check_insert(i, r, n, ref)  # FP64 refinement of every class: within 1e-12 relative
+    c.close()
