@@ -18,8 +18,11 @@
 // |b_c|). The true top-1 and runner-up are always among them, so m is the
 // margin of the full logit vector to ~1e-10 relative of the logit scale.
 // FP64 runs at a small fraction of the FP32 rate on this GPU, so only the
-// per-row margin and radius use it. The tight radius needs every class and
-// refines all of them in FP64 (products of FP32 values are exact there).
+// per-row margin and radius use it. For the tight radius the wide-tile kernel
+// refines y^G and the classes whose FP32 bracket of (s_y - s_j) /
+// ||W_y - W_j|| can reach the smallest upper bracket (they contain the
+// minimiser); the other kernels refine every class in FP64 (products of FP32
+// values are exact there).
 //
 // Besides the reported radius r, the kernel derives a certified lower bound
 // r_safe of the exact radius (the refined logits' error bounds, sigma
@@ -27,10 +30,12 @@
 // acceptance threshold rr <= r_safe^2 (1 - eps_rc) on the canonical FP32
 // squared distance, and the screen term tau.
 //
-// Two kernels compute the FP32 logits: when C <= 256 and the head fits in
-// shared memory, persistent CTAs keep W^T resident and form a register-tiled
-// product (k_certify_wres); otherwise each CTA streams W from L2 (k_certify).
-// Insertion order is kept by a block-count scan and a scatter.
+// Three kernels compute the FP32 logits. When d % 4 == 0 and the head fits
+// in shared memory, persistent CTAs keep W^T resident and take 128-row chunks
+// with 8 x NCG register tiles and the interval pass in registers
+// (k_certify_wt, both radii); with d % 4 != 0, 64-row tiles with the logits in
+// shared memory (k_certify_wres); for larger heads each CTA streams W from L2
+// (k_certify). Insertion order is kept by a block-count scan and a scatter.
 #include "internal.cuh"
 #include "tc_ptx.cuh"
 
