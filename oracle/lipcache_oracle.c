@@ -146,6 +146,8 @@ void orc_logits(const float* W, const float* b, int C, int d, const float* z, do
  *   r    <- scale * r                            (radius tightening, Sec. 5.6)
  *   payload = caller's label if given, else the proxy label y^G (Sec. 3.3)
  *   skip if consistency is required and payload != y^G, else skip if r <= 0.
+ * A row with a NaN or infinite feature has no defined margin (Eq. 20) nor
+ * terms of Eq. 29: r = NaN, so it is skipped in either radius mode.
  * ------------------------------------------------------------------------ */
 void orc_certify(const float* W, const float* b, int C, int d, double sigma, int radius_mode, double scale,
                  const float* H, int64_t n, const int32_t* payload, int require_consistency, int32_t* yG_out,
@@ -182,6 +184,10 @@ void orc_certify(const float* W, const float* b, int C, int d, double sigma, int
           if (rij < r) r = rij;
         }
       }
+      int finite = 1;
+      for (int k = 0; k < d; ++k)
+        if (!isfinite(z[k])) finite = 0;
+      if (!finite) r = NAN;
       r *= scale;
       int32_t label = payload ? payload[i] : (int32_t)y;
       int accept;

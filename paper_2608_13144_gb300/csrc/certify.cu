@@ -446,6 +446,7 @@ __device__ void certify_row(const CertArgs& a, int64_t row, const float* __restr
       rmin = warp_min_d(rmin);
       smin = warp_min_d(smin);
       any_nan = __any_sync(kFull, any_nan);
+      any_nan |= !(hn < INFINITY);  // a NaN or infinite feature: no defined term of Eq. 29
       r64 = any_nan ? NAN : a.kappa * rmin;
       rs = (smin > 0.0 && !any_nan) ? __dmul_rd(a.kappa, smin) : 0.0;
     }
@@ -917,7 +918,9 @@ __device__ __forceinline__ unsigned tight_candidates(const CertArgs& a, const fl
   const int src = hasb ? __ffs((int)hasb) - 1 : lane;
   const int jy = __shfl_sync(kFull, myjc, src);
   const float loy = __shfl_sync(kFull, mlo, src), hiy = __shfl_sync(kFull, mhi, src);
-  const bool certain = live_row && cnt == 1 && nanb == 0u;
+  // (a row whose norm bound is not finite, from an infinite feature or an
+  // overflowing |z|^2, goes to the one-warp path, which settles both)
+  const bool certain = live_row && cnt == 1 && nanb == 0u && hn < INFINITY;
   const int yc = (src & 15) * NCG + jy;
   float ub = INFINITY;
 #pragma unroll

@@ -254,3 +254,46 @@ def test_tight_radius_other_kernels(dev, d, C, kernel):
     ref = oracle.build_cache(W, b, oracle.sigma_max(W), rows, radius_mode=oracle.RADIUS_TIGHT)
     check_insert(i, r, n, ref)  # FP64 refinement of every class: within 1e-12 relative
     c.close()
+
+
+@pytest.mark.parametrize("mode", ["conservative", "tight"])
+@pytest.mark.parametrize("d,C", [(16, 10), (128, 200)])
+def test_certify_special_values(dev, mode, d, C):
+    """Rows with NaN or infinite features are skipped (a NaN margin fails
+    r > 0); zero rows and rows of magnitude 1e-30 or 1e30 are certified like
+    any other. Acceptance and indices bit-exact with the oracle, radii within
+    the refinement bound. Probes of the accepted rows inside FP32's range hit
+    themselves; the 1e30 row (its |k|^2 overflows FP32, so it has no
+    threshold) is never hit, and the zero row ties at FP32 distance 0 with the
+    1e-30 row (their squared distance underflows), lowest index first."""
+    from paper_2608_13144_gb300.lipcache import LipCache
+    rng = np.random.default_rng(d + C)
+    W = (rng.standard_normal((C, d)) / np.sqrt(d)).astype(np.float32)
+    b = (0.1 * rng.standard_normal(C)).astype(np.float32)
+    base = rng.standard_normal((12, d)).astype(np.float32)
+    rows = [base[0], base[1] * 1e-30, base[2] * 1e30, np.zeros(d, np.float32), base[3], base[4]]
+    bad = base[5:11].copy()
+    bad[0, 3] = np.nan
+    bad[1, :] = np.nan
+    bad[2, 0] = np.inf
+    bad[3, 5] = -np.inf
+    rows = np.concatenate([np.stack(rows), bad, base[11:]]).astype(np.float32)
+    c = LipCache(d, C, len(rows), mode, device=dev)
+    c.set_head(T(W, dev), T(b, dev))
+    i, r, n = c.insert(T(rows, dev))
+    i, r = i.cpu().numpy(), r.cpu().numpy()
+    assert c.info()["last_insert_kernel"] == WIDE_TILE
+    ref = oracle.build_cache(W, b, oracle.sigma_max(W), rows, radius_mode=int(mode == "tight"))
+    head = ("tight", W, b, rows, 1.0) if mode == "tight" else (W, b, rows, 1.0)
+    finite = np.all(np.isfinite(rows), axis=1)
+    assert np.all(i[~finite] == -1)
+    check_insert(i, r, n, ref, head)
+    normal = [k for k in (0, 4, 5, 11) if i[k] >= 0]
+    hit, _, dist = c.probe(T(rows[normal], dev))
+    np.testing.assert_array_equal(hit.cpu().numpy(), i[normal])
+    assert np.all(dist.cpu().numpy() == 0)
+    if i[2] >= 0:
+        assert c.probe(T(rows[2:3], dev))[0].item() == -1
+    if i[1] >= 0 and i[3] >= 0:
+        assert c.probe(T(rows[3:4], dev))[0].item() == min(i[1], i[3])
+    c.close()

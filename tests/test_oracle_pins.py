@@ -279,3 +279,19 @@ def test_certify_logits_vs_matmul():
     z = rng.standard_normal(13).astype(np.float32)
     ref = W.astype(np.float64) @ z.astype(np.float64) + b
     np.testing.assert_allclose(oracle.logits(W, b, z), ref, rtol=1e-13, atol=1e-13)
+
+
+@pytest.mark.parametrize("mode", [oracle.RADIUS_CONSERVATIVE, oracle.RADIUS_TIGHT])
+def test_non_finite_rows_skipped(mode):
+    """A row with an infinite or NaN feature has no defined margin (Eq. 20)
+    nor terms of Eq. 29, so it is skipped in either mode. The first row makes
+    exactly one logit +inf and the others -inf (margin inf - (-inf) = +inf,
+    which a plain evaluation would accept with an infinite radius); the
+    finite rows are certified as usual."""
+    W = np.array([[1, 0], [-1, 0], [-1, 1]], np.float32)
+    b = np.zeros(3, np.float32)
+    H = np.array([[np.inf, 0], [np.nan, 1], [2, -np.inf], [3, 1], [-2, 0.5]], np.float32)
+    cert = oracle.certify(W, b, oracle.sigma_max(W), H, radius_mode=mode)
+    assert cert["accept"].tolist() == [False, False, False, True, True]
+    assert np.all(np.isnan(cert["radius"][:3]))
+    assert np.all(np.isfinite(cert["radius"][3:])) and np.all(cert["radius"][3:] > 0)
