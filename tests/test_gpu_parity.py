@@ -413,3 +413,30 @@ def test_auto_path_choice(dev):
         for x, y in zip(a, c):
             assert np.array_equal(x.view(np.uint8), y.view(np.uint8))
         cache.close()
+
+
+@pytest.mark.parametrize("path", PATHS)
+def test_probe_special_queries(dev, path):
+    """Queries with NaN or infinite features, and of magnitude 1e30, miss on
+    every path (the strict test fails; nothing is accepted that the oracle
+    rejects); a zero query and tiny ones get the oracle's answer."""
+    w = synth.WORKLOADS["cifar10"].scaled(N=4000, n_queries=64)
+    W, b = synth.head(w)
+    rows = synth.cache_rows(w)
+    cache, _ = make_cache(dev, W, b, w.N)
+    cache.insert(T(rows, dev))
+    ref = oracle.build_cache(W, b, oracle.sigma_max(W), rows)
+    q = np.tile(rows[:1], (8, 1)).astype(np.float32)
+    q[0, 3] = np.nan
+    q[1, :] = np.inf
+    q[2, 7] = -np.inf
+    q[3] *= np.float32(1e30)
+    q[4] = 0
+    q[5] *= np.float32(1e-30)
+    # q[6], q[7]: the cached row itself and a copy
+    gi, gl, gd = run_probe(cache, q, dev, 64, path)
+    assert np.all(gi[:4] == -1) and np.all(gl[:4] == -1) and np.all(np.isinf(gd[:4]))
+    orc = oracle.probe(ref["keys"], ref["radius"], ref["label"], q)
+    check_probe(gi, gl, gd, ref, q, orc)
+    assert gi[6] == 0 and gi[7] == 0
+    cache.close()
