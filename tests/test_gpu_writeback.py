@@ -6,7 +6,7 @@ import pytest
 import oracle
 import synth
 from conftest import golden
-from parity_utils import check_insert, check_probe
+from parity_utils import RTOL, check_insert, check_probe, refine_slack_tight
 
 torch = pytest.importorskip("torch")
 pytestmark = pytest.mark.gpu
@@ -27,9 +27,9 @@ def T(x, dev):
     return torch.from_numpy(np.ascontiguousarray(x)).to(dev)
 
 
-def make_cache(dev, W, b, capacity, path="auto"):
+def make_cache(dev, W, b, capacity, path="auto", mode="conservative"):
     from paper_2608_13144_gb300.lipcache import LipCache
-    c = LipCache(W.shape[1], W.shape[0], capacity, device=dev)
+    c = LipCache(W.shape[1], W.shape[0], capacity, mode, device=dev)
     sigma = c.set_head(T(W, dev), T(b, dev))
     c.set_probe_path(path)
     return c, sigma
@@ -137,6 +137,54 @@ def test_writeback_workload(dev, name, path):
                cert["radius"][add]]), "label": np.concatenate([cur["label"], cert["label"][add]]),
                "yG": np.concatenate([cur["yG"], cert["yG"][add]])}
     assert total_ins > 0 and cache.size == len(cur["keys"])
+    gi, gl, gd = np_(*cache.probe(T(Q, dev)))
+    orc = oracle.probe(cur["keys"], cur["radius"], cur["label"], Q)
+    check_probe(gi, gl, gd, cur, Q, orc)
+    assert cache.info()["device_errors"] == 0
+    cache.close()
+
+
+@pytest.mark.parametrize("name,path", [("tiny", "exact"), ("cifar100", "tensor"), ("tinyimagenet", "tensor")])
+def test_writeback_tight_radius(dev, name, path):
+    """Write-back with the tight radius (Eq. 29): the misses Algorithm 1
+    accepts are certified on the same kernels as an insert, so the set
+    written back is exactly the oracle's, in query order, and each new radius
+    (rounded toward zero) exceeds the FP64 one by no more than the compensated
+    refinement's error bound. The grown cache then probes like the oracle's
+    outside the 1e-5 band."""
+    w, W, b, rows, Q = _workload(name, 2000, 1500)
+    sigma = oracle.sigma_max(W)
+    ref = oracle.build_cache(W, b, sigma, rows, radius_mode=oracle.RADIUS_TIGHT)
+    cache, _ = make_cache(dev, W, b, len(rows) + len(Q), path, "tight")
+    gidx, grad, nacc = cache.insert(T(rows, dev))
+    check_insert(gidx.cpu().numpy(), grad.cpu().numpy(), nacc, ref, ("tight", W, b, rows, 1.0))
+    cur = {k: ref[k] for k in ("keys", "radius", "label", "yG")}
+    n_base = len(cur["keys"])
+    for s, e in synth.batches(len(Q), w.batch):
+        q = Q[s:e]
+        gi, gl, gd, ins, n = cache.probe_writeback(T(q, dev))
+        gi, gl, gd, ins = np_(gi, gl, gd, ins)
+        res = oracle.probe_writeback(cur, W, b, sigma, q, radius_mode=oracle.RADIUS_TIGHT)
+        check_probe(gi, gl, gd, cur, q, res["probe"])
+        # the oracle's write-back set follows its own probe; the GPU's follows
+        # the GPU probe, which agrees outside the band (checked above)
+        add = (gi < 0) & res["cert"]["accept"]
+        exp = np.full(len(q), -1, np.int64)
+        exp[add] = len(cur["keys"]) + np.arange(int(add.sum()))
+        assert np.array_equal(ins, exp), f"{(ins != exp).sum()} write-back indices differ"
+        assert n == int(add.sum())
+        cert = res["cert"]
+        cur = {"keys": np.concatenate([cur["keys"], q[add]]), "radius": np.concatenate([cur["radius"],
+               cert["radius"][add]]), "label": np.concatenate([cur["label"], cert["label"][add]]),
+               "yG": np.concatenate([cur["yG"], cert["yG"][add]])}
+    assert cache.size == len(cur["keys"]) > n_base
+    ent = cache.entries(n_base)
+    r = cur["radius"][n_base:]
+    assert np.array_equal(ent["keys"], cur["keys"][n_base:])
+    assert np.array_equal(ent["label"], cur["label"][n_base:]) and np.array_equal(ent["yG"], cur["yG"][n_base:])
+    g_r = ent["radius"].astype(np.float64)
+    np.testing.assert_allclose(g_r, r, rtol=RTOL)
+    assert np.all(g_r <= r * (1 + 1e-12) + refine_slack_tight(W, b, cur["keys"][n_base:]))
     gi, gl, gd = np_(*cache.probe(T(Q, dev)))
     orc = oracle.probe(cur["keys"], cur["radius"], cur["label"], Q)
     check_probe(gi, gl, gd, cur, Q, orc)
