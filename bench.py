@@ -187,7 +187,7 @@ def roofline(w: synth.Workload, N: int, B: int, kernel_ms: float, pk: dict, pk_k
 
 
 # main probe kernel per path: name, ncu summary, the sources its hash covers
-INSERT_KERNELS = {1: "k_certify_wt", 2: "k_certify_wres", 3: "k_certify"}
+INSERT_KERNELS = {1: "k_certify_wt", 2: "k_certify_wres", 3: "k_certify", 4: "k_certify_tc"}
 PROBE_KERNELS = {
     4: ("k_probe_pair", "k_probe_pair_scale.md", ("probe_pair.cu", "tc_ptx.cuh", "probe_common.cuh")),
     3: ("k_probe_tc", "k_probe_tc_scale.md", ("probe_tc.cu", "tc_ptx.cuh", "probe_common.cuh")),

@@ -58,16 +58,24 @@ typedef enum lipcache_status {
 #define LIPCACHE_RADIUS_CONSERVATIVE 0 /* r  = m / (sigma_max(W) sqrt 2), Eq. 21 */
 #define LIPCACHE_RADIUS_TIGHT 1        /* r* = min_j (s_y - s_j) / ||W_y - W_j||, Eq. 29 */
 
-/* Certify kernels (lipcache_info.last_insert_kernel). WIDE_TILE: head resident
- * in shared memory, 128-row tiles, logits in registers (d % 4 == 0, head small
- * enough; both radii, the tight one refining only the classes that can be its
- * minimiser). TILE64: head resident, 64-row tiles, logits in shared memory.
- * STREAMED: head read from L2 (large heads). For the conservative radius all
- * three compute the same values; for the tight radius the last two refine
- * every class in FP64 and agree with WIDE_TILE within the refinement bound. */
+/* Certify kernels (lipcache_info.last_insert_kernel).
+ * TENSOR: TF32 tcgen05 screen of the logits into tensor memory, conservative
+ *   radius only (d % 16 == 0, d >= 32, 2 <= C <= 256, head resident in shared
+ *   memory); it refines and finishes rows exactly as WIDE_TILE.
+ * WIDE_TILE: head resident in shared memory, 128-row tiles, logits in
+ *   registers (d % 4 == 0, head small enough; both radii, the tight one
+ *   refining only the classes that can be its minimiser).
+ * TILE64: head resident, 64-row tiles, logits in shared memory.
+ * STREAMED: head read from L2 (large heads).
+ * For the conservative radius TENSOR, WIDE_TILE and TILE64 give the same bits;
+ * STREAMED refines with a 32-lane compensated sum, so its radii agree with
+ * theirs within the refinement bound. For the tight radius TILE64 and
+ * STREAMED refine every class in FP64 and agree with WIDE_TILE within the
+ * refinement bound. */
 #define LIPCACHE_INSERT_WIDE_TILE 1
 #define LIPCACHE_INSERT_TILE64 2
 #define LIPCACHE_INSERT_STREAMED 3
+#define LIPCACHE_INSERT_TENSOR 4
 
 /* Radius policies of the probe (lipcache_set_radius_policy). */
 #define LIPCACHE_POLICY_CERTIFIED 0  /* per-entry certified radius (Eq. 21 or Eq. 29) */
@@ -117,6 +125,10 @@ typedef struct lipcache_info {
   double policy_param;      /* tau (GLOBAL) or beta (INTERCLASS); 0 for CERTIFIED */
   double insert_kernel_ms_total; /* summed certify-kernel time of timed inserts since the last reset */
   int64_t insert_kernel_launches; /* number of timed certify kernels in insert_kernel_ms_total */
+  int64_t insert_refined_pairs; /* (row, class) pairs the tensor certify kernel refined (compensated dot
+                                   product) since the last reset */
+  int64_t insert_full_rows;     /* row halves it refined over every class of the half (more candidates
+                                   than slots, a NaN logit or an unbounded screen error) */
 } lipcache_info;
 
 /*
@@ -349,6 +361,14 @@ lipcache_status lipcache_read_head(lipcache_t* h, float* W_host, float* b_host, 
 /* Certify inserted rows with the 64-row-tile kernel where the wide-tile one
  * would run; both compute the same values, so tests compare them bit for bit. */
 #define LIPCACHE_DEBUG_INSERT_TILE64 2
+/* Certify with the wide-tile kernel where the tensor one would run (tests
+ * compare the two bit for bit). */
+#define LIPCACHE_DEBUG_INSERT_WIDE_TILE 4
+/* The MMA issuer of the tensor certify kernel first waits on an mbarrier that
+ * nothing arrives on: the bounded wait expires, the kernel aborts, no row is
+ * appended and lipcache_insert (and the other certifying entry points)
+ * return LIPCACHE_E_DEVICE with the cache unchanged. */
+#define LIPCACHE_DEBUG_STALL_INSERT 8
 lipcache_status lipcache_set_debug(lipcache_t* h, int32_t flags);
 
 /*

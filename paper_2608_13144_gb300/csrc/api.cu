@@ -288,7 +288,9 @@ LC_API lipcache_status lipcache_insert(lipcache_t* h, const float* H, int64_t n,
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     lc::certify_insert(h, H, n, payload, require_consistency, out_index, out_radius, s);
     LC_CUDA(cudaMemcpyAsync(h->ins_total_host, h->ins_total, sizeof(int64_t), cudaMemcpyDeviceToHost, s));
+    LC_CUDA(cudaMemcpyAsync(h->stats_host, h->stats, sizeof(lc::DevStats), cudaMemcpyDeviceToHost, s));
     LC_CUDA(cudaStreamSynchronize(s));
+    LC_REQUIRE(h->stats_host->abort_flag == 0, LIPCACHE_E_DEVICE, lc::kCertifyAbortMessage);
     const int64_t acc = *h->ins_total_host;
     const int64_t first = h->size;
     h->size += acc;
@@ -379,7 +381,9 @@ LC_API lipcache_status lipcache_probe_writeback(lipcache_t* h, const float* Q, i
     require_no_abort(h, s);  // an aborted probe reports misses: write nothing back
     lc::certify_insert(h, Q, B, payload, require_consistency, out_inserted, nullptr, s, out_index);
     LC_CUDA(cudaMemcpyAsync(h->ins_total_host, h->ins_total, sizeof(int64_t), cudaMemcpyDeviceToHost, s));
+    LC_CUDA(cudaMemcpyAsync(h->stats_host, h->stats, sizeof(lc::DevStats), cudaMemcpyDeviceToHost, s));
     LC_CUDA(cudaStreamSynchronize(s));
+    LC_REQUIRE(h->stats_host->abort_flag == 0, LIPCACHE_E_DEVICE, lc::kCertifyAbortMessage);
     const int64_t acc = *h->ins_total_host;
     const int64_t first = h->size;
     h->size += acc;
@@ -408,7 +412,9 @@ LC_API lipcache_status lipcache_consistency(lipcache_t* h, const float* Q, int64
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     lc::consistency_check(h, Q, B, hit_index, out_consistent, s);
     LC_CUDA(cudaMemcpyAsync(h->ins_total_host + 1, h->ins_total + 1, 3 * sizeof(int64_t), cudaMemcpyDeviceToHost, s));
+    LC_CUDA(cudaMemcpyAsync(h->stats_host, h->stats, sizeof(lc::DevStats), cudaMemcpyDeviceToHost, s));
     LC_CUDA(cudaStreamSynchronize(s));
+    LC_REQUIRE(h->stats_host->abort_flag == 0, LIPCACHE_E_DEVICE, lc::kCertifyAbortMessage);
     if (n_hits) *n_hits = h->ins_total_host[1];
     if (n_consistent) *n_consistent = h->ins_total_host[2];
     LC_REQUIRE(h->ins_total_host[3] == 0, LIPCACHE_E_INVALID, "hit_index holds values outside [-1, size)");
@@ -476,7 +482,9 @@ LC_API lipcache_status lipcache_read_head(lipcache_t* h, float* W_host, float* b
 LC_API lipcache_status lipcache_set_debug(lipcache_t* h, int32_t flags) {
   return guarded([&] {
     check_handle(h);
-    LC_REQUIRE((flags & ~(LIPCACHE_DEBUG_STALL_PROBE | LIPCACHE_DEBUG_INSERT_TILE64)) == 0, LIPCACHE_E_INVALID,
+    LC_REQUIRE((flags & ~(LIPCACHE_DEBUG_STALL_PROBE | LIPCACHE_DEBUG_INSERT_TILE64 |
+                          LIPCACHE_DEBUG_INSERT_WIDE_TILE | LIPCACHE_DEBUG_STALL_INSERT)) == 0,
+               LIPCACHE_E_INVALID,
                "unknown debug flags");
     h->debug_flags = flags;
   });
@@ -601,6 +609,8 @@ LC_API lipcache_status lipcache_get_info(lipcache_t* h, lipcache_info* info) {
     info->c_screen = h->c_scr;
     info->candidates = (int64_t)h->stats_host->candidates;
     info->device_errors = (int64_t)h->stats_host->errors;
+    info->insert_refined_pairs = (int64_t)h->stats_host->ins_pairs;
+    info->insert_full_rows = (int64_t)h->stats_host->ins_full_rows;
     info->probe_path = h->probe_path;
     info->last_probe_path = h->last_probe_path;
     info->last_probe_ms = h->last_ms;

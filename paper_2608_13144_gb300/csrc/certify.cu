@@ -36,7 +36,7 @@
 // (k_certify_wt, both radii); with d % 4 != 0, 64-row tiles with the logits in
 // shared memory (k_certify_wres); for larger heads each CTA streams W from L2
 // (k_certify). Insertion order is kept by a block-count scan and a scatter.
-#include "internal.cuh"
+#include "certify_common.cuh"
 #include "tc_ptx.cuh"
 
 namespace lc {
@@ -45,216 +45,6 @@ namespace {
 constexpr int kRows = 32;
 constexpr int kThreads = 256;
 constexpr int kWarps = kThreads / 32;
-constexpr unsigned kFull = 0xffffffffu;
-
-struct CertArgs {
-  const float* H;
-  int64_t n;
-  int d, C, hstride, lstride, tight, require_consistency;
-  const float* W;
-  const float* b;
-  const double* Wnorm;
-  const double* pairnorm;
-  const int32_t* payload;
-  double sigma, kappa, eps_rc, gamma_rc, c_scr, g32, g64;
-  const float* Wnorm32;  // ||W_c|| rounded up
-  float g32f;            // gamma_{d+2} with FP32 rounding slack
-  float g2f;             // error factor of the compensated dot product
-  double inv_denom;      // kappa / (sigma sqrt 2)
-  double inv_denom_safe; // kappa (1 - 8u) / (sigma (1 + slack) sqrt 2)
-  ThreshConsts tc;       // constants of the probe thresholds
-  const int64_t* miss_of;      // nullable: row accepted only if miss_of[row] < 0 (write-back)
-  const double* inv_pairnorm;  // 1 / ||W_y - W_j|| (tight mode)
-  const float* ipn_up32;       // FP32 brackets of 1 / ||W_y - W_j|| (tight mode; +inf where the rows coincide)
-  const float* ipn_dn32;
-  double tight_f;              // 1 - gamma_{d+8} (FP64)
-  uint8_t* accept;
-  int32_t* yG;
-  int32_t* label;
-  float* radius;
-  float* rr;
-  float* kn;
-  float* tau;
-  int32_t* rank;
-  int32_t* bcount;
-};
-
-__device__ __forceinline__ float warp_sum_f(float v) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(kFull, v, o);
-  return v;
-}
-__device__ __forceinline__ double warp_sum_d(double v) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(kFull, v, o);
-  return v;
-}
-__device__ __forceinline__ double warp_max_d(double v) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v = fmax(v, __shfl_xor_sync(kFull, v, o));
-  return v;
-}
-__device__ __forceinline__ double warp_min_d(double v) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v = fmin(v, __shfl_xor_sync(kFull, v, o));
-  return v;
-}
-// insert v into (t1 >= t2)
-__device__ __forceinline__ void top2_push(double& t1, double& t2, double v) {
-  if (v > t1) {
-    t2 = t1;
-    t1 = v;
-  } else if (v > t2) {
-    t2 = v;
-  }
-}
-
-// FP32 error-free transformations: a + b = s + e and a * b = p + e exactly
-// (Knuth's TwoSum; TwoProduct with a fused multiply-add).
-__device__ __forceinline__ void two_sum(float a, float b, float& s, float& e) {
-  s = __fadd_rn(a, b);
-  const float bb = __fsub_rn(s, a);
-  e = __fadd_rn(__fsub_rn(a, __fsub_rn(s, bb)), __fsub_rn(b, bb));
-}
-
-// Compensated dot product W_c . h + b_c (Ogita, Rump and Oishi's Dot2, summed
-// across the warp with the same transformations), returned as a normalised
-// pair hi + lo (|lo| <= ulp(hi)/2) whose exact sum is within
-// 2 gamma_{d+40}^2 (sum_j |W_cj h_j| + |b_c|) of the exact value. Every lane
-// gets the same bits: each butterfly step combines the two partners' pairs
-// symmetrically. wc[j * ws] and hrow[j * hs] address feature j of the
-// weights and of the row (global memory, or the transposed shared tiles).
-__device__ __forceinline__ void dot2_logit(const float* __restrict__ wc, int ws, const float* __restrict__ hrow, int hs,
-                                           float bias, int d, int lane, float& hi, float& lo) {
-  float p = 0.f, c = 0.f;
-  for (int j = lane; j < d; j += 32) {
-    const float w = wc[(size_t)j * ws], x = hrow[(size_t)j * hs];
-    const float pr = __fmul_rn(w, x);
-    const float er = __fmaf_rn(w, x, -pr);
-    float t, q;
-    two_sum(p, pr, t, q);
-    p = t;
-    c = __fadd_rn(c, __fadd_rn(q, er));
-  }
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    const float pb = __shfl_xor_sync(kFull, p, o), cb = __shfl_xor_sync(kFull, c, o);
-    float t, q;
-    two_sum(p, pb, t, q);
-    p = t;
-    c = __fadd_rn(__fadd_rn(c, cb), q);
-  }
-  float t, q;
-  two_sum(p, bias, t, q);
-  two_sum(t, __fadd_rn(c, q), hi, lo);
-}
-
-// Absolute error allowance for subnormal intermediate results: at most
-// 2^-150 per rounding, (d + 40) * 2^-150 < 1e-39 in all for d <= 1024.
-constexpr float kTinyF = 1e-35f;
-
-// Rounded-up bound E_c of |s~_c - s_c| for an FP32 logit s~_c:
-// gamma_{d+2} (||W_c|| ||z|| + |b_c|) (g32f carries the slack for its own
-// rounding), 2^-22 |s~_c| for the rounding of the interval ends, and kTinyF.
-__device__ __forceinline__ float logit_err(float g32f, float wn, float hn, float b, float sv) {
-  return __fmaf_ru(g32f, __fmaf_ru(wn, hn, fabsf(b)), __fmaf_ru(fabsf(sv), 2.3841858e-07f /* 2^-22 */, kTinyF));
-}
-
-// (ah, al) > (bh, bl) for pairs normalised by a final TwoSum (hi = RN(hi + lo)):
-// round-to-nearest is monotone, so this orders the exact sums.
-__device__ __forceinline__ bool pair_gt(float ah, float al, float bh, float bl) {
-  return ah > bh || (ah == bh && al > bl);
-}
-
-// Per-row result of the candidate refinement: the best and second-best
-// refined logits (pairs hi + lo), the error bound of the best, the largest
-// upper bound v + e among the other candidates, ||z||^2 (FP32) and y^G.
-struct RowVals {
-  float h1, l1, e1, h2, l2, up, kn;
-  int y;
-};
-
-// Upper bound of ||z|| from the FP32 sum of squares kn (any order: within
-// gamma_d < 1e-4 of ||z||^2 for d <= 1024, plus d * 2^-150 for subnormal
-// squares).
-__device__ __forceinline__ float norm_upper(float kn) {
-  return __fmul_ru(__fsqrt_ru(__fmaf_ru(kn, 1.0f + 1e-4f, kTinyF)), 1.0f + 1e-6f);
-}
-
-// Bound of |hi + lo - s_c| for a refined logit, rounded up (plus the absolute
-// error of subnormal products).
-__device__ __forceinline__ float refined_err(float g2f, float wn, float hn, float b) {
-  return __fmaf_ru(g2f, __fmaf_ru(wn, hn, fabsf(b)), kTinyF);
-}
-
-// Running selection over refined candidates, visited in any order: the best
-// by (value desc, class asc), the second-best value, and the top two upper
-// bounds with the class of the first, so that the largest upper bound among
-// the classes other than the best is available at the end.
-struct Top2 {
-  float b1h = -INFINITY, b1l = 0.f, b2h = -INFINITY, b2l = 0.f, e1 = 0.f;
-  float u1 = -INFINITY, u2 = -INFINITY;
-  int y = -1, cu1 = -1;
-  bool nan = false;  // a refined logit is NaN: the row is rejected
-  __device__ __forceinline__ void push(int c, float vh, float vl, float e) {
-    nan |= !(vh == vh && vl == vl);
-    const bool eq1 = vh == b1h && vl == b1l;
-    if (pair_gt(vh, vl, b1h, b1l) || (eq1 && c < y)) {
-      b2h = b1h;
-      b2l = b1l;
-      b1h = vh;
-      b1l = vl;
-      e1 = e;
-      y = c;
-    } else if (pair_gt(vh, vl, b2h, b2l) || (vh == b2h && vl == b2l)) {
-      b2h = vh;
-      b2l = vl;
-    }
-    const float up = __fadd_ru(vh, __fadd_ru(vl, e));
-    if (up > u1) {
-      u2 = u1;
-      u1 = up;
-      cu1 = c;
-    } else if (up > u2) {
-      u2 = up;
-    }
-  }
-  __device__ __forceinline__ RowVals result(float kn) const {
-    RowVals v;
-    v.h1 = nan ? NAN : b1h;
-    v.l1 = b1l;
-    v.e1 = e1;
-    v.h2 = b2h;
-    v.l2 = b2l;
-    v.up = (cu1 == y) ? u2 : u1;
-    v.kn = kn;
-    v.y = y < 0 ? 0 : y;  // every refined logit NaN: the margin is NaN and the row is rejected
-    return v;
-  }
-};
-
-// FP64 margin, radius, certified lower bound and probe thresholds of one row
-// (one thread), and the skip rules of Algorithm 1.
-__device__ void row_finals(const CertArgs& a, int64_t row, const RowVals& v, uint8_t* acc_slot) {
-  const double v1 = (double)v.h1 + (double)v.l1, v2 = (double)v.h2 + (double)v.l2;
-  const double mval = (v1 == v1 && v2 == v2) ? v1 - v2 : NAN;
-  // lower bound of the exact margin with downward rounding
-  const double mlo = __dsub_rd(__dsub_rd(v1, (double)v.e1), (double)v.up);
-  const double r64 = mval * a.inv_denom;
-  const double rs = (mlo > 0.0) ? __dmul_rd(mlo, a.inv_denom_safe) : 0.0;
-  const int32_t lab = a.payload ? a.payload[row] : v.y;
-  const bool acc = !(a.require_consistency && lab != v.y) && (r64 > 0.0) && !(a.miss_of && a.miss_of[row] >= 0);
-  float rr, tau;
-  thresholds(__double2float_rd(rs), v.kn, a.tc, rr, tau);
-  a.accept[row] = acc ? 1 : 0;
-  a.yG[row] = v.y;
-  a.label[row] = lab;
-  a.radius[row] = __double2float_rz(r64);
-  a.rr[row] = rr;
-  a.kn[row] = v.kn;
-  a.tau[row] = tau;
-  *acc_slot = acc ? 1 : 0;
-}
 
 // One row with one warp, conservative radius (Eq. 21): the FP32 intervals
 // s~_c +- E_c select every class that can be among the true top two; those
@@ -542,13 +332,6 @@ __global__ void __launch_bounds__(kThreads) k_certify(CertArgs a) {
 //     lowest class) and runs the FP64 finals. A row with more than
 //     kMaxCand candidates is redone by one warp with warp_row_refine.
 //     The tight radius runs certify_row (FP64) with one warp per row.
-// Start moving `bytes` (a multiple of 16) from global memory at `src` (16-byte
-// aligned) into L2, without waiting.
-__device__ __forceinline__ void prefetch_l2_bulk(const void* src, uint32_t bytes) {
-  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(reinterpret_cast<uint64_t>(src)), "r"(bytes)
-               : "memory");
-}
-
 constexpr int kWTile = 64;    // rows per tile
 constexpr int kHStride = 68;  // h^T row stride (floats): 16-byte aligned, banks spread
 constexpr int kMaxCand = 16;  // candidate slots per row
@@ -1539,8 +1322,9 @@ int wt_ncg(int C) {
 }
 
 // Exclusive scan of the per-block accepted counts (one block).
+// (after an aborted certify kernel every count reads as 0: nothing is appended)
 __global__ void __launch_bounds__(1024) k_scan(const int32_t* __restrict__ cnt, int32_t* __restrict__ off, int nb,
-                                               int64_t* __restrict__ total) {
+                                               int64_t* __restrict__ total, const DevStats* __restrict__ st) {
   __shared__ int32_t buf[1024];
   __shared__ int64_t carry;
   const int tid = threadIdx.x;
@@ -1548,7 +1332,7 @@ __global__ void __launch_bounds__(1024) k_scan(const int32_t* __restrict__ cnt, 
   __syncthreads();
   for (int base = 0; base < nb; base += 1024) {
     const int i = base + tid;
-    const int v = i < nb ? cnt[i] : 0;
+    const int v = (i < nb && st->abort_flag == 0) ? cnt[i] : 0;
     buf[tid] = v;
     __syncthreads();
     for (int s = 1; s < 1024; s <<= 1) {
@@ -1581,6 +1365,7 @@ struct ScatterArgs {
   Table t;
   int64_t* out_index;
   float* out_radius;
+  const DevStats* st;  // abort_flag set: the certify kernel gave up, nothing is appended
 };
 
 // Append accepted rows in input order. Each warp moves kScatterRows rows:
@@ -1596,7 +1381,8 @@ __global__ void __launch_bounds__(256) k_scatter(ScatterArgs a, int vec) {
   int64_t mydst = -2;  // past the end
   if (lane < kScatterRows && row0 + lane < a.n) {
     const int64_t row = row0 + lane;
-    mydst = a.accept[row] ? a.size0 + a.boff[row / kRows] + a.rank[row] : -1;
+    const bool dead = a.st->abort_flag != 0;
+    mydst = (!dead && a.accept[row]) ? a.size0 + a.boff[row / kRows] + a.rank[row] : -1;
     if (mydst >= 0) {
       a.t.kn[mydst] = a.kn[row];
       a.t.tau[mydst] = a.tau[row];
@@ -1606,7 +1392,7 @@ __global__ void __launch_bounds__(256) k_scatter(ScatterArgs a, int vec) {
       a.t.yG[mydst] = a.yG[row];
     }
     if (a.out_index) a.out_index[row] = mydst;
-    if (a.out_radius) a.out_radius[row] = a.radius[row];
+    if (a.out_radius) a.out_radius[row] = dead ? NAN : a.radius[row];
   }
   int64_t dst[kScatterRows];
 #pragma unroll
@@ -1718,6 +1504,8 @@ int timing_begin(lipcache* h, cudaStream_t s) {
 void launch_certify(lipcache* h, const float* H, int64_t n, const int32_t* payload, int require_consistency,
                     const int64_t* miss_of, cudaStream_t s) {
   ensure_insert_scratch(h, n);
+  // raised by the tensor kernel if one of its bounded waits expires
+  LC_CUDA(cudaMemsetAsync(&h->stats->abort_flag, 0, sizeof(int), s));
   CertArgs a;
   a.H = H;
   a.n = n;
@@ -1771,8 +1559,12 @@ void launch_certify(lipcache* h, const float* H, int64_t n, const int32_t* paylo
   const int ncg = wt_ncg(h->C);
   const bool vec16 = h->d % 4 == 0 && ((uintptr_t)H & 15) == 0;
   const WtLayout L = wt_layout(h->d, h->C, ncg > 0 ? ncg : 1);
-  if ((!a.tight || h->ipn_up32) && vec16 && ncg > 0 && L.total <= 227 * 1024 &&
-      !(h->debug_flags & LIPCACHE_DEBUG_INSERT_TILE64)) {
+  if (certify_tc_supported(h, H, n)) {
+    slot = timing_begin(h, s);
+    certify_tc_launch(h, a, s);
+    h->last_insert_kernel = LIPCACHE_INSERT_TENSOR;
+  } else if ((!a.tight || h->ipn_up32) && vec16 && ncg > 0 && L.total <= 227 * 1024 &&
+             !(h->debug_flags & LIPCACHE_DEBUG_INSERT_TILE64)) {
     const int64_t nb32 = (n + 31) / 32;
     const int grid = nb32 < h->num_sms ? (int)nb32 : h->num_sms;
     if (h->wt_prep_ncg != ncg) {
@@ -1826,7 +1618,7 @@ void certify_insert(lipcache* h, const float* H, int64_t n, const int32_t* paylo
                     int64_t* out_index, float* out_radius, cudaStream_t s, const int64_t* miss_of) {
   launch_certify(h, H, n, payload, require_consistency, miss_of, s);
   const int nb = (int)((n + kRows - 1) / kRows);
-  k_scan<<<1, 1024, 0, s>>>(h->ins_bcount, h->ins_boffset, nb, h->ins_total);
+  k_scan<<<1, 1024, 0, s>>>(h->ins_bcount, h->ins_boffset, nb, h->ins_total, h->stats);
   LC_LAUNCH_CHECK("k_scan");
   ScatterArgs sa;
   sa.H = H;
@@ -1846,10 +1638,17 @@ void certify_insert(lipcache* h, const float* H, int64_t n, const int32_t* paylo
   sa.t = h->table;
   sa.out_index = out_index;
   sa.out_radius = out_radius;
+  sa.st = h->stats;
   const int vec = (h->d % 4 == 0 && ((uintptr_t)H & 15) == 0) ? 1 : 0;
   const int64_t rows_per_block = 8 * kScatterRows;
   k_scatter<<<(unsigned)((n + rows_per_block - 1) / rows_per_block), 256, 0, s>>>(sa, vec);
   LC_LAUNCH_CHECK("k_scatter");
+}
+
+void require_certify_ok(lipcache* h, cudaStream_t s) {
+  LC_CUDA(cudaMemcpyAsync(h->stats_host, h->stats, sizeof(DevStats), cudaMemcpyDeviceToHost, s));
+  LC_CUDA(cudaStreamSynchronize(s));
+  LC_REQUIRE(h->stats_host->abort_flag == 0, LIPCACHE_E_DEVICE, kCertifyAbortMessage);
 }
 
 void certify_rows(lipcache* h, const float* H, int64_t n, const int32_t* payload, int require_consistency,

@@ -1,0 +1,691 @@
+// Certified insertion on the tensor cores (Sec. 3.3, Algorithm 1 loop body;
+// Eqs. 5, 6, 20, 21), conservative radius.
+//
+// The head logits of a batch, s = W z + b for every row z, form one dense
+// contraction (rows x d) . (d x C). This kernel runs it as TF32 tcgen05 MMAs
+// (M = 128 rows, N = C padded to a multiple of 16, K = 8 per instruction) into
+// tensor memory, and uses the result only as a screen that picks the classes
+// that can be among the true top two; those are recomputed with the same
+// compensated FP32 dot product, in the same order, as the wide-tile kernel, and
+// the FP64 finals are shared. The radii, labels and thresholds therefore come
+// out bit for bit as from the FP32 kernels.
+//
+// Screen bound. The MMA returns a_c with |a_c - W_c . z| <= c ||W_c|| ||z||
+// (c = c_screen: TF32 operands within 2^-10 relative, FP32-accurate
+// accumulation, doubled for safety; the probe's screen uses the same bound),
+// and s~_c = fl(a_c + b_c) adds at most 2^-24 |a_c + b_c| <= 2^-24 Mb, with
+// hn >= ||z||, wmax >= max_c ||W_c|| and Mb = (1 + c) wmax hn + max_c |b_c|:
+//     |s~_c - s_c| <= E = c wmax hn + 2^-22 Mb + tiny      (rounded up).
+// Mb also bounds every partial sum of the MMA, so when Mb < 1e38 no screen
+// value overflows or is NaN; a row with a larger (or NaN) Mb - NaN or infinite
+// features, or values near the FP32 range - has every class refined.
+// If l2 is the second-largest s~_c, every class of the true top two has
+// s_c >= (true runner-up) >= l2 - E, hence s~_c >= l2 - 2E >= T = RD(l2 - 2E):
+// the classes with s~_c >= T are the candidates.
+//
+// Schedule. Persistent CTAs, one per SM, 320 threads:
+//   warp 0     TMA producer: W (resident, 128-byte swizzle, rows past C zero
+//              filled), then each tile's 128 rows (one 16 KB box per 32-feature
+//              chunk, features past d zero filled) into one of nzb buffers,
+//              and the CTA's next tile into L2;
+//   warp 1     TMEM allocation; one thread issues the MMAs of a tile into one
+//              of two accumulators (columns 0 / 256);
+//   warps 2-9  epilogue, two warps per TMEM lane quarter (32 rows), each
+//              taking every other 32-column chunk of the classes: ||z||^2
+//              (two of its four k-ordered partial chains each) from the tile
+//              in shared memory, the top two s~ and M of its columns,
+//              exchanged with the partner warp; the candidates of its columns
+//              into the warp's pair list. The four groups of 8 lanes refine
+//              the list eight pairs at a time (two per group) into cells by
+//              (row, slot), from which each row's lane takes its own results.
+//              A row with more than kMaxCandTc
+//              candidates in a half, or whose Mb is not below 1e38, has
+//              every class of that half refined. The partner states are merged and
+//              one thread per row runs the FP64 finals.
+// Every mbarrier wait is bounded; a role that gives up raises the CTA's abort
+// flag, the others drain, and the launch counts a device error.
+#include "certify_common.cuh"
+#include "tc_ptx.cuh"
+
+namespace lc {
+namespace {
+
+constexpr int kBM = 128;                      // rows per tile (MMA M, TMEM lanes)
+constexpr int kChunkF = 32;                   // features per 128-byte swizzle row
+constexpr int kMaxChunks = 8;                 // d <= 256
+constexpr uint32_t kZChunkBytes = kBM * 128;  // one 32-feature chunk of a tile
+constexpr int kEpiWarps = 8;
+constexpr int kThreads = 32 * (2 + kEpiWarps);
+constexpr int kMaxCandTc = 8;                 // candidate slots per row and column half
+constexpr int kListCap = 32 * kMaxCandTc;     // pair list of one epilogue warp
+// per epilogue warp: the pair list, then the refined pairs hi / lo by (row lane, slot)
+constexpr uint32_t kWarpScratch = kListCap * 4 + 32 * kMaxCandTc * 8;
+constexpr int kGroupTc = 8;                   // lanes per refined pair
+constexpr uint32_t kTmemCols = 512;           // two accumulators of up to 256 columns
+constexpr uint32_t kAccStride = 256;
+constexpr long long kWaitLimit = 1LL << 31;   // ~1 s at GB300 clocks
+constexpr int kSmemBudget = 227 * 1024 - 1024;
+
+// Per-row state a half hands to its partner after the first pass: the top
+// two s~ of its columns and its half of ||z||^2.
+struct Pass1 {
+  float l1, l2, psum, pad;
+};
+
+// Shared-memory layout (offsets from a 1024-byte aligned base).
+struct TcLayout {
+  int nch, Cpad, nzb;
+  uint32_t wbytes, zbytes;
+  uint32_t off_z, off_bias, off_wn, off_list, off_x1, off_x2, off_acc, off_bar, off_misc, total;
+};
+
+TcLayout tc_layout(int d, int C, int nzb) {
+  TcLayout L;
+  L.nch = (d + kChunkF - 1) / kChunkF;
+  L.Cpad = (C + 15) / 16 * 16;
+  L.nzb = nzb;
+  L.wbytes = (uint32_t)L.nch * (uint32_t)L.Cpad * 128u;  // a multiple of 2048
+  L.zbytes = (uint32_t)L.nch * kZChunkBytes;
+  L.off_z = L.wbytes;
+  L.off_bias = L.off_z + (uint32_t)nzb * L.zbytes;
+  L.off_wn = L.off_bias + 256 * 4;
+  L.off_list = L.off_wn + 256 * 4;
+  L.off_x1 = L.off_list + kEpiWarps * kWarpScratch;
+  L.off_x2 = L.off_x1 + 2 * kBM * (uint32_t)sizeof(Pass1);
+  L.off_acc = L.off_x2 + kBM * (uint32_t)sizeof(Top2);
+  L.off_bar = (L.off_acc + kBM + 32 + 7) / 8 * 8;  // + ok flags of the halves (2 x 4 ints)
+  L.off_misc = L.off_bar + (8 + 2 * kMaxChunks) * 8;  // the barrier map is in the kernel
+  L.total = L.off_misc + 16;
+  return L;
+}
+
+// Byte offset of feature k of row r in a 128-byte-swizzled K-major tile whose
+// 32-feature chunks are `chunk_bytes` apart (TMA SWIZZLE_128B: the 16-byte
+// unit index is XORed with the row index mod 8).
+__device__ __forceinline__ uint32_t sw_off(int r, int k, uint32_t chunk_bytes) {
+  return (uint32_t)(k >> 5) * chunk_bytes + (uint32_t)r * 128u + ((((uint32_t)(k >> 2) & 7u) ^ ((uint32_t)r & 7u)) << 4) +
+         (((uint32_t)k & 3u) << 2);
+}
+
+// 16 bytes of shared memory at byte address `addr` (16-byte aligned).
+__device__ __forceinline__ float4 lds_f4(uint32_t addr) {
+  float4 v;
+  asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];" : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w) : "r"(addr));
+  return v;
+}
+
+// Named barrier of the two epilogue warps of one lane quarter.
+__device__ __forceinline__ void pair_barrier(int id) { asm volatile("bar.sync %0, 64;" ::"r"(id) : "memory"); }
+
+// Top2 over the union of two disjoint class sets from the two sets' states:
+// the same y^G, runner-up value and bounds as pushing every class into one.
+__device__ __forceinline__ void top2_merge(Top2& A, const Top2& B) {
+  const bool b_best = B.y >= 0 && (A.y < 0 || pair_gt(B.b1h, B.b1l, A.b1h, A.b1l) ||
+                                   (B.b1h == A.b1h && B.b1l == A.b1l && B.y < A.y));
+  const Top2& Wn = b_best ? B : A;
+  const Top2& Ls = b_best ? A : B;
+  float sh = Wn.b2h, sl = Wn.b2l;
+  if (pair_gt(Ls.b1h, Ls.b1l, sh, sl) || (Ls.b1h == sh && Ls.b1l == sl)) {
+    sh = Ls.b1h;
+    sl = Ls.b1l;
+  }
+  // largest upper bound among the classes other than the winner
+  const float up = fmaxf((Wn.cu1 == Wn.y) ? Wn.u2 : Wn.u1, Ls.u1);
+  Top2 R;
+  R.b1h = Wn.b1h;
+  R.b1l = Wn.b1l;
+  R.e1 = Wn.e1;
+  R.y = Wn.y;
+  R.b2h = sh;
+  R.b2l = sl;
+  R.u1 = up;
+  R.u2 = up;
+  R.cu1 = -2;
+  R.nan = A.nan || B.nan;
+  A = R;
+}
+
+// Compensated dot products W_c . z_r + b_c of two (row, class) pairs by the 8
+// lanes of a group (lane sub takes features sub, sub + 8, ...; the two chains
+// interleaved for instruction-level parallelism), each in exactly the order of
+// the wide-tile kernel's refinement: TwoProduct and TwoSum per feature, a
+// butterfly over the group, then the bias. Every lane of the group returns the
+// same pairs hi + lo. ws / zs: shared-memory byte addresses of the head and of
+// the tile's features (128-byte swizzle, chunks wchunk / kZChunkBytes apart).
+__device__ __forceinline__ void refine2(uint32_t ws, uint32_t wchunk, uint32_t zs, const int (&c)[2],
+                                        const int (&r)[2], const float (&bias)[2], int d, int sub, float (&hi)[2],
+                                        float (&lo)[2]) {
+  // lane sub reads the 16-byte unit 2 jj + sub / 4 of each 32-feature chunk
+  // (jj = 0..3), word sub % 4; the swizzle XORs the unit with the row mod 8
+  const uint32_t s2 = (uint32_t)sub >> 2, s3 = ((uint32_t)sub & 3u) << 2;
+  uint32_t wb[2], zb[2], ow[2][4], oz[2][4];
+#pragma unroll
+  for (int u = 0; u < 2; ++u) {
+    wb[u] = ws + (uint32_t)c[u] * 128u + s3;
+    zb[u] = zs + (uint32_t)r[u] * 128u + s3;
+#pragma unroll
+    for (int jj = 0; jj < 4; ++jj) {
+      ow[u][jj] = ((2u * jj + s2) ^ ((uint32_t)c[u] & 7u)) << 4;
+      oz[u][jj] = ((2u * jj + s2) ^ ((uint32_t)r[u] & 7u)) << 4;
+    }
+  }
+  // both chains in packed FP32 pairs: (pair 0, pair 1) in (low, high) halves;
+  // every operation rounds each half exactly as the scalar one would
+  uint64_t P = 0ull, CC = 0ull;
+  constexpr uint64_t kSign2 = 0x8000000080000000ull;
+  auto step = [&](uint32_t wa0, uint32_t za0, uint32_t wa1, uint32_t za1) {
+    float w0, x0, w1, x1;
+    asm volatile("ld.shared.f32 %0, [%1];" : "=f"(w0) : "r"(wa0));
+    asm volatile("ld.shared.f32 %0, [%1];" : "=f"(x0) : "r"(za0));
+    asm volatile("ld.shared.f32 %0, [%1];" : "=f"(w1) : "r"(wa1));
+    asm volatile("ld.shared.f32 %0, [%1];" : "=f"(x1) : "r"(za1));
+    const uint64_t w = ptx::pack2_f32(w0, w1), x = ptx::pack2_f32(x0, x1);
+    const uint64_t pr = ptx::mul_f32x2(w, x);                // TwoProduct: pr + er = w x
+    const uint64_t er = ptx::fma_f32x2(w, x, pr ^ kSign2);
+    const uint64_t sm = ptx::add_f32x2(P, pr);               // TwoSum(P, pr) = sm + q
+    const uint64_t bb = ptx::sub_f32x2(sm, P);
+    const uint64_t q = ptx::add_f32x2(ptx::sub_f32x2(P, ptx::sub_f32x2(sm, bb)), ptx::sub_f32x2(pr, bb));
+    P = sm;
+    CC = ptx::add_f32x2(CC, ptx::add_f32x2(q, er));
+  };
+  const int nfull = d >> 5;
+  for (int kc = 0; kc < nfull; ++kc) {
+#pragma unroll
+    for (int jj = 0; jj < 4; ++jj) step(wb[0] + ow[0][jj], zb[0] + oz[0][jj], wb[1] + ow[1][jj], zb[1] + oz[1][jj]);
+#pragma unroll
+    for (int u = 0; u < 2; ++u) {
+      wb[u] += wchunk;
+      zb[u] += kZChunkBytes;
+    }
+  }
+  if (d & 16) {  // a last half chunk (d % 32 == 16): units 0-3
+#pragma unroll
+    for (int jj = 0; jj < 2; ++jj) step(wb[0] + ow[0][jj], zb[0] + oz[0][jj], wb[1] + ow[1][jj], zb[1] + oz[1][jj]);
+  }
+  float p[2], cc[2];
+  ptx::unpack2_f32(P, p[0], p[1]);
+  ptx::unpack2_f32(CC, cc[0], cc[1]);
+#pragma unroll
+  for (int o = kGroupTc / 2; o > 0; o >>= 1) {
+#pragma unroll
+    for (int u = 0; u < 2; ++u) {
+      const float pb = __shfl_xor_sync(kFull, p[u], o), cb = __shfl_xor_sync(kFull, cc[u], o);
+      float t, q;
+      two_sum(p[u], pb, t, q);
+      p[u] = t;
+      cc[u] = __fadd_rn(__fadd_rn(cc[u], cb), q);
+    }
+  }
+#pragma unroll
+  for (int u = 0; u < 2; ++u) {
+    float t, q;
+    two_sum(p[u], bias[u], t, q);
+    two_sum(t, __fadd_rn(cc[u], q), hi[u], lo[u]);
+  }
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+    k_certify_tc(const __grid_constant__ CUtensorMap tmH, const __grid_constant__ CUtensorMap tmW, const CertArgs a,
+                 const TcLayout L, int n_tiles, DevStats* stats, int debug_stall) {
+  extern __shared__ __align__(1024) unsigned char smem_raw[];
+  unsigned char* smem =
+      reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+  const uint32_t s_base = ptx::smem_u32(smem);
+  const uint32_t s_w = s_base, s_z = s_base + L.off_z;
+  const uint32_t bar = s_base + L.off_bar;
+  // barriers: wfull, zempty[2], accfull[2], accempty[2], drain, zfull[2][kMaxChunks]
+  // (one per 32-feature chunk of each feature buffer, so the MMAs start on
+  // the first chunk while the others land)
+  const uint32_t wfull = bar, zempty = bar + 8, accfull = bar + 24, accempty = bar + 40, drain = bar + 56,
+                 zfull = bar + 64;
+  auto zfull_of = [&](int zb, int c) { return zfull + 8u * (uint32_t)(zb * kMaxChunks + c); };
+  float* bias_s = reinterpret_cast<float*>(smem + L.off_bias);
+  float* wn_s = reinterpret_cast<float*>(smem + L.off_wn);
+  unsigned char* scratch = smem + L.off_list;
+  Pass1* x1 = reinterpret_cast<Pass1*>(smem + L.off_x1);
+  Top2* x2 = reinterpret_cast<Top2*>(smem + L.off_x2);
+  uint8_t* acc_s = smem + L.off_acc;
+  volatile int* okf = reinterpret_cast<volatile int*>(smem + L.off_acc + kBM);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L.off_misc);
+  volatile int* abort_s = reinterpret_cast<volatile int*>(smem + L.off_misc + 4);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int d = a.d, C = a.C;
+  if (threadIdx.x == 0) {
+    ptx::mbar_init(wfull, 1);
+    for (int b = 0; b < 2; ++b) {
+      for (int c = 0; c < kMaxChunks; ++c) ptx::mbar_init(zfull_of(b, c), 1);
+      ptx::mbar_init(zempty + 8 * b, kEpiWarps);
+      ptx::mbar_init(accfull + 8 * b, 1);
+      ptx::mbar_init(accempty + 8 * b, kEpiWarps);
+    }
+    ptx::mbar_init(drain, 1);
+    *abort_s = 0;
+    ptx::fence_mbar_init();
+    ptx::tma_prefetch_desc(&tmH);
+    ptx::tma_prefetch_desc(&tmW);
+  }
+  for (int i = threadIdx.x; i < 256; i += kThreads) {
+    bias_s[i] = i < C ? __ldg(a.b + i) : 0.f;
+    wn_s[i] = i < C ? __ldg(a.Wnorm32 + i) : 0.f;
+  }
+  if (warp == 1) {
+    ptx::tmem_alloc(ptx::smem_u32(tmem_slot), kTmemCols);
+    ptx::tmem_relinquish();
+  }
+  ptx::tc_fence_before();
+  __syncthreads();
+  ptx::tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ producer
+    if (lane == 0) {
+      ptx::mbar_expect_tx(wfull, L.wbytes);
+      for (int c = 0; c < L.nch; ++c)
+        ptx::tma_load_2d(s_w + (uint32_t)c * (uint32_t)L.Cpad * 128u, &tmW, c * kChunkF, 0, wfull);
+      bool used[2] = {false, false};
+      uint32_t lastp[2] = {0u, 0u};
+      int t = 0;
+      for (int tile = blockIdx.x; tile < n_tiles; tile += gridDim.x, ++t) {
+        const int zb = t % L.nzb;
+        const uint32_t par = (uint32_t)(t / L.nzb) & 1u;
+        if (!ptx::mbar_wait(zempty + 8 * zb, par ^ 1u, abort_s, kWaitLimit)) break;
+        for (int c = 0; c < L.nch; ++c) {
+          ptx::mbar_expect_tx(zfull_of(zb, c), kZChunkBytes);
+          ptx::tma_load_2d(s_z + (uint32_t)zb * L.zbytes + (uint32_t)c * kZChunkBytes, &tmH, c * kChunkF, tile * kBM,
+                           zfull_of(zb, c));
+        }
+        used[zb] = true;
+        lastp[zb] = par;
+        // the CTA's next tile starts moving into L2 while this one is worked on
+        const int nxt = tile + (int)gridDim.x;
+        if (nxt < n_tiles) {
+          const int64_t r0 = (int64_t)nxt * kBM;
+          const int64_t nr = a.n - r0 < kBM ? a.n - r0 : kBM;
+          prefetch_l2_bulk(a.H + (size_t)r0 * d, (uint32_t)(nr * d * sizeof(float)));
+        }
+      }
+      // every copy into this CTA lands before it can exit (bounded; a phase
+      // that already completed returns at once)
+      volatile int never = 0;
+      for (int b = 0; b < 2; ++b)
+        for (int c = 0; c < L.nch && used[b]; ++c) ptx::mbar_wait(zfull_of(b, c), lastp[b], &never, kWaitLimit);
+      ptx::mbar_wait(wfull, 0, &never, kWaitLimit);
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      const uint32_t idesc = ptx::idesc_tf32(kBM, L.Cpad);
+      const uint64_t zdesc0 = ptx::sw128_kmajor_desc(s_z), wdesc0 = ptx::sw128_kmajor_desc(s_w);
+      const uint64_t zstep = kZChunkBytes >> 4, wstep = ((uint32_t)L.Cpad * 128u) >> 4, zbstep = L.zbytes >> 4;
+      // failure-detection test: no arrival completes this phase before the
+      // final drain, so the bounded wait expires and the kernel aborts
+      bool ok = !debug_stall || ptx::mbar_wait(drain, 0, abort_s, kWaitLimit);
+      ok = ok && ptx::mbar_wait(wfull, 0, abort_s, kWaitLimit);
+      int t = 0;
+      for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x, ++t) {
+        const int buf = t & 1, zb = t % L.nzb;
+        ok = ptx::mbar_wait(accempty + 8 * buf, ((uint32_t)(t >> 1) & 1u) ^ 1u, abort_s, kWaitLimit);
+        if (!ok) break;
+        ptx::tc_fence_after();
+        const uint32_t d_tmem = tmem + (uint32_t)buf * kAccStride;
+        uint64_t zd = zdesc0 + (uint64_t)zb * zbstep, wd = wdesc0;
+        for (int c = 0; c < L.nch; ++c, zd += zstep, wd += wstep) {
+          if (!ptx::mbar_wait(zfull_of(zb, c), (uint32_t)(t / L.nzb) & 1u, abort_s, kWaitLimit)) {
+            ok = false;
+            break;
+          }
+          ptx::tc_fence_after();
+          ptx::mma_tf32(d_tmem, zd, wd, idesc, c != 0);
+          ptx::mma_tf32(d_tmem, zd + 2, wd + 2, idesc, 1u);
+          ptx::mma_tf32(d_tmem, zd + 4, wd + 4, idesc, 1u);
+          ptx::mma_tf32(d_tmem, zd + 6, wd + 6, idesc, 1u);
+        }
+        if (!ok) break;
+        ptx::mma_commit(accfull + 8 * buf);
+      }
+      // every issued MMA completes before TMEM can be released
+      volatile int never = 0;
+      ptx::mma_commit(drain);
+      ptx::mbar_wait(drain, 0, &never, kWaitLimit);
+    }
+    __syncwarp();
+  } else {
+    // ------------------------------------------------------------ epilogue
+    const int ew = warp - 2, quarter = warp & 3, half = ew >> 2;
+    const int r = quarter * 32 + lane;  // row of the tile = TMEM lane
+    const int nck = (C + 31) / 32;
+    // this half's classes: the 32-column chunks half, half + 2, ... (t-th
+    // class of the half: chunk 2 (t / 32) + half, column t % 32)
+    int ncls = 0;
+    for (int ch = half; ch < nck; ch += 2) ncls += min(32, C - ch * 32);
+    const int g8 = lane / kGroupTc, sub = lane % kGroupTc;
+    // the warp's pair list (row lane | slot << 5 | class << 8) and the refined
+    // values by (row lane, slot)
+    int* list = reinterpret_cast<int*>(scratch + (size_t)ew * kWarpScratch);
+    float* res_hi = reinterpret_cast<float*>(scratch + (size_t)ew * kWarpScratch + kListCap * 4);
+    float* res_lo = res_hi + 32 * kMaxCandTc;
+    const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
+    const int dq = d / 4;
+    const int bar_id = 1 + quarter;
+    const uint32_t wchunk = (uint32_t)L.Cpad * 128u;
+    // screen bound terms: c ||W_c|| <= cw and (1 + c) ||W_c|| <= cw1 for every
+    // class, |b_c| <= bmax (rounded up; a NaN bias propagates into bmax)
+    float wmax = 0.f, bmax = 0.f;
+    for (int c = lane; c < C; c += 32) {
+      wmax = fmaxf(wmax, __ldg(a.Wnorm32 + c));
+      const float ab = fabsf(__ldg(a.b + c));
+      bmax = (ab > bmax || ab != ab) ? ab : bmax;
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      wmax = fmaxf(wmax, __shfl_xor_sync(kFull, wmax, o));
+      const float ob = __shfl_xor_sync(kFull, bmax, o);
+      bmax = (ob > bmax || ob != ob) ? ob : bmax;
+    }
+    const float c32 = __double2float_ru(a.c_scr);
+    const float cw = __fmul_ru(c32, wmax), cw1 = __fmul_ru(__fadd_ru(1.f, c32), wmax);
+    // top two of the s~ in a 32-column chunk, four independent trackers
+    // (columns j % 4); columns past C are masked when the chunk is partial
+    auto pass1_chunk = [&](const uint32_t (&v)[32], int ch, float (&t1)[4], float (&t2)[4]) {
+      const int lim = min(32, C - ch * 32);
+      const float4* b4 = reinterpret_cast<const float4*>(bias_s + ch * 32);
+#pragma unroll
+      for (int j4 = 0; j4 < 8; ++j4) {
+        const float4 bb = b4[j4];
+        const float bv[4] = {bb.x, bb.y, bb.z, bb.w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const int j = 4 * j4 + e;
+          float sv = __fadd_rn(__uint_as_float(v[j]), bv[e]);
+          sv = (lim == 32 || j < lim) ? sv : -INFINITY;
+          t2[e] = fmaxf(t2[e], fminf(t1[e], sv));
+          t1[e] = fmaxf(t1[e], sv);
+        }
+      }
+    };
+    // the candidates of a chunk: bit j set iff s~ >= T
+    auto pass2_chunk = [&](const uint32_t (&v)[32], int ch, float T) -> uint32_t {
+      const int lim = min(32, C - ch * 32);
+      const float4* b4 = reinterpret_cast<const float4*>(bias_s + ch * 32);
+      uint32_t mask = 0;
+#pragma unroll
+      for (int j4 = 0; j4 < 8; ++j4) {
+        const float4 bb = b4[j4];
+        const float bv[4] = {bb.x, bb.y, bb.z, bb.w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const int j = 4 * j4 + e;
+          const float sv = __fadd_rn(__uint_as_float(v[j]), bv[e]);
+          mask |= (uint32_t)(sv >= T) << j;
+        }
+      }
+      return lim == 32 ? mask : mask & ((1u << lim) - 1u);
+    };
+
+    unsigned long long n_pairs = 0, n_full = 0;  // this warp's refinement counts
+    int t = 0;
+    for (int tile = blockIdx.x; tile < n_tiles; tile += gridDim.x, ++t) {
+      const int buf = t & 1, zb = t % L.nzb;
+      bool ok = ptx::mbar_wait(accfull + 8 * buf, (uint32_t)(t >> 1) & 1u, abort_s, kWaitLimit);
+      for (int c = 0; c < L.nch && ok; ++c)  // the features are visible to these threads too
+        ok = ptx::mbar_wait(zfull_of(zb, c), (uint32_t)(t / L.nzb) & 1u, abort_s, kWaitLimit);
+      ok = __all_sync(kFull, ok);  // warp-uniform before the aligned TMEM loads
+      ptx::tc_fence_after();
+      const uint32_t zs = s_z + (uint32_t)zb * L.zbytes;
+      const int64_t grow = (int64_t)tile * kBM + r;
+      const bool live = grow < a.n;
+      const uint32_t tacc = tmem + lane_base + (uint32_t)buf * kAccStride;
+      Pass1 mine{-INFINITY, -INFINITY, 0.f, 0.f};
+      if (ok) {
+        // two of the four k-ordered partial sums of ||z||^2 (quarters 2 half,
+        // 2 half + 1 of the features; the FP32 kernels form the same chains)
+        float pc[2];
+#pragma unroll
+        for (int j = 0; j < 2; ++j) {
+          const int q = 2 * half + j;
+          float p = 0.f;
+          for (int k = q * dq; k < (q + 1) * dq; k += 4) {
+            const float4 v = lds_f4(zs + sw_off(r, k, kZChunkBytes));
+            p = fmaf(v.x, v.x, p);
+            p = fmaf(v.y, v.y, p);
+            p = fmaf(v.z, v.z, p);
+            p = fmaf(v.w, v.w, p);
+          }
+          pc[j] = p;
+        }
+        mine.psum = pc[0] + pc[1];
+        // pass 1: top two s~ of this half's columns (two chunks per TMEM wait)
+        float t1[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY}, t2[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+        for (int ch = half; ch < nck; ch += 4) {
+          uint32_t va[32], vb[32];
+          const bool two = ch + 2 < nck;
+          ptx::tmem_ld32(tacc + (uint32_t)(ch * 32), va);
+          if (two) ptx::tmem_ld32(tacc + (uint32_t)((ch + 2) * 32), vb);
+          ptx::tmem_wait_ld();
+          pass1_chunk(va, ch, t1, t2);
+          if (two) pass1_chunk(vb, ch + 2, t1, t2);
+        }
+        float l1 = t1[0], l2 = t2[0];
+#pragma unroll
+        for (int e = 1; e < 4; ++e) {
+          l2 = fmaxf(fmaxf(l2, t2[e]), fminf(l1, t1[e]));
+          l1 = fmaxf(l1, t1[e]);
+        }
+        mine.l1 = l1;
+        mine.l2 = l2;
+      }
+      x1[half * kBM + r] = mine;
+      if (lane == 0) okf[half * 4 + quarter] = ok ? 1 : 0;
+      pair_barrier(bar_id);
+      const Pass1 o = x1[(half ^ 1) * kBM + r];
+      if (!ok || okf[(half ^ 1) * 4 + quarter] == 0) break;  // both warps of the pair leave together
+      const float L2 = fmaxf(fmaxf(mine.l2, o.l2), fminf(mine.l1, o.l1));
+      const float kn = __fadd_rn(mine.psum, o.psum);  // (q0 + q1) + (q2 + q3)
+      const float hn = norm_upper(kn);
+      // |s~_c| <= Mb, so every screen value and partial sum is finite when
+      // Mb is; E covers the MMA error and the rounding of the bias addition
+      const float Mb = __fmaf_ru(cw1, hn, bmax);
+      const float E = __fmaf_ru(cw, hn, __fmaf_ru(Mb, 2.3841858e-07f /* 2^-22 */, kTinyF));
+      const float T = __fsub_rd(L2, __fmul_ru(2.f, E));
+      bool fb = live && !(Mb < 1e38f);  // NaN / infinite features, or a bound near FP32 overflow
+
+      // pass 2: the candidates of this half's columns into the warp's list;
+      // the row's lane keeps its slots' classes (one byte each)
+      int P = 0, cnt = 0;
+      uint32_t cls_lo = 0, cls_hi = 0;
+      auto append = [&](uint32_t mask, int ch) {
+        if (!live || fb) mask = 0;
+        while (__any_sync(kFull, mask != 0)) {
+          const bool has = mask != 0;
+          const int jb = __ffs((int)mask) - 1;
+          mask &= mask - 1;
+          const bool take = has && cnt < kMaxCandTc;
+          const unsigned mb = __ballot_sync(kFull, take);
+          if (take) {
+            const int c = ch * 32 + jb;
+            list[P + __popc(mb & ((1u << lane) - 1u))] = lane | (cnt << 5) | (c << 8);
+            if (cnt < 4)
+              cls_lo |= (uint32_t)c << (8 * cnt);
+            else
+              cls_hi |= (uint32_t)c << (8 * (cnt - 4));
+          }
+          cnt += has ? 1 : 0;
+          P += __popc(mb);
+        }
+      };
+      for (int ch = half; ch < nck; ch += 4) {
+        uint32_t va[32], vb[32];
+        const bool two = ch + 2 < nck;
+        ptx::tmem_ld32(tacc + (uint32_t)(ch * 32), va);
+        if (two) ptx::tmem_ld32(tacc + (uint32_t)((ch + 2) * 32), vb);
+        ptx::tmem_wait_ld();
+        const uint32_t ma = pass2_chunk(va, ch, T);
+        const uint32_t mbk = two ? pass2_chunk(vb, ch + 2, T) : 0u;
+        append(ma, ch);
+        if (two) append(mbk, ch + 2);
+      }
+      fb = fb || cnt > kMaxCandTc;
+      ptx::tc_fence_before();
+      __syncwarp();
+      if (lane == 0) ptx::mbar_arrive(accempty + 8 * buf);  // the accumulator is free for tile t + 2
+
+      // refinement: the four groups take eight pairs of the list at a time
+      // (balanced over the warp) and store hi / lo at the pair's (row, slot)
+      const int rq = quarter * 32;  // first row of the warp
+      for (int p0 = 0; p0 < P; p0 += 2 * (32 / kGroupTc)) {
+        const int i0 = p0 + 2 * g8, i1 = i0 + 1;
+        const int e0 = list[i0 < P ? i0 : p0], e1 = list[i1 < P ? i1 : p0];
+        const int cp[2] = {e0 >> 8, e1 >> 8};
+        const int rp[2] = {rq + (e0 & 31), rq + (e1 & 31)};
+        const float bp[2] = {bias_s[cp[0]], bias_s[cp[1]]};
+        float hi[2], lo[2];
+        refine2(s_w, wchunk, zs, cp, rp, bp, d, sub, hi, lo);
+        if (sub == 0) {
+          if (i0 < P) {
+            res_hi[(e0 & 0xff)] = hi[0];  // (row lane, slot) = e & 0xff: lane + 32 slot
+            res_lo[(e0 & 0xff)] = lo[0];
+          }
+          if (i1 < P) {
+            res_hi[(e1 & 0xff)] = hi[1];
+            res_lo[(e1 & 0xff)] = lo[1];
+          }
+        }
+      }
+      __syncwarp();
+      // each row's lane pushes its own candidates into its running selection
+      Top2 tp;
+      if (!fb) {
+        const int ns = cnt < kMaxCandTc ? cnt : kMaxCandTc;
+        for (int sl = 0; sl < ns; ++sl) {
+          const int c = (int)(((sl < 4 ? cls_lo >> (8 * sl) : cls_hi >> (8 * (sl - 4)))) & 0xffu);
+          tp.push(c, res_hi[lane + 32 * sl], res_lo[lane + 32 * sl], refined_err(a.g2f, wn_s[c], hn, bias_s[c]));
+        }
+      }
+      // rows that need every class of this half refined, one row at a time,
+      // eight classes a round through the row's result cells
+      const unsigned fbm = __ballot_sync(kFull, fb);
+      if (lane == 0) {
+        n_full += (unsigned long long)__popc(fbm);
+        n_pairs += (unsigned long long)P + (unsigned long long)__popc(fbm) * (unsigned long long)ncls;
+      }
+      for (unsigned fr = fbm; fr != 0; fr &= fr - 1) {
+        const int ow = __ffs((int)fr) - 1;
+        if (lane == ow) tp = Top2();
+        for (int t2 = 0; t2 < ncls; t2 += 2 * (32 / kGroupTc)) {
+          int tq[2] = {t2 + 2 * g8, t2 + 2 * g8 + 1};
+          int cp[2];
+#pragma unroll
+          for (int u = 0; u < 2; ++u) {
+            const int tt = tq[u] < ncls ? tq[u] : t2;
+            cp[u] = (2 * (tt >> 5) + half) * 32 + (tt & 31);
+          }
+          const int rp[2] = {rq + ow, rq + ow};
+          const float bp[2] = {bias_s[cp[0]], bias_s[cp[1]]};
+          float hi[2], lo[2];
+          refine2(s_w, wchunk, zs, cp, rp, bp, d, sub, hi, lo);
+          if (sub == 0) {
+#pragma unroll
+            for (int u = 0; u < 2; ++u) {
+              res_hi[ow + 32 * (2 * g8 + u)] = hi[u];
+              res_lo[ow + 32 * (2 * g8 + u)] = lo[u];
+            }
+          }
+          __syncwarp();
+          if (lane == ow)
+            for (int u = 0; u < 2 * (32 / kGroupTc) && t2 + u < ncls; ++u) {
+              const int tt = t2 + u;
+              const int c = (2 * (tt >> 5) + half) * 32 + (tt & 31);
+              tp.push(c, res_hi[ow + 32 * u], res_lo[ow + 32 * u], refined_err(a.g2f, wn_s[c], hn, bias_s[c]));
+            }
+          __syncwarp();
+        }
+      }
+      __syncwarp();
+      if (lane == 0) ptx::mbar_arrive(zempty + 8 * zb);  // this warp is done with the tile's features
+
+      // merge the halves; FP64 finals and the row's rank in its 32-row block
+      if (half == 1) x2[r] = tp;
+      pair_barrier(bar_id);
+      if (half == 0) {
+        top2_merge(tp, x2[r]);
+        if (live)
+          row_finals(a, grow, tp.result(kn), &acc_s[r]);
+        else
+          acc_s[r] = 0;
+        const unsigned mb = __ballot_sync(kFull, live && acc_s[r] != 0);
+        if (live) a.rank[grow] = __popc(mb & ((1u << lane) - 1u));
+        const int64_t blk0 = (int64_t)tile * kBM + quarter * 32;
+        if (lane == 0 && blk0 < a.n) a.bcount[blk0 / 32] = __popc(mb);
+      }
+    }
+    if (lane == 0 && (n_pairs | n_full)) {
+      atomicAdd(&stats->ins_pairs, n_pairs);
+      atomicAdd(&stats->ins_full_rows, n_full);
+    }
+  }
+  ptx::tc_fence_before();
+  __syncthreads();
+  if (threadIdx.x == 0 && *abort_s) {
+    atomicAdd(&stats->errors, 1ull);
+    atomicExch(&stats->abort_flag, 1);
+  }
+  if (warp == 1) {
+    ptx::tc_fence_after();
+    ptx::tmem_dealloc(tmem, kTmemCols);
+  }
+}
+
+void encode_rows(lipcache* h, CUtensorMap* map, const float* base, uint64_t rows, uint32_t box_rows) {
+  LC_REQUIRE(h->encode != nullptr, LIPCACHE_E_CUDA, "cuTensorMapEncodeTiled is unavailable from the driver");
+  const cuuint64_t dims[2] = {(cuuint64_t)h->d, (cuuint64_t)rows};
+  const cuuint64_t strides[1] = {(cuuint64_t)h->d * sizeof(float)};
+  const cuuint32_t box[2] = {(cuuint32_t)kChunkF, box_rows};
+  const cuuint32_t estr[2] = {1, 1};
+  const CUresult r = h->encode(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<float*>(base), dims, strides, box,
+                               estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  LC_REQUIRE(r == CUDA_SUCCESS, LIPCACHE_E_CUDA, "cuTensorMapEncodeTiled failed: " + std::to_string((int)r));
+}
+
+// Two feature buffers when they fit next to the resident head, else one.
+bool tc_plan(int d, int C, TcLayout& L) {
+  for (int nzb = 2; nzb >= 1; --nzb) {
+    L = tc_layout(d, C, nzb);
+    if (L.total <= (uint32_t)kSmemBudget) return true;
+  }
+  return false;
+}
+
+}  // namespace
+
+bool certify_tc_supported(const lipcache* h, const float* H, int64_t n) {
+  if (h->radius_mode == LIPCACHE_RADIUS_TIGHT || h->encode == nullptr) return false;
+  if (h->debug_flags & (LIPCACHE_DEBUG_INSERT_TILE64 | LIPCACHE_DEBUG_INSERT_WIDE_TILE)) return false;
+  // TMA: 16-byte aligned rows of d floats, 32-feature boxes (at most
+  // kMaxChunks of them); MMA: N <= 256
+  if (h->d < kChunkF || h->d > kChunkF * kMaxChunks || h->d % 16 != 0 || ((uintptr_t)H & 15) != 0) return false;
+  if (h->C < 2 || h->C > 256 || n <= 0 || n > ((int64_t)1 << 30)) return false;
+  TcLayout L;
+  return tc_plan(h->d, h->C, L);
+}
+
+void certify_tc_launch(lipcache* h, const CertArgs& a, cudaStream_t s) {
+  TcLayout L;
+  LC_REQUIRE(tc_plan(h->d, h->C, L), LIPCACHE_E_INVALID, "head does not fit the tensor certify kernel");
+  CUtensorMap tmH, tmW;
+  encode_rows(h, &tmH, a.H, (uint64_t)a.n, kBM);
+  encode_rows(h, &tmW, h->W, (uint64_t)h->C, (uint32_t)L.Cpad);
+  const int n_tiles = (int)((a.n + kBM - 1) / kBM);
+  const int grid = n_tiles < h->num_sms ? n_tiles : h->num_sms;
+  // at least half of the SM's shared memory, so one CTA (and one 512-column
+  // TMEM allocation) per SM
+  const int smem = (int)L.total + 1024 > 120 * 1024 ? (int)L.total + 1024 : 120 * 1024;
+  LC_CUDA(cudaFuncSetAttribute(k_certify_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
+  k_certify_tc<<<grid, kThreads, smem, s>>>(tmH, tmW, a, L, n_tiles, h->stats,
+                                            (h->debug_flags & LIPCACHE_DEBUG_STALL_INSERT) ? 1 : 0);
+  LC_LAUNCH_CHECK("k_certify_tc");
+}
+
+}  // namespace lc

@@ -115,6 +115,8 @@ struct DevStats {
   unsigned long long errors;
   int abort_flag;  // set by a kernel whose bounded wait expired; cleared per probe
   int pad;
+  unsigned long long ins_pairs;      // (row, class) pairs refined by the tensor certify kernel
+  unsigned long long ins_full_rows;  // row halves it refined over every class
 };
 
 // Scratch of the selection strategy (select.cu), grown on demand.
@@ -271,6 +273,11 @@ void set_radius_policy(lipcache* h, int policy, double param, double* rho_host, 
 // thresholds of entries [first, first + n) under the current policy
 void policy_fill(lipcache* h, int64_t first, int64_t n, cudaStream_t s);
 // certify.cu: certification of H into the insert scratch only (no append)
+// E_DEVICE (after synchronising `s`) if the last certification gave up on a
+// bounded wait; nothing was appended then.
+constexpr const char* kCertifyAbortMessage =
+    "a bounded wait of the tensor certify kernel expired; no row was certified or inserted";
+void require_certify_ok(lipcache* h, cudaStream_t s);
 void certify_rows(lipcache* h, const float* H, int64_t n, const int32_t* payload, int require_consistency,
                   cudaStream_t s);
 // select.cu: radius-prioritised de-duplication of the certified rows of H

@@ -419,6 +419,7 @@ int64_t select_insert(lipcache* h, const float* H, int64_t n, const int32_t* pay
                       cudaStream_t s) {
   SelectScratch& x = h->sel;
   certify_rows(h, H, n, payload, require_consistency, s);
+  require_certify_ok(h, s);
   const unsigned nb = (unsigned)((n + 255) / 256);
   if (out_index) {
     k_fill_i64<<<nb, 256, 0, s>>>(out_index, n, -1);
@@ -515,6 +516,7 @@ int64_t select_kcenter(lipcache* h, const float* H, int64_t n, const int32_t* pa
   SelectScratch& x = h->sel;
   const int C = h->C;
   certify_rows(h, H, n, payload, require_consistency, s);
+  require_certify_ok(h, s);
   const unsigned nb = (unsigned)((n + 255) / 256);
   if (out_index) {
     k_fill_i64<<<nb, 256, 0, s>>>(out_index, n, -1);

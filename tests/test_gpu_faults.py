@@ -1,7 +1,7 @@
-"""Failure detection on the GPU without a fault: a probe whose MMA issuer
-waits on a barrier nothing arrives on must give up after its bounded wait,
-report the batch as misses and an error, and leave the context usable
-(pytest -m gpu)."""
+"""Failure detection on the GPU without a fault: a probe or a tensor certify
+kernel whose MMA issuer waits on a barrier nothing arrives on must give up
+after its bounded wait, report an error (the probe's batch as misses, no
+inserted row), and leave the context usable (pytest -m gpu)."""
 import time
 
 import numpy as np
@@ -9,6 +9,7 @@ import pytest
 
 import oracle
 import synth
+from parity_utils import check_insert
 
 torch = pytest.importorskip("torch")
 pytestmark = pytest.mark.gpu
@@ -79,6 +80,33 @@ def test_debug_flags_validated(dev):
     from paper_2608_13144_gb300.lipcache import LipCache
     c = LipCache(4, 2, 8, device=dev)
     with pytest.raises(LipCacheError) as e:
-        c.set_debug(6)
+        c.set_debug(16)
     assert e.value.status == 1
+    c.set_debug(2 | 4 | 8)  # every known flag together is accepted
+    c.set_debug(0)
+    c.close()
+
+
+def test_certify_stall_aborts_cleanly(dev):
+    """A bounded wait of the tensor certify kernel that expires (a barrier
+    nothing arrives on) aborts the kernel: the insert returns E_DEVICE,
+    appends nothing and counts a device error; the next insert works and
+    matches the oracle."""
+    from paper_2608_13144_gb300._lib import LipCacheError
+    from paper_2608_13144_gb300.lipcache import LipCache
+    w = synth.WORKLOADS["cifar100"].scaled(N=2000)
+    W, b = synth.head(w)
+    rows = synth.cache_rows(w)
+    c = LipCache(w.d, w.C, 2 * len(rows), device=dev)
+    c.set_head(torch.from_numpy(W).to(dev), torch.from_numpy(b).to(dev))
+    c.set_debug(8)
+    with pytest.raises(LipCacheError) as e:
+        c.insert(torch.from_numpy(rows).to(dev))
+    assert e.value.status == 8 and c.size == 0  # LIPCACHE_E_DEVICE
+    assert c.info()["last_insert_kernel"] == 4 and c.info()["device_errors"] >= 1
+    c.set_debug(0)
+    idx, rad, n = c.insert(torch.from_numpy(rows).to(dev))
+    ref = oracle.build_cache(W, b, oracle.sigma_max(W), rows)
+    check_insert(idx.cpu().numpy(), rad.cpu().numpy(), n, ref, (W, b, rows, 1.0))
+    assert c.size == n
     c.close()

@@ -1,7 +1,11 @@
-"""The wide-tile certify kernel (128-row tiles, logits in registers) against
-the 64-row-tile kernel and the FP64 oracle (pytest -m gpu). Both form the same
-FP32 logit chains, candidate sets, compensated refinements and FP64 finals,
-so their outputs agree bit for bit; the oracle pins the values."""
+"""The certify kernels against each other and the FP64 oracle (pytest -m
+gpu). The wide-tile kernel (128-row tiles, logits in registers) and the
+64-row-tile kernel form the same FP32 logit chains, candidate sets,
+compensated refinements and FP64 finals, so their outputs agree bit for bit.
+The tensor kernel (TF32 tcgen05 screen) picks its candidates from wider
+intervals but refines them in the same order, so its radii, labels and
+entries agree bit for bit with the wide-tile kernel too; the oracle pins the
+values."""
 import numpy as np
 import pytest
 
@@ -12,8 +16,8 @@ from parity_utils import check_insert, refine_slack_tight
 torch = pytest.importorskip("torch")
 pytestmark = pytest.mark.gpu
 
-WIDE_TILE, TILE64, STREAMED = 1, 2, 3
-DEBUG_INSERT_TILE64 = 2
+WIDE_TILE, TILE64, STREAMED, TENSOR = 1, 2, 3, 4
+DEBUG_INSERT_TILE64, DEBUG_INSERT_WIDE_TILE = 2, 4
 
 
 @pytest.fixture(scope="module")
@@ -30,10 +34,14 @@ def T(x, dev):
 
 
 def build(dev, W, b, rows, batch, tile64, payload=None, consistency=False):
+    """tile64: True forces the 64-row-tile kernel, "wide" the wide-tile one,
+    False leaves the choice to the library."""
     from paper_2608_13144_gb300.lipcache import LipCache
     c = LipCache(W.shape[1], W.shape[0], len(rows), device=dev)
     c.set_head(T(W, dev), T(b, dev))
-    if tile64:
+    if tile64 == "wide":
+        c.set_debug(DEBUG_INSERT_WIDE_TILE)
+    elif tile64:
         c.set_debug(DEBUG_INSERT_TILE64)
     idx, rad, n = [], [], 0
     for s, e in synth.batches(len(rows), batch):
@@ -64,7 +72,7 @@ def test_wide_tile_bit_identical_and_oracle(dev, d, C, N, batch):
     W, b = synth.head(w)
     rows = synth.cache_rows(w)
     Q, _ = synth.queries(w, rows)
-    a, ia, ra, na = build(dev, W, b, rows, batch, False)
+    a, ia, ra, na = build(dev, W, b, rows, batch, "wide")
     assert a.info()["last_insert_kernel"] == WIDE_TILE
     s, is_, rs, ns = build(dev, W, b, rows, batch, True)
     assert s.info()["last_insert_kernel"] == TILE64
@@ -84,6 +92,78 @@ def test_wide_tile_bit_identical_and_oracle(dev, d, C, N, batch):
     s.close()
 
 
+# (d, C, rows, insert batch) for the tensor kernel: one and two feature
+# buffers, one and two column halves (C <= 32 and C > 32), C = 256 (N = 256,
+# eight column chunks), d % 32 == 16, ragged last tiles, fewer tiles than SMs,
+# batches smaller than one tile
+TC_SHAPES = [(32, 10, 3000, 3000), (64, 10, 20000, 20000), (128, 100, 30001, 30001), (128, 200, 40000, 16384),
+             (96, 250, 3000, 3000), (48, 3, 777, 100), (128, 200, 200, 64), (96, 256, 70000, 65536),
+             (32, 2, 500, 500)]
+
+
+@pytest.mark.parametrize("d,C,N,batch", TC_SHAPES)
+def test_tensor_bit_identical_and_oracle(dev, d, C, N, batch):
+    """The tensor kernel (TF32 screen into TMEM) against the wide-tile kernel:
+    every output and stored entry bit for bit, every probe result too (the
+    thresholds are not exported), and the oracle."""
+    w = synth.WORKLOADS["cifar100"].scaled(d=d, C=C, components=C, N=N, n_queries=512, sphere_radius=4.0)
+    W, b = synth.head(w)
+    rows = synth.cache_rows(w)
+    Q, _ = synth.queries(w, rows)
+    a, ia, ra, na = build(dev, W, b, rows, batch, False)
+    assert a.info()["last_insert_kernel"] == TENSOR
+    assert a.info()["device_errors"] == 0
+    ref = oracle.build_cache(W, b, oracle.sigma_max(W), rows)
+    check_insert(ia, ra, na, ref, (W, b, rows, 1.0))
+    s, is_, rs, ns = build(dev, W, b, rows, batch, "wide")
+    if s.info()["last_insert_kernel"] == STREAMED:
+        # too large for the wide-tile kernel: the streamed kernel refines with
+        # 32 lanes, so only acceptance, indices and y^G agree bit for bit
+        assert na == ns and np.array_equal(ia, is_)
+        np.testing.assert_array_equal(a.entries()["yG"], s.entries()["yG"])
+        a.close()
+        s.close()
+        return
+    assert s.info()["last_insert_kernel"] == WIDE_TILE
+    assert na == ns and same_bits(ia, is_) and same_bits(ra, rs)
+    ea, es = a.entries(), s.entries()
+    for k in ("keys", "radius", "label", "yG"):
+        assert same_bits(ea[k], es[k]), k
+    for path in ("exact", "tensor"):
+        a.set_probe_path(path)
+        s.set_probe_path(path)
+        for x, y in zip(a.probe(T(Q, dev)), s.probe(T(Q, dev))):
+            assert same_bits(x.cpu().numpy(), y.cpu().numpy()), path
+    a.close()
+    s.close()
+
+
+def test_tensor_overflow_rows(dev):
+    """19 identical head rows: rows whose top two lie in the tied group have
+    more candidates than the per-row slots, so the tensor kernel refines
+    every class of the row (in the 8-lane order) and the wide-tile kernel its
+    one-warp path (32 lanes). Acceptance and indices agree; radii agree with
+    the oracle within the refinement bound."""
+    rng = np.random.default_rng(21)
+    d, C = 32, 24
+    W = (rng.standard_normal((C, d)) / np.sqrt(d)).astype(np.float32)
+    W[1:20] = W[1]
+    b = (0.1 * rng.standard_normal(C)).astype(np.float32)
+    b[1:20] = b[1]
+    rows = np.concatenate([3 * W[0] + 0.3 * rng.standard_normal((700, d)),
+                           3 * W[1] + 0.3 * rng.standard_normal((700, d)),
+                           rng.standard_normal((600, d))]).astype(np.float32)
+    a, ia, ra, na = build(dev, W, b, rows, len(rows), False)
+    s, is_, rs, ns = build(dev, W, b, rows, len(rows), "wide")
+    assert a.info()["last_insert_kernel"] == TENSOR and s.info()["last_insert_kernel"] == WIDE_TILE
+    assert na == ns and np.array_equal(ia, is_)
+    np.testing.assert_array_equal(a.entries()["yG"], s.entries()["yG"])
+    ref = oracle.build_cache(W, b, oracle.sigma_max(W), rows)
+    check_insert(ia, ra, na, ref, (W, b, rows, 1.0))
+    a.close()
+    s.close()
+
+
 def test_wide_tile_overflow_rows(dev):
     """More candidate classes per row than the per-row slots (19 identical
     head rows): the kernel recomputes those rows' logits and hands them to the
@@ -97,7 +177,7 @@ def test_wide_tile_overflow_rows(dev):
     rows = np.concatenate([3 * W[0] + 0.3 * rng.standard_normal((700, d)),
                            3 * W[1] + 0.3 * rng.standard_normal((700, d)),
                            rng.standard_normal((600, d))]).astype(np.float32)
-    a, ia, ra, na = build(dev, W, b, rows, len(rows), False)
+    a, ia, ra, na = build(dev, W, b, rows, len(rows), "wide")
     s, is_, rs, ns = build(dev, W, b, rows, len(rows), True)
     assert a.info()["last_insert_kernel"] == WIDE_TILE
     assert na == ns and same_bits(ia, is_) and same_bits(ra, rs)
@@ -107,13 +187,16 @@ def test_wide_tile_overflow_rows(dev):
     s.close()
 
 
-def test_wide_tile_payload_and_consistency(dev):
-    """Payload labels and the consistency flag go through the same finals."""
+@pytest.mark.parametrize("kernel", ["wide", False])
+def test_wide_tile_payload_and_consistency(dev, kernel):
+    """Payload labels and the consistency flag go through the same finals
+    (wide-tile and tensor kernels against the 64-row-tile kernel)."""
     w = synth.WORKLOADS["cifar10"].scaled(N=6000)
     W, b = synth.head(w)
     rows = synth.cache_rows(w)
     payload = (np.arange(len(rows)) % w.C).astype(np.int32)
-    a, ia, ra, na = build(dev, W, b, rows, 4096, False, payload, True)
+    a, ia, ra, na = build(dev, W, b, rows, 4096, kernel, payload, True)
+    assert a.info()["last_insert_kernel"] == (WIDE_TILE if kernel else TENSOR)
     s, is_, rs, ns = build(dev, W, b, rows, 4096, True, payload, True)
     assert na == ns and same_bits(ia, is_) and same_bits(ra, rs)
     ref = oracle.build_cache(W, b, oracle.sigma_max(W), rows, payload=payload, require_consistency=True)
@@ -123,11 +206,17 @@ def test_wide_tile_payload_and_consistency(dev):
 
 
 def test_kernel_choice(dev):
-    """Shapes outside the wide-tile kernel's limits take the other
-    kernels: d % 4 != 0, and heads too large for shared memory."""
+    """The conservative radius takes the tensor kernel where it applies
+    (d % 16 == 0, d >= 32, 2 <= C <= 256, head resident); the other shapes
+    and the tight radius take the wide-tile kernel (d % 4 == 0, head small
+    enough), the 64-row one (d % 4 != 0) or the streamed one (large heads)."""
     from paper_2608_13144_gb300.lipcache import LipCache
     cases = [((64, 10), "tight", WIDE_TILE), ((33, 10), "tight", TILE64), ((33, 10), "conservative", TILE64),
-             ((256, 200), "conservative", STREAMED), ((128, 300), "conservative", STREAMED)]
+             ((256, 200), "conservative", STREAMED), ((128, 300), "conservative", STREAMED),
+             ((128, 200), "conservative", TENSOR), ((64, 10), "conservative", TENSOR),
+             ((32, 2), "conservative", TENSOR), ((16, 10), "conservative", WIDE_TILE),
+             ((40, 10), "conservative", WIDE_TILE), ((128, 200), "tight", WIDE_TILE),
+             ((96, 256), "conservative", TENSOR), ((128, 256), "conservative", STREAMED)]
     rng = np.random.default_rng(5)
     for (d, C), mode, kernel in cases:
         W = (rng.standard_normal((C, d)) / np.sqrt(d)).astype(np.float32)
@@ -158,8 +247,9 @@ def _near_ties(W, b, n, rng, k):
     return np.asarray(out, dtype=np.float32)
 
 
+@pytest.mark.parametrize("kernel", ["wide", False])
 @pytest.mark.parametrize("d,C", [(16, 10), (64, 40), (128, 100), (128, 200), (96, 250)])
-def test_wide_tile_near_ties(dev, d, C):
+def test_wide_tile_near_ties(dev, d, C, kernel):
     """Rows on two- and three-way logit ties: several candidate classes per
     row, refinement deciding the order, margins near zero (some rows
     rejected). Bit-identical to the 64-row-tile kernel and within the
@@ -169,9 +259,9 @@ def test_wide_tile_near_ties(dev, d, C):
     b = (0.1 * rng.standard_normal(C)).astype(np.float32)
     rows = np.concatenate([_near_ties(W, b, 600, rng, 2), _near_ties(W, b, 600, rng, 3),
                            rng.standard_normal((400, d)).astype(np.float32)])
-    a, ia, ra, na = build(dev, W, b, rows, len(rows), False)
+    a, ia, ra, na = build(dev, W, b, rows, len(rows), kernel)
     s, is_, rs, ns = build(dev, W, b, rows, len(rows), True)
-    assert a.info()["last_insert_kernel"] == WIDE_TILE
+    assert a.info()["last_insert_kernel"] == (TENSOR if not kernel and d >= 32 else WIDE_TILE)
     assert na == ns and same_bits(ia, is_) and same_bits(ra, rs)
     ref = oracle.build_cache(W, b, oracle.sigma_max(W), rows)
     check_insert(ia, ra, na, ref, (W, b, rows, 1.0))
@@ -282,7 +372,7 @@ def test_certify_special_values(dev, mode, d, C):
     c.set_head(T(W, dev), T(b, dev))
     i, r, n = c.insert(T(rows, dev))
     i, r = i.cpu().numpy(), r.cpu().numpy()
-    assert c.info()["last_insert_kernel"] == WIDE_TILE
+    assert c.info()["last_insert_kernel"] == (TENSOR if mode == "conservative" and d >= 32 else WIDE_TILE)
     ref = oracle.build_cache(W, b, oracle.sigma_max(W), rows, radius_mode=int(mode == "tight"))
     head = ("tight", W, b, rows, 1.0) if mode == "tight" else (W, b, rows, 1.0)
     finite = np.all(np.isfinite(rows), axis=1)
