@@ -99,6 +99,26 @@ TcLayout tc_layout(int d, int C, int nzb) {
   return L;
 }
 
+// Packed FP32 pairs: two additions / multiplications in one instruction (each
+// lane rounded to nearest, as the scalar operation), and packing.
+__device__ __forceinline__ uint64_t add_f32x2(uint64_t a, uint64_t b) {
+  uint64_t r;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+  return r;
+}
+__device__ __forceinline__ uint64_t mul_f32x2(uint64_t a, uint64_t b) {
+  uint64_t r;
+  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+  return r;
+}
+__device__ __forceinline__ uint64_t pack2_f32(float lo, float hi) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+  return r;
+}
+__device__ __forceinline__ void unpack2_f32(uint64_t v, float& lo, float& hi) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
 // Byte offset of feature k of row r in a 128-byte-swizzled K-major tile whose
 // 32-feature chunks are `chunk_bytes` apart (TMA SWIZZLE_128B: the 16-byte
 // unit index is XORed with the row index mod 8).
@@ -179,14 +199,14 @@ __device__ __forceinline__ void refine2(uint32_t ws, uint32_t wchunk, uint32_t z
     asm volatile("ld.shared.f32 %0, [%1];" : "=f"(x0) : "r"(za0));
     asm volatile("ld.shared.f32 %0, [%1];" : "=f"(w1) : "r"(wa1));
     asm volatile("ld.shared.f32 %0, [%1];" : "=f"(x1) : "r"(za1));
-    const uint64_t w = ptx::pack2_f32(w0, w1), x = ptx::pack2_f32(x0, x1);
-    const uint64_t pr = ptx::mul_f32x2(w, x);                // TwoProduct: pr + er = w x
+    const uint64_t w = pack2_f32(w0, w1), x = pack2_f32(x0, x1);
+    const uint64_t pr = mul_f32x2(w, x);                // TwoProduct: pr + er = w x
     const uint64_t er = ptx::fma_f32x2(w, x, pr ^ kSign2);
-    const uint64_t sm = ptx::add_f32x2(P, pr);               // TwoSum(P, pr) = sm + q
+    const uint64_t sm = add_f32x2(P, pr);               // TwoSum(P, pr) = sm + q
     const uint64_t bb = ptx::sub_f32x2(sm, P);
-    const uint64_t q = ptx::add_f32x2(ptx::sub_f32x2(P, ptx::sub_f32x2(sm, bb)), ptx::sub_f32x2(pr, bb));
+    const uint64_t q = add_f32x2(ptx::sub_f32x2(P, ptx::sub_f32x2(sm, bb)), ptx::sub_f32x2(pr, bb));
     P = sm;
-    CC = ptx::add_f32x2(CC, ptx::add_f32x2(q, er));
+    CC = add_f32x2(CC, add_f32x2(q, er));
   };
   const int nfull = d >> 5;
   for (int kc = 0; kc < nfull; ++kc) {
@@ -203,8 +223,8 @@ __device__ __forceinline__ void refine2(uint32_t ws, uint32_t wchunk, uint32_t z
     for (int jj = 0; jj < 2; ++jj) step(wb[0] + ow[0][jj], zb[0] + oz[0][jj], wb[1] + ow[1][jj], zb[1] + oz[1][jj]);
   }
   float p[2], cc[2];
-  ptx::unpack2_f32(P, p[0], p[1]);
-  ptx::unpack2_f32(CC, cc[0], cc[1]);
+  unpack2_f32(P, p[0], p[1]);
+  unpack2_f32(CC, cc[0], cc[1]);
 #pragma unroll
   for (int o = kGroupTc / 2; o > 0; o >>= 1) {
 #pragma unroll
