@@ -59,9 +59,10 @@ typedef enum lipcache_status {
 #define LIPCACHE_RADIUS_TIGHT 1        /* r* = min_j (s_y - s_j) / ||W_y - W_j||, Eq. 29 */
 
 /* Certify kernels (lipcache_info.last_insert_kernel).
- * TENSOR: TF32 tcgen05 screen of the logits into tensor memory, conservative
- *   radius only (d % 16 == 0, d >= 32, 2 <= C <= 256, head resident in shared
- *   memory); it refines and finishes rows exactly as WIDE_TILE.
+ * TENSOR: TF32 tcgen05 screen of the logits into tensor memory, both radii
+ *   (d % 16 == 0, 32 <= d <= 256, 2 <= C <= 256, head resident in shared
+ *   memory); it refines and finishes rows as WIDE_TILE does (conservative
+ *   radius: the same bits; tight radius: within the refinement bound).
  * WIDE_TILE: head resident in shared memory, 128-row tiles, logits in
  *   registers (d % 4 == 0, head small enough; both radii, the tight one
  *   refining only the classes that can be its minimiser).
@@ -70,7 +71,7 @@ typedef enum lipcache_status {
  * For the conservative radius TENSOR, WIDE_TILE and TILE64 give the same bits;
  * STREAMED refines with a 32-lane compensated sum, so its radii agree with
  * theirs within the refinement bound. For the tight radius TILE64 and
- * STREAMED refine every class in FP64 and agree with WIDE_TILE within the
+ * STREAMED refine every class in FP64, and all kernels agree within the
  * refinement bound. */
 #define LIPCACHE_INSERT_WIDE_TILE 1
 #define LIPCACHE_INSERT_TILE64 2
@@ -362,7 +363,7 @@ lipcache_status lipcache_read_head(lipcache_t* h, float* W_host, float* b_host, 
  * would run; both compute the same values, so tests compare them bit for bit. */
 #define LIPCACHE_DEBUG_INSERT_TILE64 2
 /* Certify with the wide-tile kernel where the tensor one would run (tests
- * compare the two bit for bit). */
+ * compare the two). */
 #define LIPCACHE_DEBUG_INSERT_WIDE_TILE 4
 /* The MMA issuer of the tensor certify kernel first waits on an mbarrier that
  * nothing arrives on: the bounded wait expires, the kernel aborts, no row is

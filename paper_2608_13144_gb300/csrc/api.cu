@@ -73,6 +73,8 @@ void release(lipcache* h) {
   dev_free(h->inv_pairnorm);
   dev_free(h->ipn_up32);
   dev_free(h->ipn_dn32);
+  dev_free(h->ipn_min32);
+  dev_free(h->ipn_max32);
   dev_free(h->gram[0]);
   dev_free(h->gram[1]);
   dev_free(h->spec);
@@ -198,6 +200,8 @@ LC_API lipcache_status lipcache_create(int32_t d, int32_t C, int64_t capacity, i
       dev_alloc(h->inv_pairnorm, (size_t)C * C);
       dev_alloc(h->ipn_up32, (size_t)C * C);
       dev_alloc(h->ipn_dn32, (size_t)C * C);
+      dev_alloc(h->ipn_min32, (size_t)C);
+      dev_alloc(h->ipn_max32, (size_t)C);
     }
     dev_alloc(h->gram[0], (size_t)d * d);
     dev_alloc(h->gram[1], (size_t)d * d);

@@ -735,7 +735,6 @@ __device__ __forceinline__ unsigned tight_candidates(const CertArgs& a, const fl
 // the probe thresholds; the skip rules of Algorithm 1.
 __device__ void row_finals_tight(const CertArgs& a, int64_t row, int y, int n, const uint8_t* cls, const float* rh,
                                  const float* rl, const float* re, float kn, uint8_t* acc_slot) {
-  const int C = a.C;
   double vy = NAN, ey = 0.0;
   for (int sl = 0; sl < n; ++sl)
     if (cls[sl] == y) {
@@ -747,29 +746,11 @@ __device__ void row_finals_tight(const CertArgs& a, int64_t row, int y, int n, c
   for (int sl = 0; sl < n; ++sl) {
     const int j = cls[sl];
     if (j == y) continue;
-    const double vj = (double)rh[sl] + (double)rl[sl], ej = (double)re[sl];
+    const double vj = (double)rh[sl] + (double)rl[sl];
     if (!(vj == vj)) any_nan = true;
-    const double pn = a.pairnorm[(size_t)y * C + j];
-    if (!(pn > 0.0)) continue;
-    const double ipn = a.inv_pairnorm[(size_t)y * C + j];
-    rmin = fmin(rmin, (vy - vj) * ipn);
-    const double num = __dsub_rd(__dsub_rd(vy, ey), __dadd_ru(vj, ej));
-    smin = fmin(smin, __dmul_rd(__dmul_rd(num, ipn), a.tight_f));
+    tight_term(a, y, j, vy, ey, vj, (double)re[sl], rmin, smin);
   }
-  const double r64 = any_nan ? NAN : a.kappa * rmin;
-  const double rs = (smin > 0.0 && !any_nan) ? __dmul_rd(a.kappa, smin) : 0.0;
-  const int32_t lab = a.payload ? a.payload[row] : y;
-  const bool acc = !(a.require_consistency && lab != y) && (r64 > 0.0) && !(a.miss_of && a.miss_of[row] >= 0);
-  float rr, tau;
-  thresholds(__double2float_rd(rs), kn, a.tc, rr, tau);
-  a.accept[row] = acc ? 1 : 0;
-  a.yG[row] = y;
-  a.label[row] = lab;
-  a.radius[row] = __double2float_rz(r64);
-  a.rr[row] = rr;
-  a.kn[row] = kn;
-  a.tau[row] = tau;
-  *acc_slot = acc ? 1 : 0;
+  tight_write(a, row, y, rmin, smin, any_nan, kn, acc_slot);
 }
 
 // One row of the tight radius on one warp, for rows the FP32 intervals cannot
@@ -852,32 +833,11 @@ __device__ void wt_tight_row_warp(const CertArgs& a, int64_t row, int r, const f
   for (int t = 0; t < kPer; ++t) {
     const int j = lane + 32 * t;
     if (j >= C || j == y) continue;
-    const double pn = a.pairnorm[(size_t)y * C + j];
-    if (!(pn > 0.0)) continue;
-    const double ipn = a.inv_pairnorm[(size_t)y * C + j];
-    const double vj = (double)vh[t] + (double)vl[t], ej = (double)ve[t];
-    rmin = fmin(rmin, (vy - vj) * ipn);
-    const double num = __dsub_rd(__dsub_rd(vy, ey), __dadd_ru(vj, ej));
-    smin = fmin(smin, __dmul_rd(__dmul_rd(num, ipn), a.tight_f));
+    tight_term(a, y, j, vy, ey, (double)vh[t] + (double)vl[t], (double)ve[t], rmin, smin);
   }
   rmin = warp_min_d(rmin);
   smin = warp_min_d(smin);
-  if (lane == 0) {
-    const double r64 = nan_any ? NAN : a.kappa * rmin;
-    const double rs = (smin > 0.0 && !nan_any) ? __dmul_rd(a.kappa, smin) : 0.0;
-    const int32_t lab = a.payload ? a.payload[row] : y;
-    const bool acc = !(a.require_consistency && lab != y) && (r64 > 0.0) && !(a.miss_of && a.miss_of[row] >= 0);
-    float rr, tau;
-    thresholds(__double2float_rd(rs), kn, a.tc, rr, tau);
-    a.accept[row] = acc ? 1 : 0;
-    a.yG[row] = y;
-    a.label[row] = lab;
-    a.radius[row] = __double2float_rz(r64);
-    a.rr[row] = rr;
-    a.kn[row] = kn;
-    a.tau[row] = tau;
-    *acc_slot = acc ? 1 : 0;
-  }
+  if (lane == 0) tight_write(a, row, y, rmin, smin, nan_any, kn, acc_slot);
   __syncwarp();
 }
 
@@ -1538,6 +1498,8 @@ void launch_certify(lipcache* h, const float* H, int64_t n, const int32_t* paylo
   a.inv_pairnorm = h->inv_pairnorm;
   a.ipn_up32 = h->ipn_up32;
   a.ipn_dn32 = h->ipn_dn32;
+  a.ipn_min32 = h->ipn_min32;
+  a.ipn_max32 = h->ipn_max32;
   a.tight_f = 1.0 - gamma64(h->d + 8);
   a.inv_denom = h->radius_scale / (h->sigma * 1.4142135623730951);
   a.inv_denom_safe = h->radius_scale * (1.0 - 8 * kU64) / (h->sigma * (1.0 + kSigmaSlack) * 1.4142135623730951);

@@ -27,6 +27,8 @@ struct CertArgs {
   const double* inv_pairnorm;  // 1 / ||W_y - W_j|| (tight mode)
   const float* ipn_up32;       // FP32 brackets of 1 / ||W_y - W_j|| (tight mode; +inf where the rows coincide)
   const float* ipn_dn32;
+  const float* ipn_min32;      // per class: a lower bound of every 1 / ||W_y - W_j|| (tight mode)
+  const float* ipn_max32;      // per class: an upper bound of every 1 / ||W_y - W_j|| (tight mode)
   double tight_f;              // 1 - gamma_{d+8} (FP64)
   uint8_t* accept;
   int32_t* yG;
@@ -40,7 +42,7 @@ struct CertArgs {
 };
 
 // The tensor-core certify kernel (certify_tc.cu): whether it takes this
-// insert (conservative radius, d % 16 == 0, d >= 32, 2 <= C <= 256, rows
+// insert (either radius, d % 16 == 0, 32 <= d <= 256, 2 <= C <= 256, rows
 // 16-byte aligned, head resident in shared memory), and its launch.
 bool certify_tc_supported(const lipcache* h, const float* H, int64_t n);
 void certify_tc_launch(lipcache* h, const CertArgs& a, cudaStream_t s);
@@ -229,6 +231,40 @@ __device__ void row_finals(const CertArgs& a, int64_t row, const RowVals& v, uin
   a.radius[row] = __double2float_rz(r64);
   a.rr[row] = rr;
   a.kn[row] = v.kn;
+  a.tau[row] = tau;
+  *acc_slot = acc ? 1 : 0;
+}
+
+// One term of Eq. 29 for the refined logits vy (error ey) of y^G and vj (ej)
+// of a class j: the radius candidate (s_y - s_j) / ||W_y - W_j|| and its
+// certified lower bound (rounded downwards, 1 - gamma_{d+8} for the FP64
+// reciprocal), folded into running minima. Pairs with W_j = W_y are skipped.
+__device__ __forceinline__ void tight_term(const CertArgs& a, int y, int j, double vy, double ey, double vj, double ej,
+                                           double& rmin, double& smin) {
+  const double pn = a.pairnorm[(size_t)y * a.C + j];
+  if (!(pn > 0.0)) return;
+  const double ipn = a.inv_pairnorm[(size_t)y * a.C + j];
+  rmin = fmin(rmin, (vy - vj) * ipn);
+  const double num = __dsub_rd(__dsub_rd(vy, ey), __dadd_ru(vj, ej));
+  smin = fmin(smin, __dmul_rd(__dmul_rd(num, ipn), a.tight_f));
+}
+
+// The tight radius r* = kappa rmin (Eq. 29), its certified lower bound, the
+// probe thresholds and the skip rules of Algorithm 1 for one row (one thread).
+__device__ void tight_write(const CertArgs& a, int64_t row, int y, double rmin, double smin, bool any_nan, float kn,
+                            uint8_t* acc_slot) {
+  const double r64 = any_nan ? NAN : a.kappa * rmin;
+  const double rs = (smin > 0.0 && !any_nan) ? __dmul_rd(a.kappa, smin) : 0.0;
+  const int32_t lab = a.payload ? a.payload[row] : y;
+  const bool acc = !(a.require_consistency && lab != y) && (r64 > 0.0) && !(a.miss_of && a.miss_of[row] >= 0);
+  float rr, tau;
+  thresholds(__double2float_rd(rs), kn, a.tc, rr, tau);
+  a.accept[row] = acc ? 1 : 0;
+  a.yG[row] = y;
+  a.label[row] = lab;
+  a.radius[row] = __double2float_rz(r64);
+  a.rr[row] = rr;
+  a.kn[row] = kn;
   a.tau[row] = tau;
   *acc_slot = acc ? 1 : 0;
 }

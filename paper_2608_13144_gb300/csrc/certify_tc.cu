@@ -1,5 +1,5 @@
 // Certified insertion on the tensor cores (Sec. 3.3, Algorithm 1 loop body;
-// Eqs. 5, 6, 20, 21), conservative radius.
+// Eqs. 5, 6, 20, 21; the tight radius of Remark 4.2, Eq. 29).
 //
 // The head logits of a batch, s = W z + b for every row z, form one dense
 // contraction (rows x d) . (d x C). This kernel runs it as TF32 tcgen05 MMAs
@@ -19,9 +19,18 @@
 // Mb also bounds every partial sum of the MMA, so when Mb < 1e38 no screen
 // value overflows or is NaN; a row with a larger (or NaN) Mb - NaN or infinite
 // features, or values near the FP32 range - has every class refined.
-// If l2 is the second-largest s~_c, every class of the true top two has
-// s_c >= (true runner-up) >= l2 - E, hence s~_c >= l2 - 2E >= T = RD(l2 - 2E):
-// the classes with s~_c >= T are the candidates.
+// Conservative radius: if l2 is the second-largest s~_c, every class of the
+// true top two has s_c >= (true runner-up) >= l2 - E, hence s~_c >= l2 - 2E >=
+// T = RD(l2 - 2E): the classes with s~_c >= T are the candidates.
+// Tight radius: with y1 / y2 the screen's top two, y1 is certainly y^G when
+// y2's upper end is below y1's lower end; then the candidates are y1 and the
+// classes whose lower bracket of (s_y - s_j) / ||W_y - W_j|| reaches u_{y2},
+// first with the head row's smallest reciprocal pair norm, then with the
+// class's own (the minimiser of Eq. 29 always passes). Otherwise one test
+// valid for every possible y^G (lower end above lo_1 - 2E, r* below a bound
+// from y1's row) picks the candidates, and y^G is the largest refined one.
+// Each half reduces Eq. 29 over its own candidates in FP64; rows with more
+// candidates than slots take a one-warp path over every class.
 //
 // Schedule. Persistent CTAs, one per SM, 320 threads:
 //   warp 0     TMA producer: W (resident, 128-byte swizzle, rows past C zero
@@ -61,16 +70,53 @@ constexpr int kListCap = 32 * kMaxCandTc;     // pair list of one epilogue warp
 // per epilogue warp: the pair list, then the refined pairs hi / lo by (row lane, slot)
 constexpr uint32_t kWarpScratch = kListCap * 4 + 32 * kMaxCandTc * 8;
 constexpr int kGroupTc = 8;                   // lanes per refined pair
+constexpr int kNoClass = 0xffff;              // "no class yet" in the indexed top-two trackers
 constexpr uint32_t kTmemCols = 512;           // two accumulators of up to 256 columns
 constexpr uint32_t kAccStride = 256;
 constexpr long long kWaitLimit = 1LL << 31;   // ~1 s at GB300 clocks
 constexpr int kSmemBudget = 227 * 1024 - 1024;
 
 // Per-row state a half hands to its partner after the first pass: the top
-// two s~ of its columns and its half of ||z||^2.
+// two s~ of its columns, its half of ||z||^2 and (tight radius) the classes of
+// the top two (low / high 16 bits).
 struct Pass1 {
-  float l1, l2, psum, pad;
+  float l1, l2, psum;
+  int idx;
 };
+
+// Exchange area of the tight radius (in the space of the conservative
+// radius's Top2 exchange): each half's best refined candidate (value and
+// class) and overflow flag, and half 1's partial minima of Eq. 29.
+struct TightX {
+  float2 bv[2][128];
+  int16_t bc[2][128];  // -1: no candidate
+  uint8_t ovf[2][128];
+  double rmin[128], smin[128];
+  uint8_t nan[128];
+};
+
+static_assert(sizeof(TightX) <= kBM * sizeof(Top2), "the tight exchange shares the Top2 exchange area");
+
+// (a1, j1) >= (a2, j2) are the top two (value, class) of one set; merge in
+// the top two (b1, k1) >= (b2, k2) of a disjoint set. Larger value first,
+// lower class on equal values.
+__device__ __forceinline__ void top2i_merge(float& a1, int& j1, float& a2, int& j2, float b1, int k1, float b2,
+                                            int k2) {
+  auto better = [](float x, int i, float y, int k) { return x > y || (x == y && i < k); };
+  if (better(b1, k1, a1, j1)) {
+    if (!better(a1, j1, b2, k2)) {
+      a1 = b2;
+      j1 = k2;
+    }
+    a2 = a1;
+    j2 = j1;
+    a1 = b1;
+    j1 = k1;
+  } else if (better(b1, k1, a2, j2)) {
+    a2 = b1;
+    j2 = k1;
+  }
+}
 
 // Shared-memory layout (offsets from a 1024-byte aligned base).
 struct TcLayout {
@@ -244,6 +290,93 @@ __device__ __forceinline__ void refine2(uint32_t ws, uint32_t wchunk, uint32_t z
   }
 }
 
+// The tight radius (Eq. 29) of one row on one warp, for rows the screen
+// cannot settle (several possible y^G, Mb not below 1e38, more candidates than
+// slots): every class refined with the compensated dot product (lane = class,
+// features in order, as the wide-tile kernel's fallback), y^G the largest
+// refined logit (lowest class on ties), then Eq. 29 over every other class in
+// FP64. The row's features come from the tile in shared memory (row rz).
+__device__ void tc_tight_row_warp(const CertArgs& a, int64_t row, int rz, uint32_t s_w, uint32_t wchunk, uint32_t zs,
+                                  const float* __restrict__ wn_s, const float* __restrict__ b_s, float kn, int lane,
+                                  uint8_t* acc_slot) {
+  constexpr int kPer = 8;  // classes per lane (C <= 256)
+  const int d = a.d, C = a.C;
+  const float hn = norm_upper(kn);
+  float vh[kPer], vl[kPer], ve[kPer];
+  float bh = -INFINITY, bl = 0.f;
+  int by = -1;
+  bool nan_any = false;
+#pragma unroll
+  for (int t = 0; t < kPer; ++t) {
+    const int c = lane + 32 * t;
+    vh[t] = NAN;
+    vl[t] = 0.f;
+    ve[t] = 0.f;
+    if (c < C) {
+      float p = 0.f, cc = 0.f;
+      for (int k = 0; k < d; ++k) {
+        float w, x;
+        asm volatile("ld.shared.f32 %0, [%1];" : "=f"(w) : "r"(s_w + sw_off(c, k, wchunk)));
+        asm volatile("ld.shared.f32 %0, [%1];" : "=f"(x) : "r"(zs + sw_off(rz, k, kZChunkBytes)));
+        const float pr = __fmul_rn(w, x);
+        const float er = __fmaf_rn(w, x, -pr);
+        float s1, q;
+        two_sum(p, pr, s1, q);
+        p = s1;
+        cc = __fadd_rn(cc, __fadd_rn(q, er));
+      }
+      float s1, q, hi, lo;
+      two_sum(p, b_s[c], s1, q);
+      two_sum(s1, __fadd_rn(cc, q), hi, lo);
+      vh[t] = hi;
+      vl[t] = lo;
+      ve[t] = refined_err(a.g2f, wn_s[c], hn, b_s[c]);
+      nan_any |= !(hi == hi && lo == lo);
+      if (pair_gt(hi, lo, bh, bl)) {  // ascending classes: ties keep the lowest
+        bh = hi;
+        bl = lo;
+        by = c;
+      }
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float oh = __shfl_xor_sync(kFull, bh, o), ol = __shfl_xor_sync(kFull, bl, o);
+    const int oy = __shfl_xor_sync(kFull, by, o);
+    const bool eq = oh == bh && ol == bl;
+    if (oy >= 0 && (by < 0 || pair_gt(oh, ol, bh, bl) || (eq && oy < by))) {
+      bh = oh;
+      bl = ol;
+      by = oy;
+    }
+  }
+  nan_any = __any_sync(kFull, nan_any);
+  const int y = by < 0 ? 0 : by;
+  float myh = 0.f, myl = 0.f, mye = 0.f;
+#pragma unroll
+  for (int t = 0; t < kPer; ++t)
+    if (lane + 32 * t == y) {
+      myh = vh[t];
+      myl = vl[t];
+      mye = ve[t];
+    }
+  const int owner = y & 31;
+  const double vy = (double)__shfl_sync(kFull, myh, owner) + (double)__shfl_sync(kFull, myl, owner);
+  const double ey = (double)__shfl_sync(kFull, mye, owner);
+  double rmin = INFINITY, smin = INFINITY;
+#pragma unroll
+  for (int t = 0; t < kPer; ++t) {
+    const int j = lane + 32 * t;
+    if (j >= C || j == y) continue;
+    tight_term(a, y, j, vy, ey, (double)vh[t] + (double)vl[t], (double)ve[t], rmin, smin);
+  }
+  rmin = warp_min_d(rmin);
+  smin = warp_min_d(smin);
+  if (lane == 0) tight_write(a, row, y, rmin, smin, nan_any, kn, acc_slot);
+  __syncwarp();
+}
+
+template <bool TIGHT>
 __global__ void __launch_bounds__(kThreads, 1)
     k_certify_tc(const __grid_constant__ CUtensorMap tmH, const __grid_constant__ CUtensorMap tmW, const CertArgs a,
                  const TcLayout L, int n_tiles, DevStats* stats, int debug_stall) {
@@ -404,6 +537,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       const float ob = __shfl_xor_sync(kFull, bmax, o);
       bmax = (ob > bmax || ob != ob) ? ob : bmax;
     }
+    // tight radius: the smallest lower bound of 1 / ||W_y - W_j|| over the
+    // head
+    float imA = INFINITY;
+    if constexpr (TIGHT) {
+      for (int c = lane; c < C; c += 32) imA = fminf(imA, __ldg(a.ipn_min32 + c));
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) imA = fminf(imA, __shfl_xor_sync(kFull, imA, o));
+    }
     const float c32 = __double2float_ru(a.c_scr);
     const float cw = __fmul_ru(c32, wmax), cw1 = __fmul_ru(__fadd_ru(1.f, c32), wmax);
     // top two of the s~ in a 32-column chunk, four independent trackers
@@ -443,6 +584,62 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       return lim == 32 ? mask : mask & ((1u << lim) - 1u);
     };
+    // tight radius: the top two with their classes (four trackers), and the
+    // candidates of Eq. 29: bit j set unless (lo_y - hi_j) ipn_min(y) > U
+    auto pass1_chunk_idx = [&](const uint32_t (&v)[32], int ch, float (&t1)[4], int (&i1)[4], float (&t2)[4],
+                               int (&i2)[4]) {
+      const int lim = min(32, C - ch * 32);
+      const float4* b4 = reinterpret_cast<const float4*>(bias_s + ch * 32);
+#pragma unroll
+      for (int j4 = 0; j4 < 8; ++j4) {
+        const float4 bb = b4[j4];
+        const float bv[4] = {bb.x, bb.y, bb.z, bb.w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const int j = 4 * j4 + e, c = ch * 32 + j;
+          float sv = __fadd_rn(__uint_as_float(v[j]), bv[e]);
+          sv = (lim == 32 || j < lim) ? sv : -INFINITY;
+          const bool g1 = sv > t1[e], g2 = sv > t2[e];
+          t2[e] = g1 ? t1[e] : (g2 ? sv : t2[e]);
+          i2[e] = g1 ? i1[e] : (g2 ? c : i2[e]);
+          t1[e] = g1 ? sv : t1[e];
+          i1[e] = g1 ? c : i1[e];
+        }
+      }
+    };
+    // A class passes the bound test (lo - hi_j) im <= U, then - when y^G is
+    // certain - the exact one with its own FP32 bracket of 1 / ||W_y - W_j||
+    // (irow: the bracket-table row of y). The brackets are loaded only where
+    // the bound test passed, sixteen predicated loads in flight at a time.
+    auto pass2_chunk_tight = [&](const uint32_t (&v)[32], int ch, float E, float lo, float im, float U,
+                                 const float* __restrict__ irow, bool exact) -> uint32_t {
+      const int lim = min(32, C - ch * 32);
+      const float* bc = bias_s + ch * 32;
+      uint32_t crude = 0;
+#pragma unroll
+      for (int j = 0; j < 32; ++j) {
+        const float hj = __fadd_ru(__fadd_rn(__uint_as_float(v[j]), bc[j]), E);
+        crude |= (uint32_t)(__fmul_rd(__fsub_rd(lo, hj), im) <= U) << j;
+      }
+      crude &= lim == 32 ? 0xffffffffu : (1u << lim) - 1u;
+      uint32_t mask = exact ? 0u : crude;
+#pragma unroll
+      for (int h16 = 0; h16 < 2; ++h16) {
+        float p[16];
+#pragma unroll
+        for (int k = 0; k < 16; ++k) {
+          const int j = 16 * h16 + k;
+          p[k] = (exact && ((crude >> j) & 1u)) ? __ldg(irow + ch * 32 + j) : 0.f;
+        }
+#pragma unroll
+        for (int k = 0; k < 16; ++k) {
+          const int j = 16 * h16 + k;
+          const float hj = __fadd_ru(__fadd_rn(__uint_as_float(v[j]), bc[j]), E);
+          mask |= (uint32_t)(exact && ((crude >> j) & 1u) && __fmul_rd(__fsub_rd(lo, hj), p[k]) <= U) << j;
+        }
+      }
+      return mask;
+    };
 
     unsigned long long n_pairs = 0, n_full = 0;  // this warp's refinement counts
     int t = 0;
@@ -457,7 +654,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int64_t grow = (int64_t)tile * kBM + r;
       const bool live = grow < a.n;
       const uint32_t tacc = tmem + lane_base + (uint32_t)buf * kAccStride;
-      Pass1 mine{-INFINITY, -INFINITY, 0.f, 0.f};
+      Pass1 mine{-INFINITY, -INFINITY, 0.f, kNoClass | (kNoClass << 16)};
       if (ok) {
         // two of the four k-ordered partial sums of ||z||^2 (quarters 2 half,
         // 2 half + 1 of the features; the FP32 kernels form the same chains)
@@ -478,30 +675,57 @@ __global__ void __launch_bounds__(kThreads, 1)
         mine.psum = pc[0] + pc[1];
         // pass 1: top two s~ of this half's columns (two chunks per TMEM wait)
         float t1[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY}, t2[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
-        for (int ch = half; ch < nck; ch += 4) {
-          uint32_t va[32], vb[32];
-          const bool two = ch + 2 < nck;
-          ptx::tmem_ld32(tacc + (uint32_t)(ch * 32), va);
-          if (two) ptx::tmem_ld32(tacc + (uint32_t)((ch + 2) * 32), vb);
-          ptx::tmem_wait_ld();
-          pass1_chunk(va, ch, t1, t2);
-          if (two) pass1_chunk(vb, ch + 2, t1, t2);
-        }
-        float l1 = t1[0], l2 = t2[0];
+        if constexpr (TIGHT) {
+          int i1[4] = {kNoClass, kNoClass, kNoClass, kNoClass}, i2[4] = {kNoClass, kNoClass, kNoClass, kNoClass};
+          for (int ch = half; ch < nck; ch += 4) {
+            uint32_t va[32], vb[32];
+            const bool two = ch + 2 < nck;
+            ptx::tmem_ld32(tacc + (uint32_t)(ch * 32), va);
+            if (two) ptx::tmem_ld32(tacc + (uint32_t)((ch + 2) * 32), vb);
+            ptx::tmem_wait_ld();
+            pass1_chunk_idx(va, ch, t1, i1, t2, i2);
+            if (two) pass1_chunk_idx(vb, ch + 2, t1, i1, t2, i2);
+          }
 #pragma unroll
-        for (int e = 1; e < 4; ++e) {
-          l2 = fmaxf(fmaxf(l2, t2[e]), fminf(l1, t1[e]));
-          l1 = fmaxf(l1, t1[e]);
+          for (int e = 1; e < 4; ++e) top2i_merge(t1[0], i1[0], t2[0], i2[0], t1[e], i1[e], t2[e], i2[e]);
+          mine.idx = (i1[0] & 0xffff) | (i2[0] << 16);
+        } else {
+          for (int ch = half; ch < nck; ch += 4) {
+            uint32_t va[32], vb[32];
+            const bool two = ch + 2 < nck;
+            ptx::tmem_ld32(tacc + (uint32_t)(ch * 32), va);
+            if (two) ptx::tmem_ld32(tacc + (uint32_t)((ch + 2) * 32), vb);
+            ptx::tmem_wait_ld();
+            pass1_chunk(va, ch, t1, t2);
+            if (two) pass1_chunk(vb, ch + 2, t1, t2);
+          }
+#pragma unroll
+          for (int e = 1; e < 4; ++e) {
+            t2[0] = fmaxf(fmaxf(t2[0], t2[e]), fminf(t1[0], t1[e]));
+            t1[0] = fmaxf(t1[0], t1[e]);
+          }
         }
-        mine.l1 = l1;
-        mine.l2 = l2;
+        mine.l1 = t1[0];
+        mine.l2 = t2[0];
       }
       x1[half * kBM + r] = mine;
       if (lane == 0) okf[half * 4 + quarter] = ok ? 1 : 0;
       pair_barrier(bar_id);
       const Pass1 o = x1[(half ^ 1) * kBM + r];
       if (!ok || okf[(half ^ 1) * 4 + quarter] == 0) break;  // both warps of the pair leave together
-      const float L2 = fmaxf(fmaxf(mine.l2, o.l2), fminf(mine.l1, o.l1));
+      float L1 = fmaxf(mine.l1, o.l1), L2 = fmaxf(fmaxf(mine.l2, o.l2), fminf(mine.l1, o.l1));
+      int y = kNoClass, j2 = kNoClass;
+      if constexpr (TIGHT) {
+        // both warps merge in the same order (half 0's list first), so they
+        // agree on the classes
+        const Pass1& p0 = half == 0 ? mine : o;
+        const Pass1& p1 = half == 0 ? o : mine;
+        L1 = p0.l1;
+        L2 = p0.l2;
+        y = p0.idx & 0xffff;
+        j2 = p0.idx >> 16;
+        top2i_merge(L1, y, L2, j2, p1.l1, p1.idx & 0xffff, p1.l2, p1.idx >> 16);
+      }
       const float kn = __fadd_rn(mine.psum, o.psum);  // (q0 + q1) + (q2 + q3)
       const float hn = norm_upper(kn);
       // |s~_c| <= Mb, so every screen value and partial sum is finite when
@@ -510,6 +734,40 @@ __global__ void __launch_bounds__(kThreads, 1)
       const float E = __fmaf_ru(cw, hn, __fmaf_ru(Mb, 2.3841858e-07f /* 2^-22 */, kTinyF));
       const float T = __fsub_rd(L2, __fmul_ru(2.f, E));
       bool fb = live && !(Mb < 1e38f);  // NaN / infinite features, or a bound near FP32 overflow
+      // tight radius. If y1 (the screen's top class) is certainly y^G (the
+      // runner-up's upper end below lo_1), U1 = u_{y2}(y1) bounds r*/kappa
+      // from above and (lo_1 - hi_j) ipn_min(y1) <= l_j bounds every class's
+      // bracket from below, so the minimiser of Eq. 29 passes (lo_1 - hi_j)
+      // ipn_min(y1) <= U1 (then also with its own bracket l_j). Otherwise every
+      // possible y^G has its lower end above lo* = lo_1 - 2E (less rounding) and
+      // r*/kappa below U* (below), so one test with lo*, U* and the head's
+      // smallest ipn keeps the minimiser for whichever class is y^G; y^G is
+      // then the largest refined candidate.
+      float lo1 = 0.f, U1 = 0.f, im1 = 0.f;
+      bool unc = false;
+      if constexpr (TIGHT) {
+        lo1 = __fsub_rd(L1, E);
+        const float hi1 = __fadd_ru(L1, E), lo2 = __fsub_rd(L2, E), hi2 = __fadd_ru(L2, E);
+        const bool settled = live && !fb && y < C && j2 < C;
+        if (settled) {
+          unc = !(hi2 < lo1);
+          if (!unc) {
+            U1 = __fmul_ru(__fsub_ru(hi1, lo2), __ldg(a.ipn_up32 + (size_t)y * C + j2));
+            im1 = __ldg(a.ipn_min32 + y);
+          } else {
+            // r* <= u_{y2}(y1) if y1 is y^G; for any other possible y^G (its
+            // s~ <= l2) r* <= (hi_2 - lo_1) / ||W_y - W_y1|| <= (hi_2 - lo_1)
+            // ipn_max(y1), the pair norms being symmetric
+            U1 = fmaxf(__fmul_ru(__fsub_ru(hi1, lo2), __ldg(a.ipn_up32 + (size_t)y * C + j2)),
+                       __fmul_ru(__fsub_ru(hi2, lo1), __ldg(a.ipn_max32 + y)));
+            lo1 = __fsub_rd(lo1, __fmaf_ru(E, 2.0001f, __fmaf_ru(fabsf(lo1), 9.5367432e-07f /* 2^-20 */, kTinyF)));
+            im1 = imA;
+          }
+        }
+        fb = live && !settled;  // the whole row goes to the one-warp path (both halves agree)
+      }
+      // row of the lower-bracket table for y1 (a valid address also when unused)
+      const float* irow1 = a.ipn_dn32 ? a.ipn_dn32 + (size_t)(y < C ? y : 0) * C : nullptr;
 
       // pass 2: the candidates of this half's columns into the warp's list;
       // the row's lane keeps its slots' classes (one byte each)
@@ -541,12 +799,19 @@ __global__ void __launch_bounds__(kThreads, 1)
         ptx::tmem_ld32(tacc + (uint32_t)(ch * 32), va);
         if (two) ptx::tmem_ld32(tacc + (uint32_t)((ch + 2) * 32), vb);
         ptx::tmem_wait_ld();
-        const uint32_t ma = pass2_chunk(va, ch, T);
-        const uint32_t mbk = two ? pass2_chunk(vb, ch + 2, T) : 0u;
+        uint32_t ma, mbk = 0u;
+        if constexpr (TIGHT) {
+          ma = pass2_chunk_tight(va, ch, E, lo1, im1, U1, irow1, !unc);
+          if (two) mbk = pass2_chunk_tight(vb, ch + 2, E, lo1, im1, U1, irow1, !unc);
+        } else {
+          ma = pass2_chunk(va, ch, T);
+          if (two) mbk = pass2_chunk(vb, ch + 2, T);
+        }
         append(ma, ch);
         if (two) append(mbk, ch + 2);
       }
-      fb = fb || cnt > kMaxCandTc;
+      const bool ovf = cnt > kMaxCandTc;  // (tight: the row goes to the one-warp path, below)
+      if constexpr (!TIGHT) fb = fb || ovf;
       ptx::tc_fence_before();
       __syncwarp();
       if (lane == 0) ptx::mbar_arrive(accempty + 8 * buf);  // the accumulator is free for tile t + 2
@@ -573,71 +838,162 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
       }
-      __syncwarp();
-      // each row's lane pushes its own candidates into its running selection
-      Top2 tp;
-      if (!fb) {
-        const int ns = cnt < kMaxCandTc ? cnt : kMaxCandTc;
-        for (int sl = 0; sl < ns; ++sl) {
-          const int c = (int)(((sl < 4 ? cls_lo >> (8 * sl) : cls_hi >> (8 * (sl - 4)))) & 0xffu);
-          tp.push(c, res_hi[lane + 32 * sl], res_lo[lane + 32 * sl], refined_err(a.g2f, wn_s[c], hn, bias_s[c]));
-        }
-      }
-      // rows that need every class of this half refined, one row at a time,
-      // eight classes a round through the row's result cells
-      const unsigned fbm = __ballot_sync(kFull, fb);
-      if (lane == 0) {
-        n_full += (unsigned long long)__popc(fbm);
-        n_pairs += (unsigned long long)P + (unsigned long long)__popc(fbm) * (unsigned long long)ncls;
-      }
-      for (unsigned fr = fbm; fr != 0; fr &= fr - 1) {
-        const int ow = __ffs((int)fr) - 1;
-        if (lane == ow) tp = Top2();
-        for (int t2 = 0; t2 < ncls; t2 += 2 * (32 / kGroupTc)) {
-          int tq[2] = {t2 + 2 * g8, t2 + 2 * g8 + 1};
-          int cp[2];
-#pragma unroll
-          for (int u = 0; u < 2; ++u) {
-            const int tt = tq[u] < ncls ? tq[u] : t2;
-            cp[u] = (2 * (tt >> 5) + half) * 32 + (tt & 31);
+      if constexpr (!TIGHT) {
+        __syncwarp();
+        // each row's lane pushes its own candidates into its running selection
+        Top2 tp;
+        if (!fb) {
+          const int ns = cnt < kMaxCandTc ? cnt : kMaxCandTc;
+          for (int sl = 0; sl < ns; ++sl) {
+            const int c = (int)(((sl < 4 ? cls_lo >> (8 * sl) : cls_hi >> (8 * (sl - 4)))) & 0xffu);
+            tp.push(c, res_hi[lane + 32 * sl], res_lo[lane + 32 * sl], refined_err(a.g2f, wn_s[c], hn, bias_s[c]));
           }
-          const int rp[2] = {rq + ow, rq + ow};
-          const float bp[2] = {bias_s[cp[0]], bias_s[cp[1]]};
-          float hi[2], lo[2];
-          refine2(s_w, wchunk, zs, cp, rp, bp, d, sub, hi, lo);
-          if (sub == 0) {
+        }
+        // rows that need every class of this half refined, one row at a time,
+        // eight classes a round through the row's result cells
+        const unsigned fbm = __ballot_sync(kFull, fb);
+        if (lane == 0) {
+          n_full += (unsigned long long)__popc(fbm);
+          n_pairs += (unsigned long long)P + (unsigned long long)__popc(fbm) * (unsigned long long)ncls;
+        }
+        for (unsigned fr = fbm; fr != 0; fr &= fr - 1) {
+          const int ow = __ffs((int)fr) - 1;
+          if (lane == ow) tp = Top2();
+          for (int t2 = 0; t2 < ncls; t2 += 2 * (32 / kGroupTc)) {
+            int tq[2] = {t2 + 2 * g8, t2 + 2 * g8 + 1};
+            int cp[2];
 #pragma unroll
             for (int u = 0; u < 2; ++u) {
-              res_hi[ow + 32 * (2 * g8 + u)] = hi[u];
-              res_lo[ow + 32 * (2 * g8 + u)] = lo[u];
+              const int tt = tq[u] < ncls ? tq[u] : t2;
+              cp[u] = (2 * (tt >> 5) + half) * 32 + (tt & 31);
+            }
+            const int rp[2] = {rq + ow, rq + ow};
+            const float bp[2] = {bias_s[cp[0]], bias_s[cp[1]]};
+            float hi[2], lo[2];
+            refine2(s_w, wchunk, zs, cp, rp, bp, d, sub, hi, lo);
+            if (sub == 0) {
+#pragma unroll
+              for (int u = 0; u < 2; ++u) {
+                res_hi[ow + 32 * (2 * g8 + u)] = hi[u];
+                res_lo[ow + 32 * (2 * g8 + u)] = lo[u];
+              }
+            }
+            __syncwarp();
+            if (lane == ow)
+              for (int u = 0; u < 2 * (32 / kGroupTc) && t2 + u < ncls; ++u) {
+                const int tt = t2 + u;
+                const int c = (2 * (tt >> 5) + half) * 32 + (tt & 31);
+                tp.push(c, res_hi[ow + 32 * u], res_lo[ow + 32 * u], refined_err(a.g2f, wn_s[c], hn, bias_s[c]));
+              }
+            __syncwarp();
+          }
+        }
+        __syncwarp();
+        if (lane == 0) ptx::mbar_arrive(zempty + 8 * zb);  // this warp is done with the tile's features
+
+        // merge the halves; FP64 finals and the row's rank in its 32-row block
+        if (half == 1) x2[r] = tp;
+        pair_barrier(bar_id);
+        if (half == 0) {
+          top2_merge(tp, x2[r]);
+          if (live)
+            row_finals(a, grow, tp.result(kn), &acc_s[r]);
+          else
+            acc_s[r] = 0;
+          const unsigned mb = __ballot_sync(kFull, live && acc_s[r] != 0);
+          if (live) a.rank[grow] = __popc(mb & ((1u << lane) - 1u));
+          const int64_t blk0 = (int64_t)tile * kBM + quarter * 32;
+          if (lane == 0 && blk0 < a.n) a.bcount[blk0 / 32] = __popc(mb);
+        }
+      } else {
+        // tight radius (Eq. 29): y^G is the largest refined candidate (each
+        // half's best, merged in the same order by both); each half's minima
+        // over its own candidates; half 0 combines them and takes the rows the
+        // screen could not settle
+        TightX& tx = *reinterpret_cast<TightX*>(smem + L.off_x2);
+        const int ns = cnt < kMaxCandTc ? cnt : kMaxCandTc;
+        auto slot_class = [&](int sl) {
+          return (int)((sl < 4 ? cls_lo >> (8 * sl) : cls_hi >> (8 * (sl - 4))) & 0xffu);
+        };
+        float bh = -INFINITY, bl = 0.f;
+        int bc = -1;
+        if (live && !fb && !ovf)
+          for (int sl = 0; sl < ns; ++sl) {
+            const int c = slot_class(sl);
+            const float h = res_hi[lane + 32 * sl], l = res_lo[lane + 32 * sl];
+            if (bc < 0 || pair_gt(h, l, bh, bl) || (h == bh && l == bl && c < bc)) {
+              bh = h;
+              bl = l;
+              bc = c;
             }
           }
-          __syncwarp();
-          if (lane == ow)
-            for (int u = 0; u < 2 * (32 / kGroupTc) && t2 + u < ncls; ++u) {
-              const int tt = t2 + u;
-              const int c = (2 * (tt >> 5) + half) * 32 + (tt & 31);
-              tp.push(c, res_hi[ow + 32 * u], res_lo[ow + 32 * u], refined_err(a.g2f, wn_s[c], hn, bias_s[c]));
-            }
-          __syncwarp();
+        tx.bv[half][r] = make_float2(bh, bl);
+        tx.bc[half][r] = (int16_t)bc;
+        tx.ovf[half][r] = ovf ? 1 : 0;
+        pair_barrier(bar_id);
+        const bool rowfb = fb || (live && (tx.ovf[0][r] != 0 || tx.ovf[1][r] != 0));
+        double rmin = INFINITY, smin = INFINITY;
+        bool any_nan = false;
+        int yg = y;
+        if (live && !rowfb) {
+          float2 v2 = tx.bv[0][r];
+          yg = tx.bc[0][r];
+          const float2 w2 = tx.bv[1][r];
+          const int c1 = tx.bc[1][r];
+          if (c1 >= 0 && (yg < 0 || pair_gt(w2.x, w2.y, v2.x, v2.y) || (w2.x == v2.x && w2.y == v2.y && c1 < yg))) {
+            v2 = w2;
+            yg = c1;
+          }
+          any_nan = yg < 0;  // no candidate (cannot happen: y1 always passes)
+          if (any_nan) yg = y;
+          const double vy = (double)v2.x + (double)v2.y;
+          const double ey = (double)refined_err(a.g2f, wn_s[yg], hn, bias_s[yg]);
+          any_nan = any_nan || !(vy == vy);
+          for (int sl = 0; sl < ns; ++sl) {
+            const int j = slot_class(sl);
+            if (j == yg) continue;
+            const double vj = (double)res_hi[lane + 32 * sl] + (double)res_lo[lane + 32 * sl];
+            any_nan |= !(vj == vj);
+            tight_term(a, yg, j, vy, ey, vj, (double)refined_err(a.g2f, wn_s[j], hn, bias_s[j]), rmin, smin);
+          }
         }
-      }
-      __syncwarp();
-      if (lane == 0) ptx::mbar_arrive(zempty + 8 * zb);  // this warp is done with the tile's features
-
-      // merge the halves; FP64 finals and the row's rank in its 32-row block
-      if (half == 1) x2[r] = tp;
-      pair_barrier(bar_id);
-      if (half == 0) {
-        top2_merge(tp, x2[r]);
-        if (live)
-          row_finals(a, grow, tp.result(kn), &acc_s[r]);
-        else
-          acc_s[r] = 0;
-        const unsigned mb = __ballot_sync(kFull, live && acc_s[r] != 0);
-        if (live) a.rank[grow] = __popc(mb & ((1u << lane) - 1u));
-        const int64_t blk0 = (int64_t)tile * kBM + quarter * 32;
-        if (lane == 0 && blk0 < a.n) a.bcount[blk0 / 32] = __popc(mb);
+        const unsigned fbm = __ballot_sync(kFull, rowfb);
+        if (lane == 0) {
+          n_pairs += (unsigned long long)P;
+          if (half == 0) {
+            n_full += (unsigned long long)__popc(fbm);
+            n_pairs += (unsigned long long)__popc(fbm) * (unsigned long long)C;
+          }
+        }
+        if (half == 1) {
+          tx.rmin[r] = rmin;
+          tx.smin[r] = smin;
+          tx.nan[r] = any_nan ? 1 : 0;
+        }
+        pair_barrier(bar_id);
+        if (half == 0) {
+          if (!rowfb) acc_s[r] = 0;
+          if (live && !rowfb)
+            tight_write(a, grow, yg, fmin(rmin, tx.rmin[r]), fmin(smin, tx.smin[r]), any_nan || tx.nan[r] != 0, kn,
+                        &acc_s[r]);
+        }
+        // the rows the screen could not settle, alternately on the two warps
+        int k = 0;
+        for (unsigned fr = fbm; fr != 0; fr &= fr - 1, ++k) {
+          const int ow = __ffs((int)fr) - 1;
+          if ((k & 1) == half)
+            tc_tight_row_warp(a, (int64_t)tile * kBM + rq + ow, rq + ow, s_w, wchunk, zs, wn_s, bias_s,
+                              __shfl_sync(kFull, kn, ow), lane, &acc_s[rq + ow]);
+        }
+        __syncwarp();
+        if (lane == 0) ptx::mbar_arrive(zempty + 8 * zb);  // this warp is done with the tile's features
+        pair_barrier(bar_id);  // every acceptance flag of the 32 rows is written
+        if (half == 0) {
+          const unsigned mb = __ballot_sync(kFull, live && acc_s[r] != 0);
+          if (live) a.rank[grow] = __popc(mb & ((1u << lane) - 1u));
+          const int64_t blk0 = (int64_t)tile * kBM + quarter * 32;
+          if (lane == 0 && blk0 < a.n) a.bcount[blk0 / 32] = __popc(mb);
+        }
       }
     }
     if (lane == 0 && (n_pairs | n_full)) {
@@ -681,7 +1037,11 @@ bool tc_plan(int d, int C, TcLayout& L) {
 }  // namespace
 
 bool certify_tc_supported(const lipcache* h, const float* H, int64_t n) {
-  if (h->radius_mode == LIPCACHE_RADIUS_TIGHT || h->encode == nullptr) return false;
+  if (h->encode == nullptr) return false;
+  // the tight radius needs the bracket tables of the head's pair norms
+  if (h->radius_mode == LIPCACHE_RADIUS_TIGHT &&
+      (h->ipn_up32 == nullptr || h->ipn_min32 == nullptr || h->ipn_max32 == nullptr))
+    return false;
   if (h->debug_flags & (LIPCACHE_DEBUG_INSERT_TILE64 | LIPCACHE_DEBUG_INSERT_WIDE_TILE)) return false;
   // TMA: 16-byte aligned rows of d floats, 32-feature boxes (at most
   // kMaxChunks of them); MMA: N <= 256
@@ -702,9 +1062,10 @@ void certify_tc_launch(lipcache* h, const CertArgs& a, cudaStream_t s) {
   // at least half of the SM's shared memory, so one CTA (and one 512-column
   // TMEM allocation) per SM
   const int smem = (int)L.total + 1024 > 120 * 1024 ? (int)L.total + 1024 : 120 * 1024;
-  LC_CUDA(cudaFuncSetAttribute(k_certify_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
-  k_certify_tc<<<grid, kThreads, smem, s>>>(tmH, tmW, a, L, n_tiles, h->stats,
-                                            (h->debug_flags & LIPCACHE_DEBUG_STALL_INSERT) ? 1 : 0);
+  auto kern = a.tight ? k_certify_tc<true> : k_certify_tc<false>;
+  LC_CUDA(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
+  kern<<<grid, kThreads, smem, s>>>(tmH, tmW, a, L, n_tiles, h->stats,
+                                    (h->debug_flags & LIPCACHE_DEBUG_STALL_INSERT) ? 1 : 0);
   LC_LAUNCH_CHECK("k_certify_tc");
 }
 

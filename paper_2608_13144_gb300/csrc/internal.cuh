@@ -183,6 +183,8 @@ struct lipcache {
   double* inv_pairnorm = nullptr;  // C x C: 1 / pairnorm (0 where pairnorm is 0)
   float* ipn_up32 = nullptr;       // C x C: FP32 upper bound of 1 / ||W_y - W_j|| (+inf where it is 0)
   float* ipn_dn32 = nullptr;       // C x C: FP32 lower bound (+inf where ||W_y - W_j|| is 0)
+  float* ipn_min32 = nullptr;      // C: min_j of ipn_dn32[y][j] over the rows W_j != W_y (0 if none)
+  float* ipn_max32 = nullptr;      // C: max_j of ipn_up32[y][j] over j != y (+inf if some W_j = W_y)
   double* gram[2] = {nullptr, nullptr};  // d x d FP64
   lc::SpecResult* spec = nullptr;        // device
   lc::SpecResult* spec_host = nullptr;   // pinned

@@ -205,6 +205,26 @@ __global__ void k_row_norms(const float* __restrict__ W, int C, int d, double* _
   }
 }
 
+// Bounds of a whole row of the bracket tables, which the tensor certify
+// kernel's tight-radius screen uses in place of the tables:
+// ipn_min32[y] <= 1 / ||W_y - W_j|| for every j with W_j != W_y (the minimum of
+// the FP32 lower brackets; 0 when every other row equals W_y) and
+// ipn_max32[y] >= 1 / ||W_y - W_j|| for every j != y (+inf when some W_j = W_y).
+__global__ void k_ipn_min(const double* __restrict__ pairnorm, const float* __restrict__ ipn_dn32,
+                          const float* __restrict__ ipn_up32, int C, float* __restrict__ ipn_min32,
+                          float* __restrict__ ipn_max32) {
+  const int y = blockIdx.x * blockDim.x + threadIdx.x;
+  if (y >= C) return;
+  float m = INFINITY, mx = 0.f;
+  for (int j = 0; j < C; ++j) {
+    if (j == y) continue;
+    if (pairnorm[(size_t)y * C + j] > 0.0) m = fminf(m, ipn_dn32[(size_t)y * C + j]);
+    mx = fmaxf(mx, ipn_up32[(size_t)y * C + j]);
+  }
+  ipn_min32[y] = m < INFINITY ? m : 0.f;
+  ipn_max32[y] = mx;
+}
+
 }  // namespace
 
 void spectral_norm(lipcache* h, cudaStream_t s) {
@@ -231,6 +251,10 @@ void spectral_norm(lipcache* h, cudaStream_t s) {
                                 tight ? h->inv_pairnorm : nullptr, tight ? h->ipn_up32 : nullptr,
                                 tight ? h->ipn_dn32 : nullptr);
   LC_LAUNCH_CHECK("k_row_norms");
+  if (tight) {
+    k_ipn_min<<<(C + 127) / 128, 128, 0, s>>>(h->pairnorm, h->ipn_dn32, h->ipn_up32, C, h->ipn_min32, h->ipn_max32);
+    LC_LAUNCH_CHECK("k_ipn_min");
+  }
 }
 
 }  // namespace lc

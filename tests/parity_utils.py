@@ -56,14 +56,21 @@ def check_insert(g_index, g_radius, n_acc, ref, head=None):
     assert bad.size == 0, f"{bad.size} rows differ in acceptance/index, first {bad[:5]}"
     r = cert["radius"]
     m = np.isfinite(r) & (r > 0)
-    np.testing.assert_allclose(g_radius[m], r[m], rtol=RTOL)
     if head is None:
         slack = r * 1e-12
     elif isinstance(head[0], str) and head[0] == "tight":
         slack = r * 1e-12 + refine_slack_tight(*head[1:])
     else:
         slack = refine_slack(*head)
-    assert np.all(g_radius[m].astype(np.float64) <= r[m] + slack[m])
+    g = g_radius[m].astype(np.float64)
+    # within 1e-5 relative, or within the refinement's proven absolute error
+    # where that is larger (radii of entries a hair from a decision boundary,
+    # below ~1e-6 of the logit scale); never above the exact radius by more
+    # than that error
+    err = np.abs(g - r[m])
+    bad = np.nonzero(err > RTOL * r[m] + slack[m])[0]
+    assert bad.size == 0, f"{bad.size} radii off, e.g. {g[bad[:3]]} vs {r[m][bad[:3]]}"
+    assert np.all(g <= r[m] + slack[m])
 
 
 def check_probe(gi, gl, gd, ref, Q, orc):

@@ -206,16 +206,16 @@ def test_wide_tile_payload_and_consistency(dev, kernel):
 
 
 def test_kernel_choice(dev):
-    """The conservative radius takes the tensor kernel where it applies
-    (d % 16 == 0, d >= 32, 2 <= C <= 256, head resident); the other shapes
-    and the tight radius take the wide-tile kernel (d % 4 == 0, head small
-    enough), the 64-row one (d % 4 != 0) or the streamed one (large heads)."""
+    """Both radii take the tensor kernel where it applies (d % 16 == 0,
+    32 <= d <= 256, 2 <= C <= 256, head resident); the other shapes take the
+    wide-tile kernel (d % 4 == 0, head small enough), the 64-row one
+    (d % 4 != 0) or the streamed one (large heads)."""
     from paper_2608_13144_gb300.lipcache import LipCache
-    cases = [((64, 10), "tight", WIDE_TILE), ((33, 10), "tight", TILE64), ((33, 10), "conservative", TILE64),
+    cases = [((64, 10), "tight", TENSOR), ((33, 10), "tight", TILE64), ((33, 10), "conservative", TILE64),
              ((256, 200), "conservative", STREAMED), ((128, 300), "conservative", STREAMED),
              ((128, 200), "conservative", TENSOR), ((64, 10), "conservative", TENSOR),
              ((32, 2), "conservative", TENSOR), ((16, 10), "conservative", WIDE_TILE),
-             ((40, 10), "conservative", WIDE_TILE), ((128, 200), "tight", WIDE_TILE),
+             ((40, 10), "conservative", WIDE_TILE), ((128, 200), "tight", TENSOR), ((16, 10), "tight", WIDE_TILE),
              ((96, 256), "conservative", TENSOR), ((128, 256), "conservative", STREAMED)]
     rng = np.random.default_rng(5)
     for (d, C), mode, kernel in cases:
@@ -270,11 +270,14 @@ def test_wide_tile_near_ties(dev, d, C, kernel):
 
 
 def build_tight(dev, W, b, rows, tile64, kappa=1.0):
+    """tile64 as in build(): True, "wide" or False (the library's choice)."""
     from paper_2608_13144_gb300.lipcache import LipCache
     c = LipCache(W.shape[1], W.shape[0], len(rows), "tight", device=dev)
     c.set_radius_scale(kappa)
     c.set_head(T(W, dev), T(b, dev))
-    if tile64:
+    if tile64 == "wide":
+        c.set_debug(DEBUG_INSERT_WIDE_TILE)
+    elif tile64:
         c.set_debug(DEBUG_INSERT_TILE64)
     i, r, n = c.insert(T(rows, dev))
     return c, i.cpu().numpy(), r.cpu().numpy(), n
@@ -295,7 +298,7 @@ def test_wide_tile_tight_radius(dev, d, C, kappa):
     b = (0.1 * rng.standard_normal(C)).astype(np.float32)
     rows = np.concatenate([rng.standard_normal((3000, d)).astype(np.float32) * 2,
                            _near_ties(W, b, 300, rng, 2), _near_ties(W, b, 300, rng, 3)])
-    a, ia, ra, na = build_tight(dev, W, b, rows, False, kappa)
+    a, ia, ra, na = build_tight(dev, W, b, rows, "wide", kappa)
     assert a.info()["last_insert_kernel"] == WIDE_TILE
     s, is_, rs, ns = build_tight(dev, W, b, rows, True, kappa)
     assert s.info()["last_insert_kernel"] in (TILE64, STREAMED)  # FP64 refinement of every class
@@ -310,9 +313,41 @@ def test_wide_tile_tight_radius(dev, d, C, kappa):
     s.close()
 
 
+@pytest.mark.parametrize("d,C,kappa", [(32, 10, 1.0), (64, 40, 0.8), (128, 100, 1.0), (128, 200, 1.0),
+                                       (96, 250, 0.9), (48, 3, 1.0)])
+def test_tensor_tight_radius(dev, d, C, kappa):
+    """The tight radius (Eq. 29) on the tensor kernel: y^G settled by the
+    screen, the candidates of Eq. 29 from the runner-up's bracket and the
+    head's smallest reciprocal pair norm, the same compensated refinement and
+    FP64 terms as the wide-tile kernel; rows on ties take the one-warp path.
+    Acceptance, indices and y^G as the wide-tile kernel and the oracle; radii
+    within the refinement bound of both."""
+    rng = np.random.default_rng(d * 11 + C)
+    W = (rng.standard_normal((C, d)) / np.sqrt(d)).astype(np.float32)
+    b = (0.1 * rng.standard_normal(C)).astype(np.float32)
+    rows = np.concatenate([rng.standard_normal((3000, d)).astype(np.float32) * 2,
+                           _near_ties(W, b, 300, rng, 2), _near_ties(W, b, 300, rng, 3)])
+    a, ia, ra, na = build_tight(dev, W, b, rows, False, kappa)
+    assert a.info()["last_insert_kernel"] == TENSOR and a.info()["device_errors"] == 0
+    s, is_, rs, ns = build_tight(dev, W, b, rows, "wide", kappa)
+    assert s.info()["last_insert_kernel"] == WIDE_TILE
+    ref = oracle.build_cache(W, b, oracle.sigma_max(W), rows, radius_mode=oracle.RADIUS_TIGHT, scale=kappa)
+    check_insert(ia, ra, na, ref, ("tight", W, b, rows, kappa))
+    assert na == ns and np.array_equal(ia, is_)
+    np.testing.assert_array_equal(a.entries()["yG"], s.entries()["yG"])
+    m = np.isfinite(rs) & (rs > 0)
+    slack = refine_slack_tight(W, b, rows, kappa)
+    assert np.all(np.abs(ra[m].astype(np.float64) - rs[m]) <= 1e-6 * rs[m] + 2 * slack[m])
+    print("tight radii bit-identical to the wide-tile kernel:", np.mean(ra.view(np.uint32) == rs.view(np.uint32)),
+          "rows on the one-warp path:", a.info()["insert_full_rows"])
+    a.close()
+    s.close()
+
+
 def test_wide_tile_tight_tied_head_rows(dev):
     """Identical head rows (||W_y - W_j|| = 0, skipped by Eq. 29) and rows won
-    by the tied group (several possible y^G: the FP64 row path)."""
+    by the tied group (several possible y^G: the one-warp row path), on the
+    wide-tile and the tensor kernel."""
     rng = np.random.default_rng(21)
     d, C = 32, 24
     W = (rng.standard_normal((C, d)) / np.sqrt(d)).astype(np.float32)
@@ -322,11 +357,12 @@ def test_wide_tile_tight_tied_head_rows(dev):
     rows = np.concatenate([3 * W[0] + 0.3 * rng.standard_normal((700, d)),
                            3 * W[1] + 0.3 * rng.standard_normal((700, d)),
                            rng.standard_normal((600, d))]).astype(np.float32)
-    a, ia, ra, na = build_tight(dev, W, b, rows, False)
-    assert a.info()["last_insert_kernel"] == WIDE_TILE
-    ref = oracle.build_cache(W, b, oracle.sigma_max(W), rows, radius_mode=oracle.RADIUS_TIGHT)
-    check_insert(ia, ra, na, ref, ("tight", W, b, rows, 1.0))
-    a.close()
+    for kernel, expect in (("wide", WIDE_TILE), (False, TENSOR)):
+        a, ia, ra, na = build_tight(dev, W, b, rows, kernel)
+        assert a.info()["last_insert_kernel"] == expect
+        ref = oracle.build_cache(W, b, oracle.sigma_max(W), rows, radius_mode=oracle.RADIUS_TIGHT)
+        check_insert(ia, ra, na, ref, ("tight", W, b, rows, 1.0))
+        a.close()
 
 
 @pytest.mark.parametrize("d,C,kernel", [(33, 7, TILE64), (21, 40, TILE64), (256, 200, STREAMED), (128, 300, STREAMED)])
@@ -372,7 +408,7 @@ def test_certify_special_values(dev, mode, d, C):
     c.set_head(T(W, dev), T(b, dev))
     i, r, n = c.insert(T(rows, dev))
     i, r = i.cpu().numpy(), r.cpu().numpy()
-    assert c.info()["last_insert_kernel"] == (TENSOR if mode == "conservative" and d >= 32 else WIDE_TILE)
+    assert c.info()["last_insert_kernel"] == (TENSOR if d >= 32 else WIDE_TILE)
     ref = oracle.build_cache(W, b, oracle.sigma_max(W), rows, radius_mode=int(mode == "tight"))
     head = ("tight", W, b, rows, 1.0) if mode == "tight" else (W, b, rows, 1.0)
     finite = np.all(np.isfinite(rows), axis=1)

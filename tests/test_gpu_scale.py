@@ -117,7 +117,7 @@ def test_scale_tight_radius_rows(scale):
         idx.append(i.cpu().numpy())
         rad.append(r.cpu().numpy())
         n += k
-    assert c.info()["last_insert_kernel"] == 1
+    assert c.info()["last_insert_kernel"] == 4  # the tensor certify kernel
     ref = oracle.build_cache(s["W"], s["b"], oracle.sigma_max(s["W"]), rows, radius_mode=oracle.RADIUS_TIGHT)
     check_insert(np.concatenate(idx), np.concatenate(rad), n, ref, ("tight", s["W"], s["b"], rows, 1.0))
     c.close()
