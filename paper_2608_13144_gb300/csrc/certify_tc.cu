@@ -7,8 +7,10 @@
 // tensor memory, and uses the result only as a screen that picks the classes
 // that can be among the true top two; those are recomputed with the same
 // compensated FP32 dot product, in the same order, as the wide-tile kernel, and
-// the FP64 finals are shared. The radii, labels and thresholds therefore come
-// out bit for bit as from the FP32 kernels.
+// the FP64 finals are shared. The conservative radii, labels and thresholds
+// therefore come out bit for bit as from the FP32 kernels; tight radii agree
+// with theirs within the refinement bound (bit for bit wherever both refine
+// y^G and the minimiser in the same order).
 //
 // Screen bound. The MMA returns a_c with |a_c - W_c . z| <= c ||W_c|| ||z||
 // (c = c_screen: TF32 operands within 2^-10 relative, FP32-accurate
@@ -42,15 +44,17 @@
 //   warps 2-9  epilogue, two warps per TMEM lane quarter (32 rows), each
 //              taking every other 32-column chunk of the classes: ||z||^2
 //              (two of its four k-ordered partial chains each) from the tile
-//              in shared memory, the top two s~ and M of its columns,
-//              exchanged with the partner warp; the candidates of its columns
+//              in shared memory and the top two s~ of its columns (with their
+//              classes for the tight radius), exchanged with the partner warp
+//              through a named barrier; then the candidates of its columns
 //              into the warp's pair list. The four groups of 8 lanes refine
 //              the list eight pairs at a time (two per group) into cells by
 //              (row, slot), from which each row's lane takes its own results.
-//              A row with more than kMaxCandTc
-//              candidates in a half, or whose Mb is not below 1e38, has
-//              every class of that half refined. The partner states are merged and
-//              one thread per row runs the FP64 finals.
+//              Conservative radius: a row with more than kMaxCandTc candidates
+//              in a half, or whose Mb is not below 1e38, has every class of
+//              that half refined; the partners' running selections are merged
+//              and one thread per row runs the FP64 finals. Tight radius: see
+//              above; such rows take the one-warp path.
 // Every mbarrier wait is bounded; a role that gives up raises the CTA's abort
 // flag, the others drain, and the launch counts a device error.
 #include "certify_common.cuh"
