@@ -953,12 +953,16 @@ __global__ void __launch_bounds__(kThreads, 1)
           const double vy = (double)v2.x + (double)v2.y;
           const double ey = (double)refined_err(a.g2f, wn_s[yg], hn, bias_s[yg]);
           any_nan = any_nan || !(vy == vy);
-          for (int sl = 0; sl < ns; ++sl) {
+          // unrolled over the slots so that the pair-table loads of all
+          // candidates are in flight together
+#pragma unroll
+          for (int sl = 0; sl < kMaxCandTc; ++sl) {
             const int j = slot_class(sl);
-            if (j == yg) continue;
-            const double vj = (double)res_hi[lane + 32 * sl] + (double)res_lo[lane + 32 * sl];
-            any_nan |= !(vj == vj);
-            tight_term(a, yg, j, vy, ey, vj, (double)refined_err(a.g2f, wn_s[j], hn, bias_s[j]), rmin, smin);
+            if (sl < ns && j != yg) {
+              const double vj = (double)res_hi[lane + 32 * sl] + (double)res_lo[lane + 32 * sl];
+              any_nan |= !(vj == vj);
+              tight_term(a, yg, j, vy, ey, vj, (double)refined_err(a.g2f, wn_s[j], hn, bias_s[j]), rmin, smin);
+            }
           }
         }
         const unsigned fbm = __ballot_sync(kFull, rowfb);
