@@ -177,9 +177,18 @@ lipcache_status lipcache_set_head(lipcache_t* h, const float* W, const float* b,
  *   out_radius  n FP32 (device), nullable; r of every row rounded toward zero
  *               (also for skipped rows)
  *   n_accepted  host, nullable; number of rows appended
- * Synchronises `stream`. All or nothing: if size + n > capacity nothing is
- * written and E_FULL is returned. Errors: E_STATE (no head), E_FULL,
- * E_INVALID, E_CUDA.
+ * With n_accepted given (or a radius policy other than CERTIFIED), synchronises
+ * `stream`. With n_accepted NULL the call is asynchronous on `stream`: the
+ * table's size is kept on the device (each insert takes its first index from
+ * it), out_index / out_radius are valid once the stream reaches them, and the
+ * host learns the size from the next call that needs it (lipcache_size,
+ * get_info, probe, ... synchronise that stream first; an insert on another
+ * stream does too). A device error of an asynchronous insert leaves its rows
+ * out (out_index -1) and shows in lipcache_info.device_errors.
+ * All or nothing: if size + n > capacity nothing is written and E_FULL is
+ * returned (checked against size plus the rows of unsettled asynchronous
+ * inserts, settling them when that bound exceeds the capacity).
+ * Errors: E_STATE (no head), E_FULL, E_INVALID, E_CUDA, E_DEVICE.
  */
 lipcache_status lipcache_insert(lipcache_t* h, const float* H, int64_t n, const int32_t* payload,
                                 int32_t require_consistency, int64_t* out_index, float* out_radius,

@@ -50,6 +50,12 @@ lipcache_status guarded(F&& f) {
 
 void use_device(const lipcache* h) { LC_CUDA(cudaSetDevice(h->device)); }
 
+// The exact table size (after asynchronous inserts), on the cache's device.
+void sync_size(lipcache* h) {
+  use_device(h);
+  lc::settle_size(h);
+}
+
 template <typename T>
 void dev_alloc(T*& p, size_t n) {
   LC_CUDA(cudaMalloc(&p, sizeof(T) * (n ? n : 1)));
@@ -104,6 +110,9 @@ void release(lipcache* h) {
   dev_free(h->ins_bcount);
   dev_free(h->ins_boffset);
   dev_free(h->ins_total);
+  dev_free(h->size_dev);
+  dev_free(h->ins_size0);
+  if (h->size_pinned) cudaFreeHost(h->size_pinned);
   if (h->ins_total_host) cudaFreeHost(h->ins_total_host);
   dev_free(h->qpad);
   dev_free(h->kappa);
@@ -223,6 +232,10 @@ LC_API lipcache_status lipcache_create(int32_t d, int32_t C, int64_t capacity, i
     dev_alloc(h->table.yG, rows);
     dev_alloc(h->ins_total, 4);
     LC_CUDA(cudaMallocHost(&h->ins_total_host, 4 * sizeof(int64_t)));
+    dev_alloc(h->size_dev, 1);
+    LC_CUDA(cudaMemset(h->size_dev, 0, sizeof(int64_t)));
+    dev_alloc(h->ins_size0, 1);
+    LC_CUDA(cudaMallocHost(&h->size_pinned, sizeof(int64_t)));
     dev_alloc(h->stats, 1);
     LC_CUDA(cudaMemset(h->stats, 0, sizeof(lc::DevStats)));
     LC_CUDA(cudaMallocHost(&h->stats_host, sizeof(lc::DevStats)));
@@ -243,7 +256,12 @@ LC_API lipcache_status lipcache_create(int32_t d, int32_t C, int64_t capacity, i
 
 LC_API void lipcache_destroy(lipcache_t* h) { release(h); }
 
-LC_API int64_t lipcache_size(const lipcache_t* h) { return h ? h->size : 0; }
+LC_API int64_t lipcache_size(const lipcache_t* h) {
+  if (!h) return 0;
+  lipcache* m = const_cast<lipcache*>(h);
+  guarded([&] { sync_size(m); });  // on a CUDA error the last settled size is returned
+  return m->size;
+}
 
 LC_API lipcache_status lipcache_set_head(lipcache_t* h, const float* W, const float* b, double* sigma_out,
                                          lipcache_stream_t stream) {
@@ -251,8 +269,8 @@ LC_API lipcache_status lipcache_set_head(lipcache_t* h, const float* W, const fl
     Range nvtx_range("lipcache_set_head");
     check_handle(h);
     LC_REQUIRE(W != nullptr && b != nullptr, LIPCACHE_E_INVALID, "W and b must be device pointers");
+    sync_size(h);
     LC_REQUIRE(h->size == 0, LIPCACHE_E_STATE, "set_head requires an empty cache (radii depend on W)");
-    use_device(h);
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     h->head_set = false;
     h->wt_prep_ncg = 0;
@@ -286,18 +304,31 @@ LC_API lipcache_status lipcache_insert(lipcache_t* h, const float* H, int64_t n,
     LC_REQUIRE(n >= 0, LIPCACHE_E_INVALID, "n must be >= 0");
     if (n == 0) return;
     LC_REQUIRE(H != nullptr, LIPCACHE_E_INVALID, "H is NULL");
-    LC_REQUIRE(n <= h->capacity - h->size, LIPCACHE_E_FULL, "insert would exceed the cache capacity");
     LC_REQUIRE(((uintptr_t)H & 3) == 0, LIPCACHE_E_INVALID, "H must be 4-byte aligned");
     use_device(h);
+    // unsettled asynchronous inserts grew the table by at most pending_rows
+    if (n > h->capacity - h->size - h->pending_rows) lc::settle_size(h);
+    LC_REQUIRE(n <= h->capacity - h->size - h->pending_rows, LIPCACHE_E_FULL, "insert would exceed the cache capacity");
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    if (h->size_pending && s != h->pending_stream) lc::settle_size(h);  // keep every pending insert on one stream
     lc::certify_insert(h, H, n, payload, require_consistency, out_index, out_radius, s);
+    if (n_accepted == nullptr && h->policy == LIPCACHE_POLICY_CERTIFIED) {
+      // asynchronous: nothing to report on the host, so no wait
+      h->size_pending = true;
+      h->pending_rows += n;
+      h->pending_stream = s;
+      return;
+    }
     LC_CUDA(cudaMemcpyAsync(h->ins_total_host, h->ins_total, sizeof(int64_t), cudaMemcpyDeviceToHost, s));
+    LC_CUDA(cudaMemcpyAsync(h->size_pinned, h->size_dev, sizeof(int64_t), cudaMemcpyDeviceToHost, s));
     LC_CUDA(cudaMemcpyAsync(h->stats_host, h->stats, sizeof(lc::DevStats), cudaMemcpyDeviceToHost, s));
     LC_CUDA(cudaStreamSynchronize(s));
+    h->size = *h->size_pinned;  // includes earlier asynchronous inserts on this stream
+    h->size_pending = false;
+    h->pending_rows = 0;
     LC_REQUIRE(h->stats_host->abort_flag == 0, LIPCACHE_E_DEVICE, lc::kCertifyAbortMessage);
     const int64_t acc = *h->ins_total_host;
-    const int64_t first = h->size;
-    h->size += acc;
+    const int64_t first = h->size - acc;
     if (n_accepted) *n_accepted = acc;
     if (h->policy != LIPCACHE_POLICY_CERTIFIED && acc > 0) {
       lc::policy_fill(h, first, acc, s);
@@ -311,6 +342,7 @@ LC_API lipcache_status lipcache_probe(lipcache_t* h, const float* Q, int64_t B, 
   return guarded([&] {
     Range nvtx_range("lipcache_probe");
     check_handle(h);
+    sync_size(h);  // the exact table size (after asynchronous inserts)
     LC_REQUIRE(h->head_set, LIPCACHE_E_STATE, "probe before set_head");
     LC_REQUIRE(B >= 0 && B <= (1LL << 22), LIPCACHE_E_INVALID, "B must be in [0, 2^22]");
     if (B == 0) return;
@@ -329,6 +361,7 @@ LC_API lipcache_status lipcache_insert_select(lipcache_t* h, const float* H, int
   return guarded([&] {
     Range nvtx_range("lipcache_insert_select");
     check_handle(h);
+    sync_size(h);  // the exact table size (after asynchronous inserts)
     LC_REQUIRE(strategy == LIPCACHE_SELECT_ALL || strategy == LIPCACHE_SELECT_RADIUS_DEDUP ||
                    strategy == LIPCACHE_SELECT_KCENTER,
                LIPCACHE_E_INVALID, "unknown selection strategy");
@@ -373,6 +406,7 @@ LC_API lipcache_status lipcache_probe_writeback(lipcache_t* h, const float* Q, i
   return guarded([&] {
     Range nvtx_range("lipcache_probe_writeback");
     check_handle(h);
+    sync_size(h);  // the exact table size (after asynchronous inserts)
     LC_REQUIRE(h->head_set, LIPCACHE_E_STATE, "probe before set_head");
     LC_REQUIRE(B >= 0 && B <= (1LL << 22), LIPCACHE_E_INVALID, "B must be in [0, 2^22]");
     if (B == 0) return;
@@ -407,6 +441,7 @@ LC_API lipcache_status lipcache_consistency(lipcache_t* h, const float* Q, int64
   return guarded([&] {
     Range nvtx_range("lipcache_consistency");
     check_handle(h);
+    sync_size(h);  // the exact table size (after asynchronous inserts)
     LC_REQUIRE(h->head_set, LIPCACHE_E_STATE, "consistency check before set_head");
     LC_REQUIRE(B >= 0 && B <= (1LL << 22), LIPCACHE_E_INVALID, "B must be in [0, 2^22]");
     if (B == 0) return;
@@ -430,6 +465,7 @@ LC_API lipcache_status lipcache_set_radius_policy(lipcache_t* h, int32_t policy,
   return guarded([&] {
     Range nvtx_range("lipcache_set_radius_policy");
     check_handle(h);
+    sync_size(h);  // the exact table size (after asynchronous inserts)
     LC_REQUIRE(h->head_set, LIPCACHE_E_STATE, "set_radius_policy before set_head");
     LC_REQUIRE(policy == LIPCACHE_POLICY_CERTIFIED || policy == LIPCACHE_POLICY_GLOBAL ||
                    policy == LIPCACHE_POLICY_INTERCLASS,
@@ -450,6 +486,7 @@ LC_API lipcache_status lipcache_read_entries(lipcache_t* h, int64_t first, int64
   return guarded([&] {
     Range nvtx_range("lipcache_read_entries");
     check_handle(h);
+    sync_size(h);  // the exact table size (after asynchronous inserts)
     LC_REQUIRE(first >= 0 && n >= 0 && first + n <= h->size, LIPCACHE_E_INVALID, "entries outside [0, size)");
     if (n == 0) return;
     use_device(h);
@@ -499,6 +536,7 @@ LC_API lipcache_status lipcache_probe_host(lipcache_t* h, const float* Q_host, i
   return guarded([&] {
     Range nvtx_range("lipcache_probe_host");
     check_handle(h);
+    sync_size(h);  // the exact table size (after asynchronous inserts)
     LC_REQUIRE(h->head_set, LIPCACHE_E_STATE, "probe before set_head");
     LC_REQUIRE(B >= 0 && B <= (1LL << 22), LIPCACHE_E_INVALID, "B must be in [0, 2^22]");
     if (B == 0) return;
@@ -543,6 +581,7 @@ LC_API lipcache_status lipcache_set_radius_scale(lipcache_t* h, double kappa) {
   return guarded([&] {
     check_handle(h);
     LC_REQUIRE(kappa > 0.0 && kappa <= 1.0, LIPCACHE_E_INVALID, "kappa must be in (0, 1]");
+    sync_size(h);
     LC_REQUIRE(h->size == 0, LIPCACHE_E_STATE, "the radius scale can change only while the cache is empty");
     h->radius_scale = kappa;
   });
@@ -593,7 +632,7 @@ LC_API lipcache_status lipcache_get_info(lipcache_t* h, lipcache_info* info) {
   return guarded([&] {
     check_handle(h);
     LC_REQUIRE(info != nullptr, LIPCACHE_E_INVALID, "info is NULL");
-    use_device(h);
+    sync_size(h);
     LC_CUDA(cudaDeviceSynchronize());
     LC_CUDA(cudaMemcpy(h->stats_host, h->stats, sizeof(lc::DevStats), cudaMemcpyDeviceToHost));
     lc::harvest_timing(h, true);

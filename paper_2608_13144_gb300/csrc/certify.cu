@@ -1282,9 +1282,12 @@ int wt_ncg(int C) {
 }
 
 // Exclusive scan of the per-block accepted counts (one block).
-// (after an aborted certify kernel every count reads as 0: nothing is appended)
+// (after an aborted certify kernel every count reads as 0: nothing is
+// appended). The table's device size gives the insert's base index (size0)
+// and advances by the total.
 __global__ void __launch_bounds__(1024) k_scan(const int32_t* __restrict__ cnt, int32_t* __restrict__ off, int nb,
-                                               int64_t* __restrict__ total, const DevStats* __restrict__ st) {
+                                               int64_t* __restrict__ total, const DevStats* __restrict__ st,
+                                               int64_t* __restrict__ size_dev, int64_t* __restrict__ size0) {
   __shared__ int32_t buf[1024];
   __shared__ int64_t carry;
   const int tid = threadIdx.x;
@@ -1306,12 +1309,20 @@ __global__ void __launch_bounds__(1024) k_scan(const int32_t* __restrict__ cnt, 
     if (tid == 1023) carry += buf[1023];
     __syncthreads();
   }
-  if (tid == 0) *total = carry;
+  if (tid == 0) {
+    *total = carry;
+    const int64_t s0 = *size_dev;
+    *size0 = s0;
+    *size_dev = s0 + carry;
+  }
 }
+
+__global__ void k_set_i64(int64_t* __restrict__ p, int64_t v) { *p = v; }
 
 struct ScatterArgs {
   const float* H;
-  int64_t n, size0;
+  int64_t n;
+  const int64_t* size0;  // device: the insert's base index
   int d, dpad;
   const uint8_t* accept;
   const int32_t* yG;
@@ -1342,7 +1353,7 @@ __global__ void __launch_bounds__(256) k_scatter(ScatterArgs a, int vec) {
   if (lane < kScatterRows && row0 + lane < a.n) {
     const int64_t row = row0 + lane;
     const bool dead = a.st->abort_flag != 0;
-    mydst = (!dead && a.accept[row]) ? a.size0 + a.boff[row / kRows] + a.rank[row] : -1;
+    mydst = (!dead && a.accept[row]) ? *a.size0 + a.boff[row / kRows] + a.rank[row] : -1;
     if (mydst >= 0) {
       a.t.kn[mydst] = a.kn[row];
       a.t.tau[mydst] = a.tau[row];
@@ -1580,12 +1591,12 @@ void certify_insert(lipcache* h, const float* H, int64_t n, const int32_t* paylo
                     int64_t* out_index, float* out_radius, cudaStream_t s, const int64_t* miss_of) {
   launch_certify(h, H, n, payload, require_consistency, miss_of, s);
   const int nb = (int)((n + kRows - 1) / kRows);
-  k_scan<<<1, 1024, 0, s>>>(h->ins_bcount, h->ins_boffset, nb, h->ins_total, h->stats);
+  k_scan<<<1, 1024, 0, s>>>(h->ins_bcount, h->ins_boffset, nb, h->ins_total, h->stats, h->size_dev, h->ins_size0);
   LC_LAUNCH_CHECK("k_scan");
   ScatterArgs sa;
   sa.H = H;
   sa.n = n;
-  sa.size0 = h->size;
+  sa.size0 = h->ins_size0;
   sa.d = h->d;
   sa.dpad = h->dpad;
   sa.accept = h->ins_accept;
@@ -1605,6 +1616,20 @@ void certify_insert(lipcache* h, const float* H, int64_t n, const int32_t* paylo
   const int64_t rows_per_block = 8 * kScatterRows;
   k_scatter<<<(unsigned)((n + rows_per_block - 1) / rows_per_block), 256, 0, s>>>(sa, vec);
   LC_LAUNCH_CHECK("k_scatter");
+}
+
+void store_size_dev(lipcache* h, cudaStream_t s) {
+  k_set_i64<<<1, 1, 0, s>>>(h->size_dev, h->size);
+  LC_LAUNCH_CHECK("k_set_i64");
+}
+
+void settle_size(lipcache* h) {
+  if (!h->size_pending) return;
+  LC_CUDA(cudaMemcpyAsync(h->size_pinned, h->size_dev, sizeof(int64_t), cudaMemcpyDeviceToHost, h->pending_stream));
+  LC_CUDA(cudaStreamSynchronize(h->pending_stream));
+  h->size = *h->size_pinned;
+  h->size_pending = false;
+  h->pending_rows = 0;
 }
 
 void require_certify_ok(lipcache* h, cudaStream_t s) {

@@ -205,6 +205,16 @@ struct lipcache {
   int32_t* ins_boffset = nullptr;
   int64_t* ins_total = nullptr;       // device, 4: rows appended; consistency counts
   int64_t* ins_total_host = nullptr;  // pinned, 4
+  // The table size also lives on the device: k_scan takes an insert's base
+  // index from it and advances it, so inserts chain on their stream without
+  // the host. An insert called without a host count does not wait; `size` is
+  // then settled (synchronising pending_stream) by the next call that needs it.
+  int64_t* size_dev = nullptr;     // device, 1
+  int64_t* ins_size0 = nullptr;    // device, 1: base index of the current insert
+  int64_t* size_pinned = nullptr;  // pinned, 1
+  bool size_pending = false;       // an asynchronous insert is not yet in `size`
+  int64_t pending_rows = 0;        // rows passed to those inserts (bounds their growth)
+  cudaStream_t pending_stream = nullptr;
 
   // probe scratch (grows)
   int64_t q_cap = 0;  // rows (multiple of 128)
@@ -280,6 +290,11 @@ void policy_fill(lipcache* h, int64_t first, int64_t n, cudaStream_t s);
 constexpr const char* kCertifyAbortMessage =
     "a bounded wait of the tensor certify kernel expired; no row was certified or inserted";
 void require_certify_ok(lipcache* h, cudaStream_t s);
+// Bring `size` up to date with asynchronous inserts (synchronises their
+// stream if one is pending), and write the host size to the device counter
+// after a path that grew the table from the host.
+void settle_size(lipcache* h);
+void store_size_dev(lipcache* h, cudaStream_t s);
 void certify_rows(lipcache* h, const float* H, int64_t n, const int32_t* payload, int require_consistency,
                   cudaStream_t s);
 // select.cu: radius-prioritised de-duplication of the certified rows of H

@@ -90,6 +90,15 @@ LC_API lipcache_status lipcache_probe_noalloc(lipcache_t* h, const float* Q, int
                        " bytes (ceil(B/128)*128 rows x (4*d_pad + 12) bytes), the array holds " +
                        std::to_string((long long)LIPCACHE_NOALLOC_SCRATCH_BYTES) + "; use lipcache_probe");
         LC_CUDA(cudaSetDevice(c.h->device));
+        if (c.h->size_pending) {
+          // asynchronous inserts: their size is settled by synchronising their
+          // stream, which a stream being captured into a graph must not do
+          cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+          LC_CUDA(cudaStreamIsCapturing(reinterpret_cast<cudaStream_t>(c.s), &cap));
+          LC_REQUIRE(cap == cudaStreamCaptureStatusNone, LIPCACHE_E_STATE,
+                     "asynchronous inserts are pending: settle them (lipcache_size) before capturing a probe");
+          lc::settle_size(c.h);
+        }
         unsigned char* base = static_cast<unsigned char*>(scratch_address(c.h->device));
         lc::probe_external_scratch(c.h, c.Q, c.B, c.oi, c.ol, c.od, reinterpret_cast<float*>(base + L.qpad),
                                    reinterpret_cast<float*>(base + L.kappa),

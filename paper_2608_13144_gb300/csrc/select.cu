@@ -508,6 +508,7 @@ int64_t select_insert(lipcache* h, const float* H, int64_t n, const int32_t* pay
     h->size += got;
     kept += got;
   }
+  store_size_dev(h, s);  // the table grew from the host
   return kept;
 }
 
@@ -570,6 +571,7 @@ int64_t select_kcenter(lipcache* h, const float* H, int64_t n, const int32_t* pa
   LC_CUDA(cudaStreamSynchronize(s));
   const int64_t kept = x.small_host[1];
   h->size += kept;
+  store_size_dev(h, s);  // the table grew from the host
   return kept;
 }
 

@@ -76,9 +76,12 @@ class LipCache:
         check(self.L.lipcache_set_head(self._h, _ptr(W), _ptr(b), C.byref(sigma), _stream(self.device)))
         return sigma.value
 
-    def insert(self, H: torch.Tensor, payload: torch.Tensor | None = None, require_consistency: bool = False):
+    def insert(self, H: torch.Tensor, payload: torch.Tensor | None = None, require_consistency: bool = False,
+               wait: bool = True):
         """Certify and append rows of H. Returns (index, radius, n_accepted):
-        index[i] is the cache index of row i or -1 if it was skipped."""
+        index[i] is the cache index of row i or -1 if it was skipped. With
+        wait=False the call does not synchronise (n_accepted is None; index
+        and radius are filled in stream order; `size` settles later)."""
         H = self._dev(H, torch.float32, "H")
         n = H.shape[0]
         if H.dim() != 2 or (n and H.shape[1] != self.d):
@@ -89,8 +92,9 @@ class LipCache:
         radius = torch.empty(n, dtype=torch.float32, device=self.device)
         acc = C.c_int64()
         check(self.L.lipcache_insert(self._h, _ptr(H), n, _ptr(payload), int(bool(require_consistency)),
-                                     _ptr(index), _ptr(radius), C.byref(acc), _stream(self.device)))
-        return index, radius, acc.value
+                                     _ptr(index), _ptr(radius), C.byref(acc) if wait else None,
+                                     _stream(self.device)))
+        return index, radius, (acc.value if wait else None)
 
     def insert_select(self, H: torch.Tensor, payload: torch.Tensor | None = None, require_consistency: bool = False,
                       strategy: str = "radius_dedup", budget_total: int = 0, budget_per_class: int = 0):
