@@ -442,10 +442,12 @@ lipcache_status lipcache_get_info(lipcache_t* h, lipcache_info* info);
 /* Zero the candidate / device-error counters and the kernel-time sum. */
 lipcache_status lipcache_reset_stats(lipcache_t* h);
 
-/* Number of cache entries (0 for NULL). */
+/* Number of cache entries (0 for NULL). Settles asynchronous inserts first
+ * (synchronises their stream). */
 int64_t lipcache_size(const lipcache_t* h);
 
-/* Free the cache and its device memory. NULL-safe. */
+/* Free the cache and its device memory, after waiting for asynchronous
+ * inserts still running. NULL-safe. */
 void lipcache_destroy(lipcache_t* h);
 
 /* Message of the last failed call on this thread ("" if none). */

@@ -70,6 +70,8 @@ void dev_free(T*& p) {
 void release(lipcache* h) {
   if (!h) return;
   cudaSetDevice(h->device);
+  // asynchronous inserts may still be writing the table
+  if (h->size_pending) cudaStreamSynchronize(h->pending_stream);
   dev_free(h->W);
   dev_free(h->wt_prep);
   dev_free(h->b);
