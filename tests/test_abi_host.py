@@ -93,3 +93,31 @@ def test_numerics_constants():
         g = (dpad / 32 + 33) * u / (1 - (dpad / 32 + 33) * u)
         assert g < 5e-6
     assert abs((2 * (2 ** -9 + 2 ** -20 + 128 * 2 ** -22)) - 0.00397) < 1e-4
+
+
+def test_info_struct_layout_matches_header(tmp_path):
+    """The binding's ctypes mirror of lipcache_info has the C struct's fields,
+    in order, at the same offsets and with the same size (a C program built
+    against include/lipcache.h prints them)."""
+    import ctypes
+    import shutil
+    import subprocess
+
+    from paper_2608_13144_gb300 import _lib
+
+    cc = shutil.which("gcc") or shutil.which("cc")
+    if cc is None:
+        pytest.skip("no C compiler")
+    names = [f[0] for f in _lib.Info._fields_]
+    src = tmp_path / "layout.c"
+    body = "\n".join(f'  printf("{n} %zu\\n", offsetof(lipcache_info, {n}));' for n in names)
+    src.write_text('#include <stddef.h>\n#include <stdio.h>\n#include "lipcache.h"\nint main(void) {\n'
+                   f'{body}\n  printf("sizeof %zu\\n", sizeof(lipcache_info));\n  return 0;\n}}\n')
+    exe = tmp_path / "layout"
+    include = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include")
+    subprocess.run([cc, "-I", include, str(src), "-o", str(exe)], check=True)
+    out = dict(line.split() for line in subprocess.run([str(exe)], check=True, capture_output=True,
+                                                       text=True).stdout.splitlines())
+    for n in names:
+        assert int(out[n]) == getattr(_lib.Info, n).offset, n
+    assert int(out["sizeof"]) == ctypes.sizeof(_lib.Info)
