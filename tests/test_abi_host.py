@@ -121,3 +121,42 @@ def test_info_struct_layout_matches_header(tmp_path):
     for n in names:
         assert int(out[n]) == getattr(_lib.Info, n).offset, n
     assert int(out["sizeof"]) == ctypes.sizeof(_lib.Info)
+
+
+def test_binding_signatures_match_header():
+    """Every function the binding declares takes, in order, the argument kinds
+    the header's prototype gives (pointer, int32, int64, double)."""
+    import ctypes
+
+    from paper_2608_13144_gb300 import _lib
+
+    L = _lib.load()
+    text = open(os.path.join(ROOT, "include", "lipcache.h")).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    protos = {m.group(2): m.group(3) for m in re.finditer(
+        r"(lipcache_status|int64_t|void|const char\s*\*)\s*(lipcache_\w+)\s*\(([^;]*?)\)\s*;", text, flags=re.S)}
+
+    def c_kind(arg):
+        arg = " ".join(arg.split())
+        if "*" in arg or arg.startswith("lipcache_stream_t"):
+            return "p"
+        for t, k in (("int64_t", "i64"), ("int32_t", "i32"), ("double", "f64")):
+            if arg.startswith(t) or arg.startswith("const " + t):
+                return k
+        raise AssertionError(f"unclassified argument {arg!r}")
+
+    def py_kind(t):
+        if t in (ctypes.c_void_p, ctypes.c_char_p) or (isinstance(t, type) and issubclass(t, ctypes._Pointer)):
+            return "p"
+        return {ctypes.c_int64: "i64", ctypes.c_int32: "i32", ctypes.c_double: "f64"}[t]
+
+    checked = 0
+    for name in _lib.EXPORTS:
+        if name not in protos:
+            continue
+        args = [a for a in protos[name].split(",") if a.strip() and a.strip() != "void"]
+        fn = getattr(L, name)
+        assert fn.argtypes is not None, name
+        assert [c_kind(a) for a in args] == [py_kind(t) for t in fn.argtypes], name
+        checked += 1
+    assert checked >= 20, checked
