@@ -761,7 +761,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           } else {
             // r* <= u_{y2}(y1) if y1 is y^G; for any other possible y^G (its
             // s~ <= l2) r* <= (hi_2 - lo_1) / ||W_y - W_y1|| <= (hi_2 - lo_1)
-            // ipn_max(y1), the pair norms being symmetric
+            // ipn_max(y1), the pair norms being symmetric. When hi_2 = lo_1 and
+            // some W_g = W_y1 that term is 0 x inf = NaN, which fmaxf drops:
+            // such a g is y^G only by tying y1, and its term against y2 has
+            // the pair norm ||W_y1 - W_y2||, so the first term bounds it.
             U1 = fmaxf(__fmul_ru(__fsub_ru(hi1, lo2), __ldg(a.ipn_up32 + (size_t)y * C + j2)),
                        __fmul_ru(__fsub_ru(hi2, lo1), __ldg(a.ipn_max32 + y)));
             lo1 = __fsub_rd(lo1, __fmaf_ru(E, 2.0001f, __fmaf_ru(fabsf(lo1), 9.5367432e-07f /* 2^-20 */, kTinyF)));

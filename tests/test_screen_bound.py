@@ -11,6 +11,12 @@ bit is 1, products of one sign) and FP32 partial sums in either order - and
 check the bound and E. The worst cases reach about a quarter of c, i.e. half
 of the undoubled TF32 term: the factor 2 in c is the safety margin, and a
 bound built on 2^-10 per product instead of 2^-9 would have none left.
+
+The second half emulates the insert kernel's candidate screen for the tight
+radius (Eq. 29) and checks, on adversarial screen errors of up to E, that the
+classes it keeps give the oracle's y^G and r*, including the two corner cases
+of the union test for uncertain rows (a NaN second bound, and a row that needs
+that bound).
 """
 import numpy as np
 import pytest
@@ -104,3 +110,187 @@ def test_insert_screen_E_covers_bias_rounding():
 def test_c_screen_magnitude():
     """c is twice the TF32 product error 2^-9, plus small accumulation terms."""
     assert 2 * 2.0 ** -9 < c_screen(128) < 2 * 2.0 ** -9 * 1.05
+
+
+# ---------------------------------------------------------------------------
+# The tensor insert kernel's candidate screen for the tight radius (Eq. 29),
+# emulated in FP64 (its directed roundings only widen the tests): for screen
+# values s~ with |s~ - s| <= E, the classes it keeps must contain y^G and the
+# minimiser of Eq. 29, so that refining them gives the oracle's y^G and r*.
+
+def pair_tables(W):
+    """FP64 pair norms and the kernel's bracket-table bounds: ipn (1/||W_y -
+    W_j||, +inf for equal rows, as the bracket tables hold), ipn_min(y) over
+    rows that differ from W_y (0 when none), ipn_max(y) over every j != y."""
+    C = W.shape[0]
+    pn = np.linalg.norm(W[:, None, :] - W[None, :, :], axis=2)
+    with np.errstate(divide="ignore"):
+        ipn = np.where(pn > 0, 1.0 / np.where(pn > 0, pn, 1.0), np.inf)
+    ipn_min = np.zeros(C)
+    ipn_max = np.zeros(C)
+    for y in range(C):
+        others = [j for j in range(C) if j != y]
+        nz = [ipn[y, j] for j in others if pn[y, j] > 0]
+        ipn_min[y] = min(nz) if nz else 0.0
+        ipn_max[y] = max(ipn[y, j] for j in others)
+    return pn, ipn, ipn_min, ipn_max
+
+
+def top2_lowest(v):
+    """Top two of v with the lowest index winning ties (the kernel's merges)."""
+    order = sorted(range(len(v)), key=lambda c: (-v[c], c))
+    return order[0], order[1]
+
+
+def screen_tight(st, E, ipn, ipn_min, ipn_max):
+    """Candidate classes of the tight screen, in the kernel's order of tests."""
+    C = len(st)
+    y1, y2 = top2_lowest(st)
+    l1, l2 = st[y1], st[y2]
+    lo1, hi1, lo2, hi2 = l1 - E, l1 + E, l2 - E, l2 + E
+    h = st + E
+    first = (hi1 - lo2) * ipn[y1, y2]
+    with np.errstate(invalid="ignore"):
+        if hi2 < lo1:  # y1 is certainly y^G
+            crude = (lo1 - h) * ipn_min[y1] <= first
+            exact = (lo1 - h) * ipn[y1] <= first
+            cand = crude & exact
+            cand[y1] = True
+            return np.flatnonzero(cand), y1
+        second = (hi2 - lo1) * ipn_max[y1]  # NaN (0 x inf) is dropped, as fmaxf does
+        U = np.fmax(first, second)
+        lo = lo1 - (2.0001 * E + 2.0 ** -20 * abs(lo1))
+        imA = ipn_min.min()
+        cand = (lo - h) * imA <= U
+    return np.flatnonzero(cand), None
+
+
+def refine(s, cand, pn, certain_y):
+    """y^G (largest refined candidate, lowest index on ties) and Eq. 29 over
+    the candidates (equal rows skipped)."""
+    y = certain_y if certain_y is not None else min(cand, key=lambda c: (-s[c], c))
+    terms = [(s[y] - s[j]) / pn[y, j] for j in cand if j != y and pn[y, j] > 0]
+    return y, min(terms) if terms else np.inf
+
+
+def oracle_tight(s, pn):
+    y = top2_lowest(s)[0]
+    terms = [(s[y] - s[j]) / pn[y, j] for j in range(len(s)) if j != y and pn[y, j] > 0]
+    return y, min(terms) if terms else np.inf
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_tight_screen_keeps_the_minimiser(seed):
+    rng = np.random.default_rng(100 + seed)
+    n_unc = 0
+    for trial in range(300):
+        C = int(rng.integers(3, 14))
+        d = int(rng.integers(2, 7))
+        W = rng.standard_normal((C, d))
+        b = rng.standard_normal(C) * 0.3
+        if trial % 3 == 0:  # duplicated head rows (zero pair norms)
+            g, k = sorted(rng.choice(C, 2, replace=False))
+            W[k] = W[g]
+            if trial % 2:
+                b[k] = b[g]
+        pn, ipn, ipn_min, ipn_max = pair_tables(W)
+        z = rng.standard_normal(d)
+        s = W @ z + b
+        spread = float(np.ptp(s)) + 1e-3
+        E = spread * float(rng.choice([1e-4, 1e-2, 0.1, 0.5]))
+        mode = trial % 4
+        if mode == 0:
+            e = rng.uniform(-E, E, C)
+        elif mode == 1:
+            e = rng.choice([-E, E], C)
+        elif mode == 2:  # push the true argmax down and the rest up
+            e = np.full(C, E)
+            e[top2_lowest(s)[0]] = -E
+        else:
+            e = -np.sign(s - s.mean()) * E
+        st = s + e
+        cand, certain = screen_tight(st, E, ipn, ipn_min, ipn_max)
+        n_unc += certain is None
+        y_ref, r_ref = oracle_tight(s, pn)
+        assert y_ref in cand, (seed, trial)
+        y, r = refine(s, cand, pn, certain)
+        assert y == y_ref, (seed, trial, y, y_ref)
+        assert r == r_ref, (seed, trial, r, r_ref)
+    assert n_unc > 20, n_unc  # the union test is exercised
+
+
+def test_tight_screen_nan_bound_case():
+    """Uncertain row with hi_2 = lo_1 exactly and a class g equal to y1 (W and b):
+    the second term of U* is 0 x inf = NaN and dropped. g can then be y^G only
+    by tying y1, and its Eq. 29 term against y2 has the pair norm ||W_y1 - W_y2||,
+    so the first term still bounds r*(g): the screen keeps what Eq. 29 needs."""
+    # dyadic values, so every sum below is exact
+    W = np.array([[1.0, 0.0], [0.25, 0.75], [0.25, 0.75], [-0.5, 0.5], [1.0, -0.75]])
+    b = np.array([0.0, 0.125, 0.125, -0.25, 0.0])
+    z = np.array([0.5, 1.0])
+    s = W @ z + b  # [0.5, 1, 1, 0, -0.25]: classes 1 and 2 are equal and on top
+    g, k, m = 1, 2, 0
+    E = 0.25
+    st = s - E
+    st[k] = s[k] + E  # y1 = 2
+    st[m] = s[m] + E
+    assert st[g] == st[m]  # g ties y2 = 0 on the screen and loses on the index
+    assert np.all(np.abs(st - s) <= E)
+    pn, ipn, ipn_min, ipn_max = pair_tables(W)
+    y1, y2 = top2_lowest(st)
+    assert (y1, y2) == (k, m)
+    hi2, lo1 = st[y2] + E, st[y1] - E
+    assert hi2 == lo1 and np.isinf(ipn_max[y1])
+    cand, certain = screen_tight(st, E, ipn, ipn_min, ipn_max)
+    assert certain is None
+    y_ref, r_ref = oracle_tight(s, pn)
+    assert y_ref == g
+    y, r = refine(s, cand, pn, None)
+    assert (y, r) == (y_ref, r_ref)
+
+
+def test_tight_screen_needs_the_second_term():
+    """Uncertain row whose true y^G (class 2) is neither screen winner, with the
+    Eq. 29 minimiser a far class (3): its term needs U* = (hi_2 - lo_1)
+    ipn_max(y1) (here 3.33 against 2 for u_{y2}(y1)); without that term the
+    screen drops class 3 and the refined r* (3.33) exceeds the true one (3.125).
+    Rows: y1, y2 one apart, class 2 at 0.6 from both, class 3 at 4 from class 2
+    (the largest pair norm, so the head's smallest ipn is 1/4); E = 1."""
+    h = np.sqrt(0.6 ** 2 - 0.25)
+    W = np.array([[-0.5, 0.0], [0.5, 0.0], [0.0, h], [0.0, h - 4.0]])
+    s = np.array([-1.0, -1.0, 1.0, -11.5])  # exact logits (b absorbs W z)
+    E = 1.0
+    st = np.array([0.0, 0.0, 0.0, -12.5])  # every |s~ - s| <= E
+    assert np.all(np.abs(st - s) <= E)
+    pn, ipn, ipn_min, ipn_max = pair_tables(W)
+    assert np.isclose(pn.max(), 4.0) and np.isclose(pn[2, 3], 4.0)
+    y_ref, r_ref = oracle_tight(s, pn)
+    assert y_ref == 2 and np.isclose(r_ref, 12.5 / 4.0)
+    cand, certain = screen_tight(st, E, ipn, ipn_min, ipn_max)
+    assert certain is None and 3 in cand
+    assert refine(s, cand, pn, None) == (y_ref, r_ref)
+    # the first term alone would not keep class 3
+    lo = -1.0 - (2.0001 * E + 2.0 ** -20)
+    assert (lo - (st[3] + E)) * ipn_min.min() > (2.0 * E) * ipn[0, 1]
+
+
+def test_tight_screen_lower_end_slack():
+    """lo* = lo_1 - 2E is wider than soundness needs: any y^G has s >= s_y1 >=
+    lo_1, so the union test with lo_1 (less the refinement's rounding) keeps
+    the minimiser too. Checked on the random cases with lo* = lo_1."""
+    rng = np.random.default_rng(5)
+    for trial in range(400):
+        C = int(rng.integers(3, 12))
+        W = rng.standard_normal((C, 3))
+        s = W @ rng.standard_normal(3) + rng.standard_normal(C) * 0.3
+        E = (float(np.ptp(s)) + 1e-3) * float(rng.choice([1e-2, 0.1, 0.5]))
+        st = s + rng.choice([-E, E], C)
+        pn, ipn, ipn_min, ipn_max = pair_tables(W)
+        y1, y2 = top2_lowest(st)
+        lo1, hi1, lo2, hi2 = st[y1] - E, st[y1] + E, st[y2] - E, st[y2] + E
+        if hi2 < lo1:
+            continue
+        with np.errstate(invalid="ignore"):
+            U = np.fmax((hi1 - lo2) * ipn[y1, y2], (hi2 - lo1) * ipn_max[y1])
+            cand = np.flatnonzero((lo1 - (st + E)) * ipn_min.min() <= U)
+        assert refine(s, cand, pn, None) == oracle_tight(s, pn), trial
