@@ -16,7 +16,11 @@ The second half emulates the insert kernel's candidate screen for the tight
 radius (Eq. 29) and checks, on adversarial screen errors of up to E, that the
 classes it keeps give the oracle's y^G and r*, including the two corner cases
 of the union test for uncertain rows (a NaN second bound, and a row that needs
-that bound).
+that bound). The last part emulates the probe's separable screen with its
+directed roundings and the canonical FP32 recheck distance: every pair the
+recheck would accept passes fl(a - tau_k) >= kappa_q, with about 60 % of the
+slack c |q| |k| left in the worst cases (q near k, every product of one sign,
+dropped bits all ones).
 """
 import numpy as np
 import pytest
@@ -294,3 +298,77 @@ def test_tight_screen_lower_end_slack():
             U = np.fmax((hi1 - lo2) * ipn[y1, y2], (hi2 - lo1) * ipn_max[y1])
             cand = np.flatnonzero((lo1 - (st + E)) * ipn_min.min() <= U)
         assert refine(s, cand, pn, None) == oracle_tight(s, pn), trial
+
+
+# ---------------------------------------------------------------------------
+# The probe's separable screen: a pair is kept iff fl(a - tau_k) >= kappa_q,
+# with kappa_q = RD((1 - c) |q|~^2 / 2), tau_k = RD((RD(1 - c) |k|~^2 -
+# RU(rr_k / (1 - gamma))) / 2) (|.|~^2 the FP32 norms) and a the TF32 product;
+# the recheck accepts iff the canonical FP32 squared distance is below rr_k.
+# Every pair the recheck would accept must pass the screen.
+
+def f32_rd(x):
+    f = np.float32(x)
+    return f if float(f) <= x else np.nextafter(f, np.float32(-np.inf))
+
+
+def f32_ru(x):
+    f = np.float32(x)
+    return f if float(f) >= x else np.nextafter(f, np.float32(np.inf))
+
+
+def fp32_sumsq(x):
+    acc = np.float32(0.0)
+    for v in x.astype(np.float32):
+        acc = np.float32(float(acc) + float(v) * float(v))  # one rounding: a fused multiply-add
+    return acc
+
+
+def dist2_canonical(q, k):
+    """32-wide fused multiply-add chains of the rounded differences, chunk sums
+    added in order (the recheck's canonical distance)."""
+    total = np.float32(0.0)
+    for c in range(0, len(q), 32):
+        p = np.float32(0.0)
+        for j in range(c, c + 32):
+            e = np.float32(np.float32(q[j]) - np.float32(k[j]))
+            p = np.float32(float(p) + float(e) * float(e))
+        total = np.float32(total + p)
+    return total
+
+
+@pytest.mark.parametrize("d", [16, 64, 128, 256])
+def test_probe_screen_keeps_every_acceptable_pair(d):
+    dpad = (d + 31) // 32 * 32
+    c = c_screen(dpad)
+    om_c_rd = np.nextafter(np.float32(1.0 - c), np.float32(0.0))
+    inv_omg_ru = np.nextafter(np.float32(1.0 / (1.0 - gamma32(dpad // 32 + 33))), np.float32(2.0))
+    rng = np.random.default_rng(1000 + d)
+    tightest = np.inf
+    for trial in range(120):
+        q = np.zeros(dpad, np.float32)
+        k = np.zeros(dpad, np.float32)
+        scale = float(rng.choice([1e-3, 1.0, 37.0]))
+        k[:d] = np.abs(worst_mantissa(rng, d, scale))  # every product of one sign
+        if trial % 3 == 0:
+            q[:d] = k[:d]  # distance zero
+        elif trial % 3 == 1:  # a near neighbour, also with dropped bits all ones
+            w = np.abs(worst_mantissa(rng, d, scale))
+            near = (k[:d] + np.float32(0.01) * (w - k[:d])).astype(np.float32)
+            q[:d] = (near.view(np.uint32) | np.uint32(0x1FFF)).view(np.float32)
+        else:  # a different norm: the AM-GM step is loose there
+            q[:d] = (k[:d] * np.float32(rng.uniform(0.5, 2.0))).astype(np.float32)
+        d2 = dist2_canonical(q, k)
+        rr = np.nextafter(d2, np.float32(np.inf))  # the pair is accepted just barely
+        kn, qn = fp32_sumsq(k), fp32_sumsq(q)
+        tau = np.float32(float(f32_rd(float(f32_rd(float(om_c_rd) * float(kn))) -
+                                      float(f32_ru(float(rr) * float(inv_omg_ru))))) * 0.5)
+        kappa = f32_rd((1.0 - c) * float(qn) * 0.5)
+        qk = float(np.linalg.norm(q.astype(np.float64)) * np.linalg.norm(k.astype(np.float64)))
+        for rev in (False, True):
+            a = np.float32(fp32_dot(tf32(q), tf32(k), rev))
+            kept = np.float32(a - tau) >= kappa
+            assert d2 < rr and kept, (d, trial, rev)
+            tightest = min(tightest, (float(np.float32(a - tau)) - float(kappa)) / (c * qk))
+    # not vacuous: the worst case uses a good part of the slack c |q| |k|
+    assert 0.0 <= tightest < 0.8, tightest
