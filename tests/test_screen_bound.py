@@ -12,11 +12,12 @@ check the bound and E. The worst cases reach about a quarter of c, i.e. half
 of the undoubled TF32 term: the factor 2 in c is the safety margin, and a
 bound built on 2^-10 per product instead of 2^-9 would have none left.
 
-The second half emulates the insert kernel's candidate screen for the tight
-radius (Eq. 29) and checks, on adversarial screen errors of up to E, that the
-classes it keeps give the oracle's y^G and r*, including the two corner cases
-of the union test for uncertain rows (a NaN second bound, and a row that needs
-that bound). The last part emulates the probe's separable screen with its
+The second half emulates the insert kernel's candidate screens on
+adversarial screen errors of up to E: the conservative radius's threshold
+l2 - 2E always keeps the true top two, and the tight radius's (Eq. 29)
+bracket and union tests keep what gives the oracle's y^G and r*, including
+the union test's two corner cases for uncertain rows (a NaN second bound,
+and a row that needs that bound). The last part emulates the probe's separable screen with its
 directed roundings and the canonical FP32 recheck distance: every pair the
 recheck would accept passes fl(a - tau_k) >= kappa_q, with about 60 % of the
 slack c |q| |k| left in the worst cases (q near k, every product of one sign,
@@ -372,3 +373,33 @@ def test_probe_screen_keeps_every_acceptable_pair(d):
             tightest = min(tightest, (float(np.float32(a - tau)) - float(kappa)) / (c * qk))
     # not vacuous: the worst case uses a good part of the slack c |q| |k|
     assert 0.0 <= tightest < 0.8, tightest
+
+
+@pytest.mark.parametrize("seed", range(4))
+def test_conservative_screen_keeps_the_top_two(seed):
+    """Conservative radius: with l2 the second-largest screen value, the
+    candidates s~_c >= T = l2 - 2E hold both classes of the true top two (so
+    the refined y^G, runner-up and margin of Eq. 20 are exact), on screen
+    errors of up to E in the adversarial directions."""
+    rng = np.random.default_rng(300 + seed)
+    for trial in range(500):
+        C = int(rng.integers(2, 40))
+        s = rng.standard_normal(C) * float(rng.choice([0.01, 1.0, 100.0]))
+        if trial % 5 == 0:
+            s[rng.integers(C)] = s.max()  # a tie at the top
+        E = (float(np.ptp(s)) + 1e-9) * float(rng.choice([1e-3, 0.05, 0.3]))
+        top = sorted(range(C), key=lambda c: (-s[c], c))[:2]
+        e = rng.choice([-E, E], C)
+        e[top] = -E  # push the true top two down ...
+        e[[c for c in range(C) if c not in top]] = E  # ... and every other class up
+        if trial % 2:
+            e = rng.uniform(-E, E, C)
+        st = s + e
+        l2 = sorted(st)[-2]
+        cand = np.flatnonzero(st >= l2 - 2 * E)
+        assert set(top) <= set(cand.tolist()), (seed, trial)
+        # refining the candidates reproduces y^G and the margin of Eq. 20
+        y = min(cand, key=lambda c: (-s[c], c))
+        runner = max(s[c] for c in cand if c != y)
+        ys = top2_lowest(s)[0]
+        assert y == ys and runner == max(s[c] for c in range(C) if c != ys)
