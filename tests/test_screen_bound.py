@@ -403,3 +403,30 @@ def test_conservative_screen_keeps_the_top_two(seed):
         runner = max(s[c] for c in cand if c != y)
         ys = top2_lowest(s)[0]
         assert y == ys and runner == max(s[c] for c in range(C) if c != ys)
+
+
+@pytest.mark.parametrize("d", [32, 128, 256])
+def test_insert_screen_E_worst_case(d):
+    """E on the worst inputs: head rows and features whose dropped bits are all
+    ones, every product of one sign, FP32 sums in either order, biases of
+    either sign; the worst error uses a good part of E."""
+    rng = np.random.default_rng(40 + d)
+    K = (d + 31) // 32 * 32
+    c = c_screen(K)
+    C = 24
+    z = np.abs(worst_mantissa(rng, d, 2.0))
+    W = np.abs(np.stack([worst_mantissa(rng, d, float(rng.choice([0.05, 1.0]))) for _ in range(C)]))
+    b = (rng.standard_normal(C) * float(np.abs(W @ z).mean())).astype(np.float32)
+    wmax = float(np.linalg.norm(W.astype(np.float64), axis=1).max())
+    hn = float(np.linalg.norm(z.astype(np.float64)))
+    Mb = (1 + c) * wmax * hn + float(np.abs(b).max())
+    E = c * wmax * hn + 2.0 ** -22 * Mb
+    worst = 0.0
+    for j in range(C):
+        s = float(np.dot(W[j].astype(np.float64), z.astype(np.float64))) + float(b[j])
+        for rev in (False, True):
+            a = np.float32(fp32_dot(tf32(W[j]), tf32(z), rev))
+            err = abs(float(np.float32(a + b[j])) - s)
+            assert err <= E, (d, j, err, E)
+            worst = max(worst, err / E)
+    assert worst > 0.1, worst
