@@ -38,6 +38,8 @@ import synth  # noqa: E402
 METRIC = "certified probe queries/s and query-key pairs/s at N=4M; % of HBM/TC roofline"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 TF32_OVER_BF16 = 1.1 / 2.25  # nominal dense TF32 / BF16 tensor rates of GB300
+# LIPCACHE_DEBUG_INSERT_WIDE_TILE / LIPCACHE_DEBUG_INSERT_TILE64 of the C ABI
+INSERT_KERNEL_FLAGS = {"auto": 0, "wide": 4, "tile64": 2}
 
 
 def parse():
@@ -51,6 +53,8 @@ def parse():
     p.add_argument("--cpu-seconds", type=float, default=15.0, help="budget of the oracle CPU baseline")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cache-rows", type=int, default=0, help="override the workload's cache size N (profiling)")
+    p.add_argument("--insert-kernel", default="auto", choices=sorted(INSERT_KERNEL_FLAGS),
+                   help="certify on an FP32 kernel instead of the default choice (profiling)")
     return p.parse_args()
 
 
@@ -270,6 +274,8 @@ def run_ours(args, dist: Dist):
         call; the accepted total comes from the size afterwards), and the
         library's events around each certify kernel."""
         c = LipCache(w.d, w.C, w.N, mode, device=dev)
+        if INSERT_KERNEL_FLAGS[args.insert_kernel]:
+            c.set_debug(INSERT_KERNEL_FLAGS[args.insert_kernel])
         sig = c.set_head(torch.from_numpy(W).to(dev), torch.from_numpy(b).to(dev))
         torch.cuda.synchronize(dev)
         c.enable_timing(True)
