@@ -430,3 +430,20 @@ def test_insert_screen_E_worst_case(d):
             assert err <= E, (d, j, err, E)
             worst = max(worst, err / E)
     assert worst > 0.1, worst
+
+
+def test_probe_chunk_pretest_never_drops_a_kept_pair():
+    """The probe tests each 32-key chunk with fl(max a - min tau) >= kappa before
+    the per-pair test fl(a_j - tau_j) >= kappa: rounding to nearest is monotone,
+    so a chunk holding a kept pair always passes."""
+    rng = np.random.default_rng(77)
+    for trial in range(3000):
+        scale = float(rng.choice([1e-3, 1.0, 1e4]))
+        a = (rng.standard_normal(32) * scale).astype(np.float32)
+        tau = (rng.standard_normal(32) * scale).astype(np.float32)
+        kept = (a - tau).astype(np.float32)
+        kappa = np.float32(kept.max()) if trial % 2 else np.float32(rng.choice(kept))
+        if trial % 3 == 0:
+            kappa = np.nextafter(kappa, np.float32(-np.inf))
+        assert np.any(kept >= kappa)
+        assert np.float32(a.max() - tau.min()) >= kappa, trial
