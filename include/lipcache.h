@@ -334,7 +334,8 @@ lipcache_status lipcache_set_radius_policy(lipcache_t* h, int32_t policy, double
                                            lipcache_stream_t stream);
 
 /*
- * Read back cache entries [first, first + n) (insertion order), e.g. to
+ * Read back cache entries [first, first + n) (insertion order): the triples
+ * (z_i, y~_i, r_i) of the cache (Sec. 3.1), with y^G of each key, e.g. to
  * inspect a cache or to persist it: re-inserting the returned keys with their
  * labels as payload into a cache with the same head rebuilds the same entries.
  *   keys_host    n x d FP32 (host), nullable
@@ -347,7 +348,8 @@ lipcache_status lipcache_read_entries(lipcache_t* h, int64_t first, int64_t n, f
                                       int32_t* label_host, int32_t* yG_host, lipcache_stream_t stream);
 
 /*
- * Copy the head set by lipcache_set_head back to the host (with
+ * Copy the head set by lipcache_set_head, W and b of the affine
+ * classification head (Eq. 5), back to the host (with
  * lipcache_read_entries, what a checkpoint needs: a cache is restored by
  * set_head and re-inserting the entries' keys with their labels as payload,
  * which re-certifies them to the same radii).
@@ -382,8 +384,9 @@ lipcache_status lipcache_read_head(lipcache_t* h, float* W_host, float* b_host, 
 lipcache_status lipcache_set_debug(lipcache_t* h, int32_t flags);
 
 /*
- * lipcache_probe for callers holding HOST buffers: copies Q to the device,
- * probes, copies the results back and synchronises `stream`.
+ * lipcache_probe (Algorithm 2, Eqs. 13-15) for callers holding HOST buffers:
+ * copies Q to the device, probes, copies the results back and synchronises
+ * `stream`.
  *   Q_host     B x d FP32 (host; pinned memory gives asynchronous copies)
  *   out_*_host host, same meaning as lipcache_probe (out_label/out_dist nullable)
  * Returns LIPCACHE_E_DEVICE (outputs written: all misses) if a bounded wait
@@ -414,43 +417,53 @@ lipcache_status lipcache_probe_host(lipcache_t* h, const float* Q_host, int64_t 
 lipcache_status lipcache_probe_noalloc(lipcache_t* h, const float* Q, int64_t B, int64_t* out_index,
                                        int32_t* out_label, float* out_dist, lipcache_stream_t stream);
 
-/* Select the probe kernel (LIPCACHE_PROBE_*). E_INVALID for an unknown path
- * or TENSOR when d > 256. */
+/* Select the probe kernel (LIPCACHE_PROBE_*) that evaluates the lookup of
+ * Algorithm 2 (Eqs. 13-15, the O(Nd) scan of Sec. 3.4 / Eq. 16); every path
+ * returns the same results. E_INVALID for an unknown path or TENSOR when
+ * d > 256. */
 lipcache_status lipcache_set_probe_path(lipcache_t* h, int32_t path);
 
 /* Radius tightening kappa in (0, 1] (Sec. 5.6): radii of rows inserted
  * afterwards are multiplied by kappa. Only while the cache is empty. */
 lipcache_status lipcache_set_radius_scale(lipcache_t* h, double kappa);
 
-/* Spectral-norm options: `squarings` (0..60) normalised squarings of W^T W
- * before the power iteration and `max_iter` (>= 1) power iterations. */
+/* Options of the spectral norm sigma_max(W) (Sec. 4.1, Eqs. 17-19):
+ * `squarings` (0..60) normalised squarings of W^T W before the power
+ * iteration and `max_iter` (>= 1) power iterations. */
 lipcache_status lipcache_set_spectral_options(lipcache_t* h, int32_t squarings, int32_t max_iter);
 
 /* Pre-size the probe scratch for batches of up to max_batch queries so that
- * later probes allocate nothing. */
+ * later probes allocate nothing (memory management of this library; no
+ * counterpart in the paper). */
 lipcache_status lipcache_reserve(lipcache_t* h, int64_t max_batch);
 
-/* When on, each probe times its main kernel (the screen/recheck kernel, not
- * the prologue and finalize) with a pair of CUDA events recorded on `stream`.
- * lipcache_get_info returns the last duration and the sum and count since the
- * last lipcache_reset_stats. */
+/* Instrumentation (no counterpart in the paper). When on, each probe times
+ * its main kernel (the screen/recheck kernel, not the prologue and
+ * finalize), and each certifying call its certify kernel, with a pair of
+ * CUDA events recorded on the call's stream. lipcache_get_info returns the
+ * last probe duration and, for probes and certify kernels, the sum and count
+ * since the last lipcache_reset_stats. */
 lipcache_status lipcache_enable_timing(lipcache_t* h, int32_t on);
 
-/* Fill *info (host). Synchronises the device work of this handle. */
+/* Fill *info (host): sizes, sigma_max (Sec. 4.1), kernels used, counters and
+ * timings (introspection; no counterpart in the paper). Synchronises the
+ * device work of this handle. */
 lipcache_status lipcache_get_info(lipcache_t* h, lipcache_info* info);
 
-/* Zero the candidate / device-error counters and the kernel-time sum. */
+/* Zero the candidate / device-error counters and the kernel-time sum
+ * (instrumentation; no counterpart in the paper). */
 lipcache_status lipcache_reset_stats(lipcache_t* h);
 
-/* Number of cache entries (0 for NULL). Settles asynchronous inserts first
- * (synchronises their stream). */
+/* Number of cache entries |C| (Sec. 3.1; 0 for NULL). Settles asynchronous
+ * inserts first (synchronises their stream). */
 int64_t lipcache_size(const lipcache_t* h);
 
-/* Free the cache and its device memory, after waiting for asynchronous
- * inserts still running. NULL-safe. */
+/* Free the cache C (Sec. 3.1), its head and its device memory, after waiting
+ * for asynchronous inserts still running. NULL-safe. */
 void lipcache_destroy(lipcache_t* h);
 
-/* Message of the last failed call on this thread ("" if none). */
+/* Message of the last failed call on this thread ("" if none; error
+ * reporting of this library, no counterpart in the paper). */
 const char* lipcache_last_error(void);
 
 #ifdef __cplusplus

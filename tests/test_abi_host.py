@@ -160,3 +160,18 @@ def test_binding_signatures_match_header():
         assert [c_kind(a) for a in args] == [py_kind(t) for t in fn.argtypes], name
         checked += 1
     assert checked >= 20, checked
+
+
+def test_every_declaration_cites_its_passage():
+    """Each entry point's documentation (the text since the previous
+    declaration) names the passage of the paper it implements, or says that it
+    has none (options, instrumentation, test hooks)."""
+    text = open(os.path.join(ROOT, "include", "lipcache.h")).read()
+    decls = list(re.finditer(r"(?:lipcache_status|int64_t|void|const char\s*\*)\s*(lipcache_\w+)\s*\([^;]*\)\s*;", text))
+    assert len(decls) >= 20
+    cite = re.compile(r"Sec\.|Eqs?\.|Algorithm|Remark|Lemma|counterpart|not part of the method|Test hooks")
+    prev = 0
+    for m in decls:
+        doc = text[prev:m.start()]
+        assert cite.search(doc), m.group(1)
+        prev = m.end()
