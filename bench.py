@@ -13,9 +13,11 @@ needed between steps.
   python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
   python bench.py --impl reference ...   # FP64 CPU oracle on host cores
 
-Prints one JSON line (rank 0). Under torchrun each rank runs an independent
-replica on its own GPU ("replicas only"; the lookup never exchanges data),
-and the line reports the units of all ranks over the slowest rank's time.
+Prints one JSON line (rank 0). The lookup runs on one GPU: its tensor-core
+probe kernels load query tiles with TMA multicast inside a thread-block
+cluster, which is meant for single-GPU runs only, so the GPU arm refuses to
+start under torchrun with WORLD_SIZE > 1 (exit status 2, one JSON line that
+says why). The reference arm (the CPU oracle) runs on rank 0 alone there.
 """
 from __future__ import annotations
 
@@ -252,6 +254,10 @@ def cpu_baseline(w, W, b, rows, Q, budget_s: float) -> dict:
 
 
 # ---------------------------------------------------------------- our arm
+SINGLE_GPU_ONLY = ("the GPU arm runs on one GPU only: its tensor-core probe kernels use TMA cluster "
+                   "multicast, which is kept to single-GPU runs")
+
+
 def run_ours(args, dist: Dist):
     import torch
 
@@ -368,7 +374,7 @@ def run_ours(args, dist: Dist):
         "data": "synthetic (seeded Gaussian-mixture GuardNet features; no datasets or trained weights)",
         "config": {"workload": w.name, "N": N, "d": w.d, "C": w.C, "batch": B, "radius": "conservative",
                    "probe_path": {2: "exact", 3: "tensor_single", 4: "tensor_pair"}[info["last_probe_path"]],
-                   "parallelism": f"replicas{dist.world}" if dist.world > 1 else "single",
+                   "parallelism": "single",
                    "l2": f"inputs larger than L2 ({N * (4 * info['d_pad'] + 16) / 1e9:.2f} GB key table)"},
         "pairs_per_s": value * N,
         "roofline": rf,
@@ -475,6 +481,11 @@ def main():
             if dist.rank != 0:
                 return
             line = run_reference(args, dist)
+        elif dist.world > 1:
+            if dist.rank == 0:
+                print(json.dumps({"metric": METRIC, "n_gpus": dist.world, "error": SINGLE_GPU_ONLY}), flush=True)
+            print(f"bench.py: {SINGLE_GPU_ONLY}; run it with --gpus 1 and no torchrun", file=sys.stderr)
+            sys.exit(2)
         else:
             line = run_ours(args, dist)
         if dist.rank == 0:

@@ -411,7 +411,10 @@ lipcache_status lipcache_probe_host(lipcache_t* h, const float* Q_host, int64_t 
  * device address (cudaGetSymbolAddress); make that first call before any
  * stream capture. All calls on a device share the array: calls whose GPU work
  * overlaps (other streams, handles or threads on the same device) race on it
- * and must be serialised by the caller.
+ * and must be serialised by the caller. The resolved address is cached for the
+ * life of the process: like every handle, it does not survive a reset of the
+ * device's primary context (cudaDeviceReset); do not call this entry point
+ * after one.
  */
 #define LIPCACHE_NOALLOC_SCRATCH_BYTES 4259840
 lipcache_status lipcache_probe_noalloc(lipcache_t* h, const float* Q, int64_t B, int64_t* out_index,

@@ -111,6 +111,34 @@ def test_golden_three_class():
         assert ct["radius"][0] >= c["radius"][0]
 
 
+def test_golden_radius_tightening():
+    """Sec. 5.6: kappa multiplies the radius itself (not r^2), in both radius
+    modes, after certification: a row's acceptance does not depend on kappa
+    in (0, 1], and a hit needs D < kappa r (strict)."""
+    for case in golden("radius_tightening.json")["cases"]:
+        W, b = np.array(case["W"], np.float32), np.array(case["b"], np.float32)
+        rows = np.array(case["rows"], np.float32)
+        s = oracle.sigma_max(W)
+        assert s == pytest.approx(case["sigma"], rel=1e-15)
+        kappa = case["kappa"]
+        for mode, key in ((oracle.RADIUS_CONSERVATIVE, "radius"), (oracle.RADIUS_TIGHT, "radius_tight")):
+            c = oracle.certify(W, b, s, rows, radius_mode=mode, scale=kappa)
+            assert list(c["accept"]) == case["accept"]
+            np.testing.assert_allclose(c["radius"], case[key], rtol=1e-15, atol=0)
+            # acceptance is the same at kappa = 1 and the radius is kappa times it
+            c1 = oracle.certify(W, b, s, rows, radius_mode=mode)
+            assert list(c1["accept"]) == case["accept"]
+            np.testing.assert_allclose(c["radius"], kappa * c1["radius"], rtol=1e-15, atol=0)
+        if "queries" in case:
+            Q = np.array(case["queries"], np.float32)
+            cache = oracle.build_cache(W, b, s, rows, scale=kappa)
+            out = oracle.probe(cache["keys"], cache["radius"], cache["label"], Q)
+            assert list(out["index"]) == case["expect_index"]
+            cache1 = oracle.build_cache(W, b, s, rows)
+            out1 = oracle.probe(cache1["keys"], cache1["radius"], cache1["label"], Q)
+            assert list(out1["index"]) == case["expect_index_kappa1"]
+
+
 def test_golden_skip_rules():
     g = golden("certify_skip_rules.json")
     t = g["tie"]

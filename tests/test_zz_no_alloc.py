@@ -6,8 +6,10 @@ library instead of scratch grown with cudaMalloc.
 
 Through the C ABI, two calls in a row must return what lipcache_probe returns
 for the same batches (indices and labels exactly, distances within the 1e-5
-relative tolerance of the parity tests), on both probe kernels; batches too
-large for the array must be refused with E_INVALID. This file is collected
+relative tolerance of the parity tests), on every probe kernel, for the
+largest documented batch and a ragged one; nothing may be allocated on a
+fresh handle; batches too large for the array must be refused with
+E_INVALID. This file is collected
 last and also passes on its own in a fresh process.
 """
 import ctypes as C
@@ -52,13 +54,11 @@ def _noalloc(c, Qb, dev):
     return [t.cpu().numpy() for t in out]
 
 
-@pytest.mark.parametrize("path", ["tensor", "exact"])
-def test_noalloc_matches_probe_twice(dev, path):
-    w = synth.WORKLOADS["cifar100"].scaled(N=20000, n_queries=3000)
-    c, Q = _cache(dev, w)
-    c.set_probe_path(path)
+def _compare(c, Q, dev, spans):
+    """Two or more calls in a row on different batches: the no-allocation
+    probe returns what lipcache_probe returns."""
     hits = 0
-    for s, e in [(0, 1500), (1500, 3000)]:  # two calls in a row, different batches
+    for s, e in spans:
         Qb = Q[s:e].contiguous()
         ref = [t.cpu().numpy() for t in c.probe(Qb)]
         got = _noalloc(c, Qb, dev)
@@ -70,6 +70,67 @@ def test_noalloc_matches_probe_twice(dev, path):
         hits += int(hit.sum())
     assert hits > 0
     assert c.info()["device_errors"] == 0
+
+
+@pytest.mark.parametrize("path", ["tensor", "tensor_pair", "exact"])
+def test_noalloc_matches_probe_twice(dev, path):
+    w = synth.WORKLOADS["cifar100"].scaled(N=20000, n_queries=3000)
+    c, Q = _cache(dev, w)
+    c.set_probe_path(path)
+    _compare(c, Q, dev, [(0, 1500), (1500, 3000)])
+    c.close()
+
+
+@pytest.mark.parametrize("path", ["tensor", "tensor_pair"])
+def test_noalloc_largest_batch_and_ragged(dev, path):
+    """d = 256 (d_pad = 256): the documented largest batch, 4,096 queries,
+    fills the array; then a batch of 1,100 queries (padded to 1,152 rows, not
+    a multiple of 256) exercises the kernels' row guards on the array's
+    exactly sized regions."""
+    from paper_2608_13144_gb300 import _lib
+    w = synth.WORKLOADS["tinyimagenet"].scaled(N=20000, n_queries=5196)
+    assert (4096 * (4 * 256 + 12) + 512) <= _lib.NOALLOC_SCRATCH_BYTES
+    c, Q = _cache(dev, w)
+    c.set_probe_path(path)
+    _compare(c, Q, dev, [(0, 4096), (4096, 5196)])
+    c.close()
+
+
+def test_noalloc_allocates_nothing_on_a_fresh_handle(dev):
+    """On a handle whose probe scratch was never grown, the no-allocation
+    probe leaves the device's free memory and torch's allocator unchanged,
+    while an ordinary probe of the same batch then allocates its scratch."""
+    w = synth.WORKLOADS["tinyimagenet"].scaled(N=5000, n_queries=4096)
+    # warm-up on another handle: loads the kernels' modules and resolves the
+    # array's device address, both of which may take device memory once
+    warm, Qw = _cache(dev, w)
+    _noalloc(warm, Qw, dev)
+    warm.probe(Qw)
+    torch.cuda.synchronize(dev)
+    warm.close()
+    c, Q = _cache(dev, w)
+    torch.cuda.synchronize(dev)
+    free0 = torch.cuda.mem_get_info(dev)[0]
+    alloc0 = torch.cuda.memory_stats(dev).get("allocation.all.allocated", 0)
+    out = (torch.empty(4096, dtype=torch.int64, device=dev), torch.empty(4096, dtype=torch.int32, device=dev),
+           torch.empty(4096, dtype=torch.float32, device=dev))
+    alloc1 = torch.cuda.memory_stats(dev).get("allocation.all.allocated", 0)
+    torch.cuda.synchronize(dev)
+    free1 = torch.cuda.mem_get_info(dev)[0]
+    for _ in range(2):
+        st = c.L.lipcache_probe_noalloc(c._h, C.c_void_p(Q.data_ptr()), 4096, C.c_void_p(out[0].data_ptr()),
+                                        C.c_void_p(out[1].data_ptr()), C.c_void_p(out[2].data_ptr()),
+                                        C.c_void_p(torch.cuda.current_stream(dev).cuda_stream))
+        assert st == 0, c.L.lipcache_last_error()
+    torch.cuda.synchronize(dev)
+    assert torch.cuda.mem_get_info(dev)[0] == free1
+    assert torch.cuda.memory_stats(dev).get("allocation.all.allocated", 0) == alloc1
+    assert int((out[0] >= 0).sum()) > 0
+    # the check can see an allocation: the ordinary probe grows ~4 MB of scratch
+    c.probe(Q)
+    torch.cuda.synchronize(dev)
+    assert torch.cuda.mem_get_info(dev)[0] < free1
+    assert alloc1 >= alloc0 and free1 <= free0
     c.close()
 
 
