@@ -54,6 +54,7 @@ def parse():
     p.add_argument("--path", default="auto", choices=["auto", "tensor", "tensor_single", "tensor_pair", "exact"])
     p.add_argument("--cpu-seconds", type=float, default=15.0, help="budget of the oracle CPU baseline")
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-tf32-peak", action="store_true", help="skip the live cuBLAS TF32 peak measurement")
     p.add_argument("--cache-rows", type=int, default=0, help="override the workload's cache size N (profiling)")
     p.add_argument("--insert-kernel", default="auto", choices=sorted(INSERT_KERNEL_FLAGS),
                    help="certify on an FP32 kernel instead of the default choice (profiling)")
@@ -192,6 +193,54 @@ def roofline(w: synth.Workload, N: int, B: int, kernel_ms: float, pk: dict, pk_k
             "peak_source": f"{pk_kind} copy bandwidth", "kernel": kernel, "kernel_ms": kernel_ms}
 
 
+def measure_tf32_peak(dev, n: int = 8192, reps: int = 10, sustain_s: float = 2.0) -> dict:
+    """Dense TF32 tensor throughput of this GPU, measured in this run the way
+    the BF16 peak of MEASURED_PEAKS.json was: a cuBLAS (torch.matmul) FP32 GEMM
+    with TF32 tensor cores allowed, n^3 with n = 8192 (2 n^3 flops), best of
+    `reps` timed with CUDA events (burst), then back to back for `sustain_s`
+    seconds (sustained), with nvidia-smi clocks sampled meanwhile. A
+    measurement for the roofline only; the lookup never calls cuBLAS."""
+    import torch
+    prev = torch.backends.cuda.matmul.allow_tf32
+    torch.backends.cuda.matmul.allow_tf32 = True
+    try:
+        g = torch.Generator(device=dev).manual_seed(1)
+        a = torch.randn(n, n, device=dev, generator=g)
+        b = torch.randn(n, n, device=dev, generator=g)
+        c = torch.empty(n, n, device=dev)
+        for _ in range(3):
+            torch.matmul(a, b, out=c)
+        torch.cuda.synchronize(dev)
+        clk = Clocks(dev.index)
+        clk.mark_start()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        best = float("inf")
+        for _ in range(reps):
+            e0.record()
+            torch.matmul(a, b, out=c)
+            e1.record()
+            torch.cuda.synchronize(dev)
+            best = min(best, e0.elapsed_time(e1) * 1e-3)
+        k, t0 = 0, time.perf_counter()
+        e0.record()
+        while time.perf_counter() - t0 < sustain_s:
+            for _ in range(10):
+                torch.matmul(a, b, out=c)
+            k += 10
+            torch.cuda.synchronize(dev)
+        e1.record()
+        torch.cuda.synchronize(dev)
+        sustained = 2.0 * n ** 3 * k / (e0.elapsed_time(e1) * 1e-3) / 1e12
+        clk.mark_end()
+        clocks = clk.stop()
+        del a, b, c
+        return {"burst_tflops": 2.0 * n ** 3 / best / 1e12, "sustained_tflops": sustained, "clocks": clocks,
+                "how": f"torch.matmul FP32 {n}^3 with TF32 tensor cores (cuBLAS): best of {reps} (burst), "
+                       f"back to back for {sustain_s:.0f} s (sustained)"}
+    finally:
+        torch.backends.cuda.matmul.allow_tf32 = prev
+
+
 # main probe kernel per path: name, ncu summary, the sources its hash covers
 INSERT_KERNELS = {1: "k_certify_wt", 2: "k_certify_wres", 3: "k_certify", 4: "k_certify_tc"}
 PROBE_KERNELS = {
@@ -295,7 +344,8 @@ def run_ours(args, dist: Dist):
         inf = c.info()
         c.enable_timing(False)
         kern = (INSERT_KERNELS.get(inf["last_insert_kernel"], "?"), inf["insert_kernel_ms_total"],
-                inf["insert_kernel_launches"], inf["insert_refined_pairs"], inf["insert_full_rows"])
+                inf["insert_kernel_launches"], inf["insert_refined_pairs"], inf["insert_full_rows"],
+                inf["insert_fp64_rows"])
         return c, sig, acc, e0.elapsed_time(e1), kern
 
     # the tight radius (Eq. 29, Sec. 5.6) on the same rows, then the
@@ -365,6 +415,12 @@ def run_ours(args, dist: Dist):
 
     path_id = info["last_probe_path"]
     rf = roofline(w, N, B, kernel_ms, pk, pk_kind, PROBE_KERNELS[path_id][0])
+    if rf["bound"] == "tensor" and not args.no_tf32_peak:
+        # the TF32 peak measured live beside the derived one (MEASURED_PEAKS.json holds BF16 only)
+        tf = measure_tf32_peak(dev)
+        tf["frac_of_burst"] = rf["achieved"] / tf["burst_tflops"]
+        tf["frac_of_sustained"] = rf["achieved"] / tf["sustained_tflops"]
+        rf["tf32_measured"] = tf
     if path_id in (3, 4) and w.N == synth.WORKLOADS[w.name].N:
         rf["traffic"] = recorded_traffic(w.name, path_id)
     line = {
@@ -417,7 +473,8 @@ def insert_summary(w, n_acc, insert_ms, sms, clocks, kernel=None, tf32_peak=None
            "batch": w.insert_batch,
            "e2e": {"achieved": e2e, "unit": "TFLOP/s", "frac_alu": e2e / alu_peak}}
     if kernel and kernel[2] > 0:
-        name, k_ms_total, launches, pairs, full_rows = kernel
+        name, k_ms_total, launches, pairs, full_rows, fp64_rows = kernel
+        out["rows_fp64_pass"] = fp64_rows
         achieved = flops / (k_ms_total * 1e-3) / 1e12
         out["kernel"] = name
         out["kernel_ms"] = k_ms_total / launches

@@ -130,6 +130,9 @@ typedef struct lipcache_info {
                                    product) since the last reset */
   int64_t insert_full_rows;     /* row halves it refined over every class of the half (more candidates
                                    than slots, a NaN logit or an unbounded screen error) */
+  int64_t insert_fp64_rows;     /* rows re-certified in FP64 since the last reset: rows whose margin (or
+                                   minimising term of Eq. 29) the compensated FP32 refinement could not
+                                   pin to 5e-6 relative */
 } lipcache_info;
 
 /*

@@ -38,7 +38,7 @@ class Info(C.Structure):
                 ("last_cluster", C.c_int32), ("radius_policy", C.c_int32), ("last_insert_kernel", C.c_int32),
                 ("policy_param", C.c_double), ("insert_kernel_ms_total", C.c_double),
                 ("insert_kernel_launches", C.c_int64), ("insert_refined_pairs", C.c_int64),
-                ("insert_full_rows", C.c_int64)]
+                ("insert_full_rows", C.c_int64), ("insert_fp64_rows", C.c_int64)]
 
 
 class LipCacheError(RuntimeError):

@@ -109,6 +109,7 @@ void release(lipcache* h) {
   dev_free(h->ins_kn);
   dev_free(h->ins_tau);
   dev_free(h->ins_rank);
+  dev_free(h->ins_fix);
   dev_free(h->ins_bcount);
   dev_free(h->ins_boffset);
   dev_free(h->ins_total);
@@ -656,6 +657,7 @@ LC_API lipcache_status lipcache_get_info(lipcache_t* h, lipcache_info* info) {
     info->device_errors = (int64_t)h->stats_host->errors;
     info->insert_refined_pairs = (int64_t)h->stats_host->ins_pairs;
     info->insert_full_rows = (int64_t)h->stats_host->ins_full_rows;
+    info->insert_fp64_rows = (int64_t)h->stats_host->ins_fp64_rows;
     info->probe_path = h->probe_path;
     info->last_probe_path = h->last_probe_path;
     info->last_probe_ms = h->last_ms;

@@ -1281,17 +1281,214 @@ int wt_ncg(int C) {
   return need <= 1 ? 1 : need <= 4 ? 4 : need <= 7 ? 7 : need <= 13 ? 13 : need <= 16 ? 16 : 0;
 }
 
+// ---------------------------------------------------------------- FP64 pass
+// Re-certification in FP64 of the rows the compensated FP32 refinement could
+// not pin down (listed by row_finals / tight_write: a margin, or a minimising
+// term of Eq. 29, smaller than 1 / kFixRel times its error bound - rows a hair
+// from a decision boundary, about 0.3 % of the rows of the scale workload).
+// One warp per listed row: the row's FP32 logits (plain fused multiply-add
+// chains) with their error bounds pick the classes that can matter, which are
+// recomputed in FP64 (products of FP32 values are exact in FP64, so the sum's
+// error is gamma_{d+8} of the sum of |products|); y^G, the margin or Eq. 29,
+// the certified lower bound, the thresholds and the skip rules of Algorithm 1
+// are then taken from the FP64 values and overwrite the row's results.
+// Conservative radius: the candidates are the classes whose FP32 interval
+// reaches the second-largest lower end, which include the true top two.
+// Tight radius: the possible y^G (intervals reaching the largest lower end),
+// then, for the FP64 y^G, the classes whose lower bracket of
+// (s_y - s_j) / ||W_y - W_j|| reaches the smallest upper bracket, which
+// include the minimiser of Eq. 29.
+constexpr int kFixWarps = 4;
+
+// FP64 logit of class c for the row in shared memory (the whole warp), with
+// the rounding bound g64 (sum |W_cj z_j| + |b_c|); every lane gets the values.
+__device__ __forceinline__ void logit_fp64(const CertArgs& a, int c, const float* __restrict__ zs, int lane, double& v,
+                                           double& e) {
+  const float* wc = a.W + (size_t)c * a.d;
+  double p = 0.0, pa = 0.0;
+  for (int j = lane; j < a.d; j += 32) {
+    const double t = (double)__ldg(wc + j) * (double)zs[j];
+    p += t;
+    pa += fabs(t);
+  }
+  p = warp_sum_d(p);
+  pa = warp_sum_d(pa);
+  const double bc = (double)__ldg(a.b + c);
+  v = p + bc;
+  e = __dmul_ru(a.g64, __dadd_ru(pa, fabs(bc)));
+}
+
+__global__ void __launch_bounds__(kFixWarps * 32) k_certify_fix(const CertArgs a, DevStats* stats) {
+  extern __shared__ __align__(16) float fix_smem[];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int d = a.d, C = a.C;
+  float* zs = fix_smem + (size_t)warp * (size_t)(d + 2 * C);
+  float* sv = zs + d;   // FP32 logits
+  float* ev = sv + C;   // their error bounds
+  const int nfix = *a.fix_count;
+  if (blockIdx.x == 0 && threadIdx.x == 0 && nfix > 0) atomicAdd(&stats->ins_fp64_rows, (unsigned long long)nfix);
+  for (int k = blockIdx.x * kFixWarps + warp; k < nfix; k += gridDim.x * kFixWarps) {
+    const int64_t row = a.fix_list[k];
+    const float* z = a.H + (size_t)row * d;
+    __syncwarp();  // the previous row's reads of this warp's shared memory are done
+    for (int j = lane; j < d; j += 32) zs[j] = __ldg(z + j);
+    __syncwarp();
+    const float kn = a.kn[row];
+    const float hn = norm_upper(kn);
+    if (!(hn < INFINITY)) continue;  // no finite bounds: keep the FP32 kernel's result
+    // FP32 logits and the top two lower ends of their intervals
+    double l1 = -INFINITY, l2 = -INFINITY;
+    bool nan = false;
+    for (int c = lane; c < C; c += 32) {
+      const float* wc = a.W + (size_t)c * d;
+      float p = 0.f;
+      for (int j = 0; j < d; ++j) p = fmaf(__ldg(wc + j), zs[j], p);
+      const float bc = __ldg(a.b + c);
+      const float s = __fadd_rn(p, bc);
+      const float e = logit_err(a.g32f, __ldg(a.Wnorm32 + c), hn, bc, s);
+      sv[c] = s;
+      ev[c] = e;
+      nan |= !(s == s);
+      top2_push(l1, l2, __dsub_rd((double)s, (double)e));
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const double o1 = __shfl_xor_sync(kFull, l1, o), o2 = __shfl_xor_sync(kFull, l2, o);
+      double t1 = l1, t2 = l2;
+      top2_push(t1, t2, o1);
+      top2_push(t1, t2, o2);
+      l1 = t1;
+      l2 = t2;
+    }
+    if (__any_sync(kFull, nan)) continue;  // keep the FP32 kernel's result (a rejected row)
+    __syncwarp();
+    // FP64 values of the candidate classes, in ascending class order (strict
+    // comparisons keep the lowest class on ties)
+    const double Lc = a.tight ? l1 : l2;
+    double b1 = -INFINITY, b2 = -INFINITY, e1 = 0.0, u1 = -INFINITY, u2 = -INFINITY;
+    int y = -1, cu1 = -1;
+    for (int cb = 0; cb < C; cb += 32) {
+      const int c = cb + lane;
+      const bool cand = c < C && __dadd_ru((double)sv[c], (double)ev[c]) >= Lc;
+      unsigned m = __ballot_sync(kFull, cand);
+      while (m) {
+        const int cc = cb + __ffs(m) - 1;
+        m &= m - 1;
+        double v, e;
+        logit_fp64(a, cc, zs, lane, v, e);
+        if (v > b1) {
+          b2 = b1;
+          b1 = v;
+          e1 = e;
+          y = cc;
+        } else if (v > b2) {
+          b2 = v;
+        }
+        const double up = __dadd_ru(v, e);
+        if (up > u1) {
+          u2 = u1;
+          u1 = up;
+          cu1 = cc;
+        } else if (up > u2) {
+          u2 = up;
+        }
+      }
+    }
+    if (y < 0) continue;
+    if (!a.tight) {
+      const double mval = b1 - b2;
+      const double mlo = __dsub_rd(__dsub_rd(b1, e1), cu1 == y ? u2 : u1);
+      const double r64 = mval * a.inv_denom;
+      const double rs = (mlo > 0.0) ? __dmul_rd(mlo, a.inv_denom_safe) : 0.0;
+      if (lane == 0) {
+        const int32_t lab = a.payload ? a.payload[row] : y;
+        const bool acc =
+            !(a.require_consistency && lab != y) && (r64 > 0.0) && !(a.miss_of && a.miss_of[row] >= 0);
+        float rr, tau;
+        thresholds(__double2float_rd(rs), kn, a.tc, rr, tau);
+        a.accept[row] = acc ? 1 : 0;
+        a.yG[row] = y;
+        a.label[row] = lab;
+        a.radius[row] = __double2float_rz(r64);
+        a.rr[row] = rr;
+        a.tau[row] = tau;
+      }
+    } else {
+      // Eq. 29 for the FP64 y^G: brackets of every term from the FP32 logits,
+      // then FP64 for the classes that can be the minimiser
+      const double vy = b1, ey = e1;
+      double U = INFINITY;
+      for (int j = lane; j < C; j += 32) {
+        if (j == y || !(a.pairnorm[(size_t)y * C + j] > 0.0)) continue;
+        const double ipn = a.inv_pairnorm[(size_t)y * C + j] * (1.0 + 1e-12);
+        U = fmin(U, __dmul_ru(__dsub_ru(__dadd_ru(vy, ey), __dsub_rd((double)sv[j], (double)ev[j])), ipn));
+      }
+      U = warp_min_d(U);
+      double rmin = INFINITY, smin = INFINITY;
+      for (int cb = 0; cb < C; cb += 32) {
+        const int j = cb + lane;
+        bool cand = false;
+        if (j < C && j != y && a.pairnorm[(size_t)y * C + j] > 0.0) {
+          const double ipn = a.inv_pairnorm[(size_t)y * C + j] * (1.0 - 1e-12);
+          cand = __dmul_rd(__dsub_rd(__dsub_rd(vy, ey), __dadd_ru((double)sv[j], (double)ev[j])), ipn) <= U;
+        }
+        unsigned m = __ballot_sync(kFull, cand);
+        while (m) {
+          const int jj = cb + __ffs(m) - 1;
+          m &= m - 1;
+          double v, e;
+          logit_fp64(a, jj, zs, lane, v, e);
+          tight_term(a, y, jj, vy, ey, v, e, rmin, smin);
+        }
+      }
+      if (lane == 0) {
+        const double r64 = a.kappa * rmin;
+        const double rs = smin > 0.0 ? __dmul_rd(a.kappa, smin) : 0.0;
+        const int32_t lab = a.payload ? a.payload[row] : y;
+        const bool acc =
+            !(a.require_consistency && lab != y) && (r64 > 0.0) && !(a.miss_of && a.miss_of[row] >= 0);
+        float rr, tau;
+        thresholds(__double2float_rd(rs), kn, a.tc, rr, tau);
+        a.accept[row] = acc ? 1 : 0;
+        a.yG[row] = y;
+        a.label[row] = lab;
+        a.radius[row] = __double2float_rz(r64);
+        a.rr[row] = rr;
+        a.tau[row] = tau;
+      }
+    }
+    __syncwarp();
+  }
+}
+
+size_t fix_smem_bytes(int d, int C) { return sizeof(float) * (size_t)kFixWarps * (size_t)(d + 2 * C); }
+
 // Exclusive scan of the per-block accepted counts (one block).
 // (after an aborted certify kernel every count reads as 0: nothing is
 // appended). The table's device size gives the insert's base index (size0)
 // and advances by the total.
-__global__ void __launch_bounds__(1024) k_scan(const int32_t* __restrict__ cnt, int32_t* __restrict__ off, int nb,
+__global__ void __launch_bounds__(1024) k_scan(int32_t* __restrict__ cnt, int32_t* __restrict__ off, int nb,
                                                int64_t* __restrict__ total, const DevStats* __restrict__ st,
-                                               int64_t* __restrict__ size_dev, int64_t* __restrict__ size0) {
+                                               int64_t* __restrict__ size_dev, int64_t* __restrict__ size0,
+                                               const int32_t* __restrict__ fix_list, const uint8_t* __restrict__ accept,
+                                               int32_t* __restrict__ rank, int64_t n) {
   __shared__ int32_t buf[1024];
   __shared__ int64_t carry;
   const int tid = threadIdx.x;
   if (tid == 0) carry = 0;
+  // the FP64 pass may have changed a listed row's acceptance: recount its
+  // 32-row block (rows listed twice in a block write the same values)
+  const int nfix = st->fix_count;
+  for (int k = tid; k < nfix; k += 1024) {
+    const int64_t r0 = (int64_t)(fix_list[k] / kRows) * kRows;
+    const int64_t r1 = r0 + kRows < n ? r0 + kRows : n;
+    int c = 0;
+    for (int64_t r = r0; r < r1; ++r) {
+      rank[r] = c;
+      c += accept[r] ? 1 : 0;
+    }
+    cnt[r0 / kRows] = c;
+  }
   __syncthreads();
   for (int base = 0; base < nb; base += 1024) {
     const int i = base + tid;
@@ -1444,6 +1641,7 @@ void ensure_insert_scratch(lipcache* h, int64_t n) {
   grow(h->ins_kn, cap);
   grow(h->ins_tau, cap);
   grow(h->ins_rank, cap);
+  grow(h->ins_fix, cap);
   grow(h->ins_bcount, nb);
   grow(h->ins_boffset, nb);
   h->ins_cap = cap;
@@ -1475,8 +1673,9 @@ int timing_begin(lipcache* h, cudaStream_t s) {
 void launch_certify(lipcache* h, const float* H, int64_t n, const int32_t* payload, int require_consistency,
                     const int64_t* miss_of, cudaStream_t s) {
   ensure_insert_scratch(h, n);
-  // raised by the tensor kernel if one of its bounded waits expires
-  LC_CUDA(cudaMemsetAsync(&h->stats->abort_flag, 0, sizeof(int), s));
+  // the abort flag (raised by the tensor kernel if one of its bounded waits
+  // expires) and the FP64 pass's row count
+  LC_CUDA(cudaMemsetAsync(&h->stats->abort_flag, 0, 2 * sizeof(int), s));
   CertArgs a;
   a.H = H;
   a.n = n;
@@ -1523,6 +1722,8 @@ void launch_certify(lipcache* h, const float* H, int64_t n, const int32_t* paylo
   a.tau = h->ins_tau;
   a.rank = h->ins_rank;
   a.bcount = h->ins_bcount;
+  a.fix_count = &h->stats->fix_count;
+  a.fix_list = h->ins_fix;
   const int nb = (int)((n + kRows - 1) / kRows);
   const int Cp = (h->C + 7) / 8 * 8;
   const size_t smem_wres = sizeof(float) * ((size_t)h->dpad * Cp + (size_t)h->dpad * kHStride +
@@ -1579,6 +1780,14 @@ void launch_certify(lipcache* h, const float* H, int64_t n, const int32_t* paylo
     LC_LAUNCH_CHECK("k_certify");
     h->last_insert_kernel = LIPCACHE_INSERT_STREAMED;
   }
+  // the FP64 pass over the rows the kernel listed (usually a few per thousand;
+  // none from the kernels that refine in FP64 already)
+  {
+    const size_t fsm = fix_smem_bytes(h->d, h->C);
+    if (fsm > 48 * 1024) LC_CUDA(cudaFuncSetAttribute(k_certify_fix, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)fsm));
+    k_certify_fix<<<h->num_sms, kFixWarps * 32, fsm, s>>>(a, h->stats);
+    LC_LAUNCH_CHECK("k_certify_fix");
+  }
   if (slot >= 0) {
     LC_CUDA(cudaEventRecord(h->tev1[slot], s));
     ++h->t_issued;
@@ -1591,7 +1800,8 @@ void certify_insert(lipcache* h, const float* H, int64_t n, const int32_t* paylo
                     int64_t* out_index, float* out_radius, cudaStream_t s, const int64_t* miss_of) {
   launch_certify(h, H, n, payload, require_consistency, miss_of, s);
   const int nb = (int)((n + kRows - 1) / kRows);
-  k_scan<<<1, 1024, 0, s>>>(h->ins_bcount, h->ins_boffset, nb, h->ins_total, h->stats, h->size_dev, h->ins_size0);
+  k_scan<<<1, 1024, 0, s>>>(h->ins_bcount, h->ins_boffset, nb, h->ins_total, h->stats, h->size_dev, h->ins_size0,
+                            h->ins_fix, h->ins_accept, h->ins_rank, n);
   LC_LAUNCH_CHECK("k_scan");
   ScatterArgs sa;
   sa.H = H;

@@ -39,7 +39,18 @@ struct CertArgs {
   float* tau;
   int32_t* rank;
   int32_t* bcount;
+  // rows whose radius the compensated FP32 refinement cannot pin to kFixRel
+  // relative: listed here for the FP64 pass (k_certify_fix); nullable
+  int* fix_count;
+  int32_t* fix_list;
 };
+
+// Relative accuracy the reported radius must reach without the FP64 pass: a
+// row whose margin (conservative radius) or minimising term of Eq. 29 (tight
+// radius) is not known to within this fraction from the compensated FP32
+// refinement's error bounds is re-certified in FP64. Half of the 1e-5 the
+// radii are compared at, leaving room for the FP32 rounding of the result.
+constexpr double kFixRel = 5e-6;
 
 // The tensor-core certify kernel (certify_tc.cu): whether it takes this
 // insert (either radius, d % 16 == 0, 32 <= d <= 256, 2 <= C <= 256, rows
@@ -223,6 +234,11 @@ __device__ void row_finals(const CertArgs& a, int64_t row, const RowVals& v, uin
   const double rs = (mlo > 0.0) ? __dmul_rd(mlo, a.inv_denom_safe) : 0.0;
   const int32_t lab = a.payload ? a.payload[row] : v.y;
   const bool acc = !(a.require_consistency && lab != v.y) && (r64 > 0.0) && !(a.miss_of && a.miss_of[row] >= 0);
+  // The margin is known to within e1 + 2 (up - v2) (the best class's bound and
+  // the width of the runner-up's interval); where that is not below kFixRel m,
+  // the row goes to the FP64 pass, which rewrites everything below.
+  if (a.fix_list && mval == mval && !(mval * kFixRel > (double)v.e1 + 2.0 * ((double)v.up - v2)))
+    a.fix_list[atomicAdd(a.fix_count, 1)] = (int32_t)row;
   float rr, tau;
   thresholds(__double2float_rd(rs), v.kn, a.tc, rr, tau);
   a.accept[row] = acc ? 1 : 0;
@@ -257,6 +273,11 @@ __device__ void tight_write(const CertArgs& a, int64_t row, int y, double rmin, 
   const double rs = (smin > 0.0 && !any_nan) ? __dmul_rd(a.kappa, smin) : 0.0;
   const int32_t lab = a.payload ? a.payload[row] : y;
   const bool acc = !(a.require_consistency && lab != y) && (r64 > 0.0) && !(a.miss_of && a.miss_of[row] >= 0);
+  // rmin - smin bounds the error of rmin (smin is the certified lower bound
+  // of the same minimum); rows where it is not below kFixRel rmin (a near
+  // tie for y^G or a tiny term of Eq. 29) go to the FP64 pass
+  if (a.fix_list && !any_nan && rmin < INFINITY && !((rmin - smin) < kFixRel * rmin))
+    a.fix_list[atomicAdd(a.fix_count, 1)] = (int32_t)row;
   float rr, tau;
   thresholds(__double2float_rd(rs), kn, a.tc, rr, tau);
   a.accept[row] = acc ? 1 : 0;

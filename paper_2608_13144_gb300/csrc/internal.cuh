@@ -114,9 +114,10 @@ struct DevStats {
   unsigned long long candidates;
   unsigned long long errors;
   int abort_flag;  // set by a kernel whose bounded wait expired; cleared per probe
-  int pad;
+  int fix_count;   // rows of the current certification listed for the FP64 pass (cleared per certification)
   unsigned long long ins_pairs;      // (row, class) pairs refined by the tensor certify kernel
   unsigned long long ins_full_rows;  // row halves it refined over every class
+  unsigned long long ins_fp64_rows;  // rows re-certified by the FP64 pass
 };
 
 // Scratch of the selection strategy (select.cu), grown on demand.
@@ -201,6 +202,7 @@ struct lipcache {
   float* ins_kn = nullptr;
   float* ins_tau = nullptr;
   int32_t* ins_rank = nullptr;
+  int32_t* ins_fix = nullptr;  // rows listed for the FP64 pass of the current certification
   int32_t* ins_bcount = nullptr;
   int32_t* ins_boffset = nullptr;
   int64_t* ins_total = nullptr;       // device, 4: rows appended; consistency counts
