@@ -415,6 +415,7 @@ def run_ours(args, dist: Dist):
 
     path_id = info["last_probe_path"]
     rf = roofline(w, N, B, kernel_ms, pk, pk_kind, PROBE_KERNELS[path_id][0])
+    tf32_derived = pk["bf16_tflops"] * TF32_OVER_BF16
     if rf["bound"] == "tensor" and not args.no_tf32_peak:
         # the TF32 peak measured live beside the derived one (MEASURED_PEAKS.json holds BF16 only)
         tf = measure_tf32_peak(dev)
@@ -440,10 +441,10 @@ def run_ours(args, dist: Dist):
         "gpu_launches": 3 * args.steps,
         "clocks": clocks,
         "insert": insert_summary(w, n_acc, insert_ms, torch.cuda.get_device_properties(dev).multi_processor_count,
-                                 clocks, kernel=insert_kernel, tf32_peak=rf.get("peak")),
+                                 clocks, kernel=insert_kernel, tf32_peak=tf32_derived, hbm_peak=pk["hbm_gbs"]),
         "insert_tight": insert_summary(w, n_acc_t, insert_ms_t,
                                        torch.cuda.get_device_properties(dev).multi_processor_count, clocks,
-                                       kernel=insert_kernel_t, tf32_peak=rf.get("peak")),
+                                       kernel=insert_kernel_t, tf32_peak=tf32_derived, hbm_peak=pk["hbm_gbs"]),
         "stats": {"sigma": sigma, "hit_rate": hit_rate,
                   "candidates_per_query": info["candidates"] / max(1, args.steps * B),
                   "device_errors": info["device_errors"], "kernel_ms": kernel_ms,
@@ -452,22 +453,25 @@ def run_ours(args, dist: Dist):
     return line
 
 
-def insert_summary(w, n_acc, insert_ms, sms, clocks, kernel=None, tf32_peak=None):
-    """Certified insertion of the whole cache (Algorithm 1); algorithmic work
-    2 C d flops per row (the head contraction). The FP32 certify kernels run
-    it on the CUDA cores: roofline the FP32 ALU, the SM count x 128 FP32
-    lanes x 2 flops x the maximum SM clock seen by nvidia-smi. The tensor
-    kernel (k_certify_tc) runs it as TF32 MMAs: roofline the TF32 tensor
-    peak, with the same flops against the FP32 ALU peak beside it for
-    comparison; that kernel is bound by its epilogue (candidate passes and
-    compensated refinement on the CUDA cores), not by the tensor pipe.
-    `roofline` divides by the certify kernel's own time (CUDA events around
-    each launch, summed over the launches); `e2e` by the time of the whole
-    insert calls (certify, scan, scatter, the count read back to the host)."""
+def insert_summary(w, n_acc, insert_ms, sms, clocks, kernel=None, tf32_peak=None, hbm_peak=None):
+    """Certified insertion of the whole cache (Algorithm 1). Algorithmic work
+    per row: 2 C d flops (the head contraction) and 8 d + 16 bytes (the row
+    read, its key written to the table, the per-entry fields). The tensor
+    kernel (k_certify_tc) runs the contraction as TF32 MMAs, so the larger of
+    the byte time at the HBM peak and the flop time at the TF32 peak bounds
+    it, and that is the byte time: `roofline` reports it against the measured
+    HBM copy bandwidth, with the flops against the TF32 and FP32-ALU peaks
+    beside it. The FP32 certify kernels run the contraction on the CUDA cores:
+    roofline the FP32 ALU (SM count x 128 FP32 lanes x 2 flops x the maximum
+    SM clock seen by nvidia-smi). `roofline` divides by the certify kernel's
+    own time (CUDA events around each launch and its FP64 pass, summed over
+    the launches); `e2e` by the time of the whole insert calls (certify, scan,
+    scatter, the count read back to the host)."""
     mhz = (clocks or {}).get("sm_max_mhz") or 2070
     alu_peak = sms * 128 * 2 * mhz * 1e6 / 1e12
     alu_kind = f"derived: {sms} SMs x 128 FP32 lanes x 2 x {mhz} MHz"
     flops = 2.0 * w.N * w.C * w.d
+    nbytes = float(w.N) * (8 * w.d + 16)
     e2e = flops / (insert_ms * 1e-3) / 1e12
     out = {"rows": w.N, "accepted": n_acc, "ms": insert_ms, "rows_per_s": w.N / (insert_ms * 1e-3),
            "batch": w.insert_batch,
@@ -475,14 +479,19 @@ def insert_summary(w, n_acc, insert_ms, sms, clocks, kernel=None, tf32_peak=None
     if kernel and kernel[2] > 0:
         name, k_ms_total, launches, pairs, full_rows, fp64_rows = kernel
         out["rows_fp64_pass"] = fp64_rows
-        achieved = flops / (k_ms_total * 1e-3) / 1e12
+        secs = k_ms_total * 1e-3
+        achieved = flops / secs / 1e12
         out["kernel"] = name
         out["kernel_ms"] = k_ms_total / launches
         out["kernel_launches"] = launches
-        if name == "k_certify_tc" and tf32_peak:
-            out["roofline"] = {"bound": "tensor", "achieved": achieved, "peak": tf32_peak, "unit": "TFLOP/s",
-                               "frac": achieved / tf32_peak,
-                               "peak_kind": "measured bf16 burst x nominal tf32/bf16 ratio",
+        if name == "k_certify_tc" and tf32_peak and hbm_peak:
+            gbs = nbytes / secs / 1e9
+            out["roofline"] = {"bound": "hbm", "achieved": gbs, "peak": hbm_peak, "unit": "GB/s",
+                               "frac": gbs / hbm_peak, "algorithmic_bytes_per_row": 8 * w.d + 16,
+                               "peak_kind": "measured copy bandwidth",
+                               "tensor_equiv": {"achieved": achieved, "peak": tf32_peak, "unit": "TFLOP/s",
+                                                "frac": achieved / tf32_peak,
+                                                "peak_kind": "measured bf16 burst x nominal tf32/bf16 ratio"},
                                "alu_equiv": {"peak": alu_peak, "frac": achieved / alu_peak, "peak_kind": alu_kind},
                                "refined_pairs_per_row": pairs / w.N, "rows_refined_over_all_classes": full_rows}
         else:
