@@ -275,9 +275,14 @@ def recorded_traffic(workload: str, path_id: int = 3):
     return float(rec["traffic_bytes_per_launch"])
 
 
-def cpu_baseline(w, W, b, rows, Q, budget_s: float) -> dict:
+def cpu_baseline(w, W, b, rows, Q, budget_s: float, gpu=None):
     """The FP64 oracle as it stands, on the host cores, on a bounded sample:
-    the first n queries against the whole cache (n sized to the budget)."""
+    the first n queries against the whole cache (n sized to the budget).
+    With gpu = (index, label, dist) of the GPU's first batch, also compares
+    the sampled queries with the GPU's answers (untimed): returns
+    (baseline, parity) where parity counts identical answers, the oracle's
+    1e-5 band, disagreements inside and outside it, and unsafe accepts (GPU
+    hits the oracle's FP64 distance and radius reject)."""
     import oracle
     t0 = time.perf_counter()
     sigma = oracle.sigma_max(W)
@@ -285,21 +290,39 @@ def cpu_baseline(w, W, b, rows, Q, budget_s: float) -> dict:
     t_build = time.perf_counter() - t0
     n = max(1, oracle.threads())
     t0 = time.perf_counter()
-    oracle.probe(cache["keys"], cache["radius"], cache["label"], Q[:n])
+    res = [oracle.probe(cache["keys"], cache["radius"], cache["label"], Q[:n])]
     t1 = time.perf_counter() - t0
     total_q, total_t = n, t1
     if t1 < budget_s:
         m = int(min(len(Q) - n, max(0, (budget_s - t1) / t1 * n)))
+        if gpu is not None:
+            m = min(m, len(gpu[0]) - n)
         if m > 0:
             t0 = time.perf_counter()
-            oracle.probe(cache["keys"], cache["radius"], cache["label"], Q[n:n + m])
+            res.append(oracle.probe(cache["keys"], cache["radius"], cache["label"], Q[n:n + m]))
             total_t += time.perf_counter() - t0
             total_q += m
     N = len(cache["keys"])
-    return {"value": total_q / total_t, "unit": "queries/s", "cores": oracle.threads(), "kind": "oracle",
+    base = {"value": total_q / total_t, "unit": "queries/s", "cores": oracle.threads(), "kind": "oracle",
             "pairs_per_s": total_q * N / total_t,
             "sample": f"{total_q} queries of the '{w.name}' workload against the full {N}-entry cache "
                       f"(FP64 brute force, {total_t:.1f} s; oracle cache build {t_build:.1f} s untimed)"}
+    if gpu is None:
+        return base, None
+    orc = {k: np.concatenate([r[k] for r in res]) for k in ("index", "label", "decision_band", "selection_band")}
+    gi, gl = gpu[0][:total_q], gpu[1][:total_q]
+    band = (orc["decision_band"] | orc["selection_band"]).astype(bool)
+    same = (gi == orc["index"]) & (gl == orc["label"])
+    hit = np.nonzero(gi >= 0)[0]
+    unsafe = 0
+    if hit.size:
+        D = oracle.pair_dist(Q[:total_q], cache["keys"], hit, gi[hit])
+        unsafe = int((~(D < cache["radius"][gi[hit]])).sum())
+    parity = {"queries": int(total_q), "identical": int(same.sum()), "band": int(band.sum()),
+              "mismatch_in_band": int((~same & band).sum()), "mismatch_outside_band": int((~same & ~band).sum()),
+              "unsafe_accepts": unsafe, "gpu_hits": int(hit.size), "oracle_hits": int((orc["index"] >= 0).sum()),
+              "sample": "the cpu_baseline queries (the first batch's first ones) against the oracle's FP64 cache"}
+    return base, parity
 
 
 # ---------------------------------------------------------------- our arm
@@ -408,9 +431,10 @@ def run_ours(args, dist: Dist):
     e2e_s = time.perf_counter() - t0
     e2e_value, _ = aggregate(dist, e2e_steps * B, e2e_s)
 
-    cpu = None
+    cpu = parity = None
     if dist.rank == 0 and not args.no_cpu_baseline:
-        cpu = cpu_baseline(w, W, b, rows, Q, args.cpu_seconds)
+        g0 = [t.cpu().numpy() for t in outs[0]]  # the first batch, Q[:B]
+        cpu, parity = cpu_baseline(w, W, b, rows, Q, args.cpu_seconds, gpu=g0)
     cache.close()
 
     path_id = info["last_probe_path"]
@@ -436,6 +460,7 @@ def run_ours(args, dist: Dist):
         "pairs_per_s": value * N,
         "roofline": rf,
         "cpu_baseline": cpu,
+        "parity": parity,
         "e2e": {"value": e2e_value, "unit": "queries/s", "h2d_bytes_per_step": B * w.d * 4,
                 "d2h_bytes_per_step": B * (8 + 4 + 4)},
         "gpu_launches": 3 * args.steps,

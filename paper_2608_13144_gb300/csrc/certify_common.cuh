@@ -43,6 +43,7 @@ struct CertArgs {
   // relative: listed here for the FP64 pass (k_certify_fix); nullable
   int* fix_count;
   int32_t* fix_list;
+  float gfix;  // rounding-error factor of the FP64 pass's logits (rounded up)
 };
 
 // Relative accuracy the reported radius must reach without the FP64 pass: a
@@ -161,6 +162,7 @@ __device__ __forceinline__ bool pair_gt(float ah, float al, float bh, float bl) 
 // upper bound v + e among the other candidates, ||z||^2 (FP32) and y^G.
 struct RowVals {
   float h1, l1, e1, h2, l2, up, kn;
+  float em;  // the largest error bound among the refined classes
   int y;
 };
 
@@ -184,10 +186,12 @@ __device__ __forceinline__ float refined_err(float g2f, float wn, float hn, floa
 struct Top2 {
   float b1h = -INFINITY, b1l = 0.f, b2h = -INFINITY, b2l = 0.f, e1 = 0.f;
   float u1 = -INFINITY, u2 = -INFINITY;
+  float em = 0.f;  // largest error bound pushed
   int y = -1, cu1 = -1;
   bool nan = false;  // a refined logit is NaN: the row is rejected
   __device__ __forceinline__ void push(int c, float vh, float vl, float e) {
     nan |= !(vh == vh && vl == vl);
+    em = fmaxf(em, e);
     const bool eq1 = vh == b1h && vl == b1l;
     if (pair_gt(vh, vl, b1h, b1l) || (eq1 && c < y)) {
       b2h = b1h;
@@ -218,6 +222,7 @@ struct Top2 {
     v.l2 = b2l;
     v.up = (cu1 == y) ? u2 : u1;
     v.kn = kn;
+    v.em = em;
     v.y = y < 0 ? 0 : y;  // every refined logit NaN: the margin is NaN and the row is rejected
     return v;
   }
@@ -234,10 +239,13 @@ __device__ void row_finals(const CertArgs& a, int64_t row, const RowVals& v, uin
   const double rs = (mlo > 0.0) ? __dmul_rd(mlo, a.inv_denom_safe) : 0.0;
   const int32_t lab = a.payload ? a.payload[row] : v.y;
   const bool acc = !(a.require_consistency && lab != v.y) && (r64 > 0.0) && !(a.miss_of && a.miss_of[row] >= 0);
-  // The margin is known to within e1 + 2 (up - v2) (the best class's bound and
-  // the width of the runner-up's interval); where that is not below kFixRel m,
-  // the row goes to the FP64 pass, which rewrites everything below.
-  if (a.fix_list && mval == mval && !(mval * kFixRel > (double)v.e1 + 2.0 * ((double)v.up - v2)))
+  // The margin is known to within e1 + em (the best class's error bound and
+  // the largest among the others: whichever class is the true runner-up, the
+  // refined runner-up value is within em of it); where that is not below
+  // kFixRel m, the row goes to the FP64 pass, which rewrites everything below.
+  // (up, an FP32 upper end, cannot serve here: its rounding is an ulp of the
+  // logit, far above the refinement's error.)
+  if (a.fix_list && mval == mval && !(mval * kFixRel > (double)v.e1 + (double)v.em))
     a.fix_list[atomicAdd(a.fix_count, 1)] = (int32_t)row;
   float rr, tau;
   thresholds(__double2float_rd(rs), v.kn, a.tc, rr, tau);

@@ -211,6 +211,7 @@ __device__ __forceinline__ void top2_merge(Top2& A, const Top2& B) {
   R.u1 = up;
   R.u2 = up;
   R.cu1 = -2;
+  R.em = fmaxf(A.em, B.em);
   R.nan = A.nan || B.nan;
   A = R;
 }

@@ -121,4 +121,19 @@ def check_probe(gi, gl, gd, ref, Q, orc):
     assert not out.any(), (f"{out.sum()} queries differ outside the 1e-5 band: "
                            f"gpu {gi[out][:5]} oracle {orc['index'][out][:5]}")
     return {"queries": len(gi), "hits": int(hits.sum()), "oracle_hits": int((orc["index"] >= 0).sum()),
-            "band": int(band.sum()), "band_mismatch": int((mism & band).sum())}
+            "identical": int((~mism).sum()), "band": int(band.sum()),
+            "decision_band": int(orc["decision_band"].astype(bool).sum()),
+            "selection_band": int(orc["selection_band"].astype(bool).sum()),
+            "band_mismatch": int((mism & band).sum()), "unsafe_accepts": 0}
+
+
+def record_parity(workload, path, stats):
+    """Append one parity record (the counts check_probe returns, the unsafe
+    accepts among them asserted to be 0) as a JSON line to the file named by
+    LIPCACHE_PARITY_OUT, when that variable is set."""
+    import json
+    import os
+    dst = os.environ.get("LIPCACHE_PARITY_OUT")
+    if dst:
+        with open(dst, "a") as f:
+            f.write(json.dumps({"workload": workload, "path": path, **stats}) + "\n")

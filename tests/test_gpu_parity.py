@@ -5,7 +5,7 @@ import pytest
 import oracle
 import synth
 from conftest import golden
-from parity_utils import check_insert, check_probe
+from parity_utils import check_insert, check_probe, record_parity
 
 torch = pytest.importorskip("torch")
 pytestmark = pytest.mark.gpu
@@ -220,6 +220,7 @@ def test_probe_parity(built, dev, name, path):
     s = built(name)
     gi, gl, gd = run_probe(s["cache"], s["Q"], dev, s["w"].batch, path)
     stats = check_probe(gi, gl, gd, s["ref"], s["Q"], s["orc"])
+    record_parity(name, path, stats)
     print(name, path, stats)
 
 
