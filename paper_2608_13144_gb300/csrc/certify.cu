@@ -95,7 +95,7 @@ __device__ RowVals warp_row_refine(const CertArgs& a, const float* __restrict__ 
       const float bc = bias[cc];
       float vh, vl;
       dot2_logit(wmat + (size_t)cc * wcs, wjs, hrow, hs, bc, d, lane, vh, vl);
-      t.push(cc, vh, vl, refined_err(a.g2f, wn32[cc], hn, bc));
+      t.push(cc, vh, vl, refined_err(a.g2f32, wn32[cc], hn, bc));
     }
   }
   return t.result(kn);
@@ -578,7 +578,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_certify_wres(CertArgs a, int Cp
             two_sum(t, __fadd_rn(cc, q), hi, lo);
             ts.rh[r][slot] = hi;
             ts.rl[r][slot] = lo;
-            ts.re[r][slot] = refined_err(a.g2f, wn_s[c], ts.hn[r], b_s[c]);
+            ts.re[r][slot] = refined_err(a.g2f8, wn_s[c], ts.hn[r], b_s[c]);
           }
         }
       }
@@ -1173,7 +1173,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_certify_wt(CertArgs a, WtLayout
           two_sum(t, __fadd_rn(cc[u], qq), hi, lo);
           ts.rh[r[u]][slot[u]] = hi;
           ts.rl[r[u]][slot[u]] = lo;
-          ts.re[r[u]][slot[u]] = refined_err(a.g2f, wn_s[c[u]], ts.hn[r[u]], b_s[c[u]]);
+          ts.re[r[u]][slot[u]] = refined_err(a.g2f8, wn_s[c[u]], ts.hn[r[u]], b_s[c[u]]);
         }
       }
     }
@@ -1409,11 +1409,15 @@ __global__ void __launch_bounds__(kFixWarps * 32) k_certify_fix(const CertArgs a
   const float* Wm = a.W;
   int ws = d;
   if (w_smem) {
+    // asynchronous 4-byte copies, all in flight at once
     float* wsm = p;
     p += ((size_t)C * (d + 1) + 3) / 4 * 4;
     for (int c = warp; c < C; c += kFixWarps)
-#pragma unroll 4
-      for (int j = lane; j < d; j += 32) wsm[(size_t)c * (d + 1) + j] = __ldg(a.W + (size_t)c * d + j);
+      for (int j = lane; j < d; j += 32) {
+        const uint32_t dst = (uint32_t)__cvta_generic_to_shared(wsm + (size_t)c * (d + 1) + j);
+        asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(dst), "l"(a.W + (size_t)c * d + j) : "memory");
+      }
+    asm volatile("cp.async.wait_all;" ::: "memory");
     Wm = wsm;
     ws = d + 1;
   }
@@ -1802,6 +1806,22 @@ size_t certify_smem_bytes(int d, int C) {
 
 namespace {
 
+// Error factor G of a compensated dot product (Dot2) evaluated as L lane
+// chains of n terms each, combined by a butterfly of log2 L levels, then the
+// bias: |hi + lo - exact| <= G (sum |W_cj z_j| + |b_c|). The pair hi + lo is
+// error-free except for the plain FP32 sum c of the TwoProduct and TwoSum
+// error terms: each term passes at most D = n + 2 log2 L + 2 roundings (the
+// chain, two per butterfly level, one before the final TwoSum), and the terms
+// sum to at most u (n + log2 L + 2) (sum |W_cj z_j| + |b_c|) (the products'
+// errors, then one TwoSum error per chain step, per level and for the bias,
+// each bounded by u times a partial sum). Hence G = gamma_D u (n + log2 L + 2),
+// with a margin for the second-order factors and the float conversion.
+double dot2_factor(int n, int L) {
+  int lg = 0;
+  while ((1 << lg) < L) ++lg;
+  return gamma32(n + 2 * lg + 2) * kU32 * (double)(n + lg + 2) * (1.0 + 1e-3);
+}
+
 // With timing enabled: a slot of the event ring for a certify kernel, its
 // start recorded on `s` (-1 when timing is off).
 int timing_begin(lipcache* h, cudaStream_t s) {
@@ -1844,10 +1864,9 @@ void launch_certify(lipcache* h, const float* H, int64_t n, const int32_t* paylo
   a.g64 = gamma64(h->d + 8) * (1.0 + 1e-6);
   a.Wnorm32 = h->Wnorm32;
   a.g32f = (float)(gamma32(h->d + 2) * (1.0 + 1e-4));
-  {
-    const double g = gamma32(h->d + 40);
-    a.g2f = (float)(2.0 * g * g * (1.0 + 1e-4));
-  }
+  a.g2f = (float)dot2_factor(h->d, 1);             // a lane per class over every feature
+  a.g2f8 = (float)dot2_factor((h->d + 7) / 8, 8);    // 8-lane groups
+  a.g2f32 = (float)dot2_factor((h->d + 31) / 32, 32);  // whole warps
   a.tc = thresh_consts(h->dpad);
   a.miss_of = miss_of;
   a.inv_pairnorm = h->inv_pairnorm;

@@ -19,7 +19,9 @@ struct CertArgs {
   double sigma, kappa, eps_rc, gamma_rc, c_scr, g32, g64;
   const float* Wnorm32;  // ||W_c|| rounded up
   float g32f;            // gamma_{d+2} with FP32 rounding slack
-  float g2f;             // error factor of the compensated dot product
+  // error factors of the compensated dot products (dot2_factor): the whole
+  // feature sequence in one lane, 8-lane groups, and 32-lane warps
+  float g2f, g2f8, g2f32;
   double inv_denom;      // kappa / (sigma sqrt 2)
   double inv_denom_safe; // kappa (1 - 8u) / (sigma (1 + slack) sqrt 2)
   ThreshConsts tc;       // constants of the probe thresholds
@@ -111,7 +113,7 @@ __device__ __forceinline__ void two_sum(float a, float b, float& s, float& e) {
 // Compensated dot product W_c . h + b_c (Ogita, Rump and Oishi's Dot2, summed
 // across the warp with the same transformations), returned as a normalised
 // pair hi + lo (|lo| <= ulp(hi)/2) whose exact sum is within
-// 2 gamma_{d+40}^2 (sum_j |W_cj h_j| + |b_c|) of the exact value. Every lane
+// g2f32 (sum_j |W_cj h_j| + |b_c|) of the exact value (dot2_factor). Every lane
 // gets the same bits: each butterfly step combines the two partners' pairs
 // symmetrically. wc[j * ws] and hrow[j * hs] address feature j of the
 // weights and of the row (global memory, or the transposed shared tiles).
@@ -174,7 +176,8 @@ __device__ __forceinline__ float norm_upper(float kn) {
 }
 
 // Bound of |hi + lo - s_c| for a refined logit, rounded up (plus the absolute
-// error of subnormal products).
+// error of subnormal products); g2f: the factor of the refinement's lane
+// layout (CertArgs::g2f, g2f8 or g2f32).
 __device__ __forceinline__ float refined_err(float g2f, float wn, float hn, float b) {
   return __fmaf_ru(g2f, __fmaf_ru(wn, hn, fabsf(b)), kTinyF);
 }

@@ -854,7 +854,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           const int ns = cnt < kMaxCandTc ? cnt : kMaxCandTc;
           for (int sl = 0; sl < ns; ++sl) {
             const int c = (int)(((sl < 4 ? cls_lo >> (8 * sl) : cls_hi >> (8 * (sl - 4)))) & 0xffu);
-            tp.push(c, res_hi[lane + 32 * sl], res_lo[lane + 32 * sl], refined_err(a.g2f, wn_s[c], hn, bias_s[c]));
+            tp.push(c, res_hi[lane + 32 * sl], res_lo[lane + 32 * sl], refined_err(a.g2f8, wn_s[c], hn, bias_s[c]));
           }
         }
         // rows that need every class of this half refined, one row at a time,
@@ -891,7 +891,7 @@ __global__ void __launch_bounds__(kThreads, 1)
               for (int u = 0; u < 2 * (32 / kGroupTc) && t2 + u < ncls; ++u) {
                 const int tt = t2 + u;
                 const int c = (2 * (tt >> 5) + half) * 32 + (tt & 31);
-                tp.push(c, res_hi[ow + 32 * u], res_lo[ow + 32 * u], refined_err(a.g2f, wn_s[c], hn, bias_s[c]));
+                tp.push(c, res_hi[ow + 32 * u], res_lo[ow + 32 * u], refined_err(a.g2f8, wn_s[c], hn, bias_s[c]));
               }
             __syncwarp();
           }
@@ -955,7 +955,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           any_nan = yg < 0;  // no candidate (cannot happen: y1 always passes)
           if (any_nan) yg = y;
           const double vy = (double)v2.x + (double)v2.y;
-          const double ey = (double)refined_err(a.g2f, wn_s[yg], hn, bias_s[yg]);
+          const double ey = (double)refined_err(a.g2f8, wn_s[yg], hn, bias_s[yg]);
           any_nan = any_nan || !(vy == vy);
           // unrolled over the slots so that the pair-table loads of all
           // candidates are in flight together
@@ -965,7 +965,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (sl < ns && j != yg) {
               const double vj = (double)res_hi[lane + 32 * sl] + (double)res_lo[lane + 32 * sl];
               any_nan |= !(vj == vj);
-              tight_term(a, yg, j, vy, ey, vj, (double)refined_err(a.g2f, wn_s[j], hn, bias_s[j]), rmin, smin);
+              tight_term(a, yg, j, vy, ey, vj, (double)refined_err(a.g2f8, wn_s[j], hn, bias_s[j]), rmin, smin);
             }
           }
         }

@@ -447,3 +447,99 @@ def test_probe_chunk_pretest_never_drops_a_kept_pair():
             kappa = np.nextafter(kappa, np.float32(-np.inf))
         assert np.any(kept >= kappa)
         assert np.float32(a.max() - tau.min()) >= kappa, trial
+
+
+# ---------------------------------------------------------------- compensated refinement (Dot2) bound
+# The certify kernels refine candidate logits with a compensated dot product
+# (Ogita, Rump and Oishi's Dot2: TwoProduct by FMA, TwoSum accumulation, the
+# error terms summed in plain FP32) evaluated as L lane chains of n features
+# each, a butterfly over the L lanes, then the bias. Its bound, used for the
+# certified radius lower bound and for sending rows to the FP64 pass, is
+# |hi + lo - exact| <= G (sum |w z| + |b|), G = gamma_D u (n + log2 L + 2),
+# D = n + 2 log2 L + 2 (dot2_factor in certify.cu). Emulated here in FP32 with
+# round-to-nearest, against exact sums.
+
+def dot2_factor(n, L):
+    lg = 0
+    while (1 << lg) < L:
+        lg += 1
+    return gamma32(n + 2 * lg + 2) * U32 * (n + lg + 2) * (1.0 + 1e-3)
+
+
+def f32(x):
+    return np.float32(x)
+
+
+def two_sum(a, b):
+    s = f32(a + b)
+    bb = f32(s - a)
+    return s, f32(f32(a - f32(s - bb)) + f32(b - bb))
+
+
+def dot2_lanes(w, z, b, L):
+    """The kernels' evaluation order: lane l takes features l, l + L, ...;
+    lanes combined by xor butterfly; then the bias and a final TwoSum."""
+    d = len(w)
+    P = [f32(0)] * L
+    Cc = [f32(0)] * L
+    for l in range(L):
+        p, c = f32(0), f32(0)
+        for j in range(l, d, L):
+            pr = f32(w[j] * z[j])
+            er = f32(float(w[j]) * float(z[j]) - float(pr))  # exact: the FMA's TwoProduct error
+            t, q = two_sum(p, pr)
+            p = t
+            c = f32(c + f32(q + er))
+        P[l], Cc[l] = p, c
+    o = L // 2
+    while o > 0:
+        NP, NC = list(P), list(Cc)
+        for l in range(L):
+            t, q = two_sum(P[l], P[l ^ o])
+            NP[l] = t
+            NC[l] = f32(f32(Cc[l] + Cc[l ^ o]) + q)
+        P, Cc = NP, NC
+        o //= 2
+    t, q = two_sum(P[0], f32(b))
+    hi, lo = two_sum(t, f32(Cc[0] + q))
+    return float(hi) + float(lo)  # exact in FP64: lo is at most half an ulp of hi
+
+
+def exact_dot(w, z, b):
+    from fractions import Fraction
+    return sum((Fraction(float(x)) * Fraction(float(y)) for x, y in zip(w, z)), Fraction(float(b)))
+
+
+@pytest.mark.parametrize("d,L", [(128, 8), (256, 8), (48, 8), (128, 32), (64, 1)])
+def test_dot2_refinement_bound(d, L):
+    from fractions import Fraction
+    rng = np.random.default_rng(d * 7 + L)
+    G = dot2_factor((d + L - 1) // L, L)
+    worst = 0.0
+    for trial in range(60):
+        kind = trial % 3
+        z = rng.standard_normal(d).astype(np.float32) * 3
+        w = rng.standard_normal(d).astype(np.float32) / np.sqrt(d)
+        if kind == 1:  # heavy cancellation: w nearly orthogonal to z
+            w64 = w.astype(np.float64) - (w.astype(np.float64) @ z.astype(np.float64)) / (z @ z) * z.astype(np.float64)
+            w = w64.astype(np.float32)
+        elif kind == 2:  # features over a wide exponent range
+            w = (w * np.exp2(rng.integers(-20, 20, d))).astype(np.float32)
+        b = np.float32(0.1 * rng.standard_normal())
+        got = dot2_lanes(w, z, b, L)
+        ex = exact_dot(w, z, b)
+        err = abs(Fraction(got) - ex)
+        scale = float(np.sum(np.abs(w.astype(np.float64) * z.astype(np.float64)))) + abs(float(b))
+        assert err <= Fraction(G * scale), (d, L, trial, float(err), G * scale)
+        worst = max(worst, float(err) / (G * scale))
+    assert worst < 1.0
+
+
+def test_dot2_factor_is_tighter_than_the_sequential_bound():
+    # 8-lane groups over d = 128: chains of 16 features; about 1e-12, some
+    # hundred times below 2 gamma_{d+40}^2
+    g8 = dot2_factor(16, 8)
+    assert 1e-12 < g8 < 3e-12
+    assert g8 * 50 < 2 * gamma32(168) ** 2
+    # one lane over every feature: about (d u)^2
+    assert dot2_factor(128, 1) > (128 * U32) ** 2
