@@ -56,6 +56,9 @@ def parse():
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-tf32-peak", action="store_true", help="skip the live cuBLAS TF32 peak measurement")
     p.add_argument("--cache-rows", type=int, default=0, help="override the workload's cache size N (profiling)")
+    p.add_argument("--noise", type=float, default=None,
+                   help="override the near-duplicate queries' per-feature noise (e.g. 0.002: most of them hit)")
+    p.add_argument("--dup", type=float, default=None, help="override the fraction of near-duplicate queries")
     p.add_argument("--insert-kernel", default="auto", choices=sorted(INSERT_KERNEL_FLAGS),
                    help="certify on an FP32 kernel instead of the default choice (profiling)")
     return p.parse_args()
@@ -164,6 +167,17 @@ class Clocks:
 
 
 # ---------------------------------------------------------------- workload
+def workload_of(args) -> synth.Workload:
+    w = synth.WORKLOADS[args.workload]
+    if args.cache_rows:
+        w = w.scaled(N=args.cache_rows)
+    if args.noise is not None:
+        w = w.scaled(noise=args.noise)
+    if args.dup is not None:
+        w = w.scaled(dup_frac=args.dup)
+    return w
+
+
 def workload_data(w: synth.Workload):
     W, b = synth.head(w)
     rows = synth.cache_rows(w)
@@ -335,9 +349,7 @@ def run_ours(args, dist: Dist):
 
     from paper_2608_13144_gb300.lipcache import LipCache
 
-    w = synth.WORKLOADS[args.workload]
-    if args.cache_rows:
-        w = w.scaled(N=args.cache_rows)
+    w = workload_of(args)
     dev = torch.device("cuda", dist.local_rank)
     torch.cuda.set_device(dev)
     pk, pk_kind = peaks()
@@ -454,6 +466,7 @@ def run_ours(args, dist: Dist):
         "scaling": "weak", "vs_baseline": None, "dtype": "tf32" if info["last_probe_path"] in (3, 4) else "fp32",
         "data": "synthetic (seeded Gaussian-mixture GuardNet features; no datasets or trained weights)",
         "config": {"workload": w.name, "N": N, "d": w.d, "C": w.C, "batch": B, "radius": "conservative",
+                   "near_duplicates": w.dup_frac, "near_duplicate_noise": w.noise,
                    "probe_path": {2: "exact", 3: "tensor_single", 4: "tensor_pair"}[info["last_probe_path"]],
                    "parallelism": "single",
                    "l2": f"inputs larger than L2 ({N * (4 * info['d_pad'] + 16) / 1e9:.2f} GB key table)"},
@@ -534,9 +547,7 @@ def run_reference(args, dist: Dist):
     workload: each step probes a bounded sample of queries (one per core)
     against the whole cache."""
     import oracle
-    w = synth.WORKLOADS[args.workload]
-    if args.cache_rows:
-        w = w.scaled(N=args.cache_rows)
+    w = workload_of(args)
     W, b, rows, Q = workload_data(w)
     sigma = oracle.sigma_max(W)
     cache = oracle.build_cache(W, b, sigma, rows)

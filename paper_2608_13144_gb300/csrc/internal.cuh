@@ -248,6 +248,21 @@ struct lipcache {
   double eps_rc = 0.0, c_scr = 0.0;
   lc::EncodeTiledFn encode = nullptr;
   int pair_clusters = -1;  // resident clusters of the pair probe kernel (-1: not yet queried)
+  // Launch state of the tensor probe kernels kept across calls, so that a
+  // probe's host side does not repeat the occupancy query, the shared-memory
+  // attribute and the tensor-map encoding: [0] k_probe_tc with 256-key
+  // tiles, [1] with 128-key tiles, [2] k_probe_pair.
+  struct ProbeLaunch {
+    int resident = 0;  // clusters that fit (0: not queried yet)
+    int smem = 0;      // dynamic shared memory the attribute was set for
+    CUtensorMap tmK, tmQ;
+    const void* k_base = nullptr;
+    uint64_t k_rows = 0;
+    const void* q_base = nullptr;
+    uint64_t q_rows = 0;
+  } probe_launch[3];
+  cudaEvent_t launch_event = nullptr;  // recorded right before the main probe kernel when set
+  bool probe_carveout_set = false;     // the prologue / finalize kernels' carveout preference
   int debug_flags = 0;     // LIPCACHE_DEBUG_* test hooks
   int last_insert_kernel = 0;  // LIPCACHE_INSERT_*
   float* wt_prep = nullptr;    // the head in the wide-tile certify kernel's shared-memory layout

@@ -181,10 +181,23 @@ void reserve_probe(lipcache* h, int64_t max_batch) {
   ensure_probe_scratch(h, (max_batch + 127) / 128 * 128);
 }
 
+// The small kernels around the tensor probe prefer the same shared-memory
+// carveout as the probe itself, so that the SM does not switch its L1 /
+// shared-memory split between the three launches of a probe.
+void set_probe_carveout(lipcache* h) {
+  if (h->probe_carveout_set) return;
+  LC_CUDA(cudaFuncSetAttribute(k_prologue, cudaFuncAttributePreferredSharedMemoryCarveout,
+                               (int)cudaSharedmemCarveoutMaxShared));
+  LC_CUDA(cudaFuncSetAttribute(k_finalize, cudaFuncAttributePreferredSharedMemoryCarveout,
+                               (int)cudaSharedmemCarveoutMaxShared));
+  h->probe_carveout_set = true;
+}
+
 void probe(lipcache* h, const float* Q, int64_t B, int64_t* out_index, int32_t* out_label, float* out_dist,
            cudaStream_t s) {
   const int64_t Bpad = (B + 127) / 128 * 128;
   ensure_probe_scratch(h, Bpad);
+  set_probe_carveout(h);
   k_prologue<<<(unsigned)((Bpad + 7) / 8), 256, 0, s>>>(Q, B, h->d, h->dpad, Bpad, h->qpad, h->kappa, h->best,
                                                       1.0 - h->c_scr, h->stats);
   LC_LAUNCH_CHECK("k_prologue");
@@ -197,11 +210,15 @@ void probe(lipcache* h, const float* Q, int64_t B, int64_t* out_index, int32_t* 
       if (h->t_issued - h->t_harvested >= lipcache::kTimingRing) harvest_timing(h, false);
       slot = (int)(h->t_issued % lipcache::kTimingRing);
       h->t_kind[slot] = 0;
-      LC_CUDA(cudaEventRecord(h->tev0[slot], s));
     }
     if (path != LIPCACHE_PROBE_EXACT) {
+      // the start event is recorded by the launcher, after its host-side
+      // preparation, right before the kernel
+      h->launch_event = slot >= 0 ? h->tev0[slot] : nullptr;
       h->last_probe_path = launch_probe_tc(h, B, path, s);
+      h->launch_event = nullptr;
     } else {
+      if (slot >= 0) LC_CUDA(cudaEventRecord(h->tev0[slot], s));
       dim3 grid((unsigned)((h->size + kEK - 1) / kEK), (unsigned)((B + kEQ - 1) / kEQ));
       h->last_grid = (int)(grid.x * grid.y);
       h->last_cluster = 1;
@@ -224,6 +241,7 @@ void probe(lipcache* h, const float* Q, int64_t B, int64_t* out_index, int32_t* 
 void probe_external_scratch(lipcache* h, const float* Q, int64_t B, int64_t* out_index, int32_t* out_label,
                             float* out_dist, float* qpad, float* kappa, unsigned long long* best, cudaStream_t s) {
   const int64_t Bpad = (B + 127) / 128 * 128;
+  set_probe_carveout(h);
   k_prologue<<<(unsigned)((Bpad + 7) / 8), 256, 0, s>>>(Q, B, h->d, h->dpad, Bpad, qpad, kappa, best,
                                                       1.0 - h->c_scr, h->stats);
   LC_LAUNCH_CHECK("k_prologue");

@@ -410,7 +410,8 @@ int probe_pair_clusters(lipcache* h) {
   const int nst = PairLayout::stages_for(nch);
   if (nst < 2) return 0;
   const int smem = PairLayout{nch, nst}.total() + 1024;
-  if (cudaFuncSetAttribute(k_probe_pair, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess) {
+  if (cudaFuncSetAttribute(k_probe_pair, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBudget + 1024) !=
+      cudaSuccess) {
     cudaGetLastError();
     return 0;
   }
@@ -431,9 +432,17 @@ void launch_probe_pair(lipcache* h, int64_t B, const float* qpad, const float* k
   const int clusters_max = probe_pair_clusters(h);
   LC_REQUIRE(clusters_max >= 1, LIPCACHE_E_CUDA, "no cluster of the pair probe kernel fits on this device");
   const int64_t Bpad = (B + 127) / 128 * 128;  // rows of the padded query buffer
-  CUtensorMap tmQ, tmK;
-  encode_rows(h, &tmQ, qpad, (uint64_t)Bpad, kHM / 2);  // a quarter of the pair's query tile per CTA
-  encode_rows(h, &tmK, h->table.keys, (uint64_t)h->table_rows, kHN);
+  lipcache::ProbeLaunch& pl = h->probe_launch[2];
+  if (pl.q_base != qpad || pl.q_rows != (uint64_t)Bpad) {
+    encode_rows(h, &pl.tmQ, qpad, (uint64_t)Bpad, kHM / 2);  // a quarter of the pair's query tile per CTA
+    pl.q_base = qpad;
+    pl.q_rows = (uint64_t)Bpad;
+  }
+  if (pl.k_base != h->table.keys || pl.k_rows != (uint64_t)h->table_rows) {
+    encode_rows(h, &pl.tmK, h->table.keys, (uint64_t)h->table_rows, kHN);
+    pl.k_base = h->table.keys;
+    pl.k_rows = (uint64_t)h->table_rows;
+  }
   PairArgs a;
   a.nch = h->dpad / kChunkF;
   a.nst = PairLayout::stages_for(a.nch);
@@ -474,7 +483,11 @@ void launch_probe_pair(lipcache* h, int64_t B, const float* qpad, const float* k
   a.stats = h->stats;
   a.debug_stall = (h->debug_flags & LIPCACHE_DEBUG_STALL_PROBE) ? 1 : 0;
   const int smem = PairLayout{a.nch, a.nst}.total() + 1024;
-  LC_CUDA(cudaFuncSetAttribute(k_probe_pair, cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
+  if (pl.smem == 0) {
+    // the attribute belongs to the kernel: the largest size any shape uses
+    LC_CUDA(cudaFuncSetAttribute(k_probe_pair, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBudget + 1024));
+    pl.smem = kSmemBudget + 1024;
+  }
   cudaLaunchAttribute attr[1];
   cudaLaunchConfig_t cfg = pair_config(smem, s, attr);
   int clusters = clusters_max;
@@ -482,7 +495,8 @@ void launch_probe_pair(lipcache* h, int64_t B, const float* qpad, const float* k
   cfg.gridDim = dim3((unsigned)(clusters * kCluster));
   h->last_grid = clusters * kCluster;
   h->last_cluster = kCluster;
-  LC_CUDA(cudaLaunchKernelEx(&cfg, k_probe_pair, tmQ, tmK, a));
+  if (h->launch_event) LC_CUDA(cudaEventRecord(h->launch_event, s));
+  LC_CUDA(cudaLaunchKernelEx(&cfg, k_probe_pair, pl.tmQ, pl.tmK, a));
   LC_LAUNCH_CHECK("k_probe_pair");
 }
 

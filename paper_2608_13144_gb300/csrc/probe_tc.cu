@@ -29,11 +29,13 @@
 //   warps 2-9  epilogue: tcgen05.ld of the accumulator (warp w reads TMEM
 //              lane quarter w % 4, column half (w - 2) / 4), screen, recheck,
 //              atomicMin of the packed (distance, index) word.
-// A work unit is one key-tile pair against a group of query tiles; units are
-// dealt round-robin over the clusters. When the number of key tiles is odd the
-// last pair's second tile lies past the table: that CTA multiplies the TMA's
-// zero fill and its epilogue skips the unit, so both CTAs still consume every
-// query stage.
+// Work: the items (key-tile pair, query tile), pair-major, are split into
+// equal contiguous ranges, one per cluster; a run is the part of a range on
+// one pair, and its key tile stays resident through the run (a pair split
+// between two clusters is loaded by both). When the number of key tiles is odd
+// the last pair's second tile lies past the table: that CTA multiplies the
+// TMA's zero fill and its epilogue skips the run, so both CTAs still consume
+// every query stage.
 #include "internal.cuh"
 #include "probe_common.cuh"
 #include "tc_ptx.cuh"
@@ -63,9 +65,7 @@ struct TcArgs {
   int nch;       // d_pad / 32
   int dpad;
   int nq;        // query tiles
-  int qpg;       // query tiles per unit
-  int n_qg;      // query groups
-  int n_units;   // key-tile pairs x query groups
+  int n_pairs;   // key-tile pairs
   int n_kt;      // key tiles holding cache entries
   const float* kappa;
   const float* qpad;
@@ -101,14 +101,26 @@ struct Layout {
   }
 };
 
-// Unit u of this cluster -> this CTA's key tile and the query-tile range.
-__device__ __forceinline__ void unit_range(const TcArgs& a, int u, uint32_t rank, int& kt, int& qt0, int& qt1) {
-  const int pair = u / a.n_qg;
-  const int g = u - pair * a.n_qg;
-  kt = pair * kCluster + (int)rank;
-  qt0 = g * a.qpg;
-  qt1 = min(a.nq, qt0 + a.qpg);
-}
+// The runs of one cluster: its range [it, end) of items (pair, query tile),
+// pair-major; next() gives this CTA's key tile and the run's query tiles.
+struct RunCursor {
+  long long it, end;
+  __device__ RunCursor(const TcArgs& a, int cluster_id, int n_clusters) {
+    const long long T = (long long)a.n_pairs * a.nq;
+    it = T * cluster_id / n_clusters;
+    end = T * (cluster_id + 1) / n_clusters;
+  }
+  __device__ bool next(const TcArgs& a, uint32_t rank, int& kt, int& qt0, int& qt1) {
+    if (it >= end) return false;
+    const int pair = (int)(it / a.nq);
+    qt0 = (int)(it - (long long)pair * a.nq);
+    const long long run_end = min(end, (long long)(pair + 1) * a.nq);
+    qt1 = qt0 + (int)(run_end - it);
+    kt = pair * kCluster + (int)rank;
+    it = run_end;
+    return true;
+  }
+};
 
 template <int BN>
 __global__ void __launch_bounds__(kThreads, 1)
@@ -177,13 +189,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         last_q_par[s] = 0;
       }
       bool ok = true;
-      for (int u = cluster_id; u < a.n_units && ok; u += n_clusters, ++i) {
-        int kt, qt0, qt1;
-        unit_range(a, u, rank, kt, qt0, qt1);
+      RunCursor rc(a, cluster_id, n_clusters);
+      int kt, qt0, qt1;
+      for (; ok && rc.next(a, rank, kt, qt0, qt1); ++i) {
         for (int qt = qt0; qt < qt1 && ok; ++qt) {
           for (int c = 0; c < a.nch && ok; ++c) {
             if (qt == qt0) {
-              // key chunk c of this unit, as soon as the previous unit's last
+              // key chunk c of this run, as soon as the previous run's last
               // query tile has finished with it (past the table: zero fill)
               ok = ptx::mbar_wait(empty_k + 8 * c, (uint32_t)(i & 1) ^ 1u, abort_s, kWaitLimit);
               if (!ok) break;
@@ -233,9 +245,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       // failure-detection test: no arrival ever completes this phase, so the
       // bounded wait expires and the kernel takes its abort path
       bool ok = !a.debug_stall || ptx::mbar_wait(drain, 0, abort_s, kWaitLimit);
-      for (int u = cluster_id; u < a.n_units && ok; u += n_clusters, ++i) {
-        int kt, qt0, qt1;
-        unit_range(a, u, rank, kt, qt0, qt1);
+      RunCursor rc(a, cluster_id, n_clusters);
+      int kt, qt0, qt1;
+      for (; ok && rc.next(a, rank, kt, qt0, qt1); ++i) {
         for (int qt = qt0; qt < qt1 && ok; ++qt, ++t) {
           const int buf = t & 1;
           ok = ptx::mbar_wait(acc_empty + 8 * buf, (uint32_t)((t >> 1) & 1) ^ 1u, abort_s, kWaitLimit);
@@ -245,7 +257,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           const bool first = qt == qt0, last = qt == qt1 - 1;
           uint64_t kd = kdesc0;
           if (first || last) {
-            // Unit edges: the key chunk arrives once per unit (TMA completion on
+            // Run edges: the key chunk arrives once per run (TMA completion on
             // the mbarrier already orders the copies before the MMA's reads),
             // and the last query tile hands each chunk back to the producer.
             for (int c = 0; c < nch; ++c, kd += kKStride) {
@@ -310,13 +322,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     int t = 0;
     bool ok = true;
     unsigned long long ncand = 0;
-    for (int u = cluster_id; u < a.n_units && ok; u += n_clusters) {
-      int kt, qt0, qt1;
-      unit_range(a, u, rank, kt, qt0, qt1);
+    RunCursor rc(a, cluster_id, n_clusters);
+    int kt, qt0, qt1;
+    while (ok && rc.next(a, rank, kt, qt0, qt1)) {
       const bool live = kt < a.n_kt;
       const int key0 = kt * BN + half * kColsPerWarp;
-      // this warp's screen terms for the unit's key tile, staged once per
-      // unit, and their minimum over each 32-key chunk
+      // this warp's screen terms for the run's key tile, staged once per
+      // run, and their minimum over each 32-key chunk
       __syncwarp();
       if (live)
         for (int v4 = lane; v4 < kColsPerWarp / 4; v4 += 32)
@@ -423,9 +435,17 @@ void encode_2d(lipcache* h, CUtensorMap* map, const float* base, uint64_t rows, 
 template <int BN>
 void launch(lipcache* h, int64_t B, const float* qpad, const float* kappa, unsigned long long* best, cudaStream_t s) {
   const int64_t Bpad = (B + kBM - 1) / kBM * kBM;
-  CUtensorMap tmQ, tmK;
-  encode_2d(h, &tmQ, qpad, (uint64_t)Bpad, kBM / 2);  // half a query tile per CTA of the pair
-  encode_2d(h, &tmK, h->table.keys, (uint64_t)h->table_rows, BN);
+  lipcache::ProbeLaunch& pl = h->probe_launch[BN == 256 ? 0 : 1];
+  if (pl.q_base != qpad || pl.q_rows != (uint64_t)Bpad) {
+    encode_2d(h, &pl.tmQ, qpad, (uint64_t)Bpad, kBM / 2);  // half a query tile per CTA of the pair
+    pl.q_base = qpad;
+    pl.q_rows = (uint64_t)Bpad;
+  }
+  if (pl.k_base != h->table.keys || pl.k_rows != (uint64_t)h->table_rows) {
+    encode_2d(h, &pl.tmK, h->table.keys, (uint64_t)h->table_rows, BN);
+    pl.k_base = h->table.keys;
+    pl.k_rows = (uint64_t)h->table_rows;
+  }
   TcArgs a;
   a.nch = h->dpad / kChunkF;
   a.nst = Layout<BN>::stages_for(a.nch);
@@ -436,15 +456,8 @@ void launch(lipcache* h, int64_t B, const float* qpad, const float* kappa, unsig
   const int64_t n_pairs = (n_kt + kCluster - 1) / kCluster;
   const int max_clusters = h->num_sms / kCluster;
   LC_REQUIRE(max_clusters >= 1, LIPCACHE_E_CUDA, "device has fewer than two SMs");
-  // enough units to keep every cluster busy when the cache is small
-  int n_qg = (int)((2LL * max_clusters + n_pairs - 1) / n_pairs);
-  if (n_qg < 1) n_qg = 1;
-  if (n_qg > a.nq) n_qg = a.nq;
-  a.qpg = (a.nq + n_qg - 1) / n_qg;
-  a.n_qg = (a.nq + a.qpg - 1) / a.qpg;
-  const int64_t n_units = n_pairs * a.n_qg;
-  LC_REQUIRE(n_units < (1LL << 31), LIPCACHE_E_INVALID, "too many work units");
-  a.n_units = (int)n_units;
+  LC_REQUIRE(n_pairs * a.nq < (1LL << 40), LIPCACHE_E_INVALID, "too many work items");
+  a.n_pairs = (int)n_pairs;
   a.n_kt = (int)n_kt;
   a.kappa = kappa;
   a.qpad = qpad;
@@ -456,7 +469,12 @@ void launch(lipcache* h, int64_t B, const float* qpad, const float* kappa, unsig
   a.debug_stall = (h->debug_flags & LIPCACHE_DEBUG_STALL_PROBE) ? 1 : 0;
   const Layout<BN> L{a.nch, a.nst};
   const int smem = L.total() + 1024;
-  LC_CUDA(cudaFuncSetAttribute(k_probe_tc<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
+  if (pl.smem == 0) {
+    // the attribute belongs to the kernel, not to this cache: set it to the
+    // largest size any shape uses, so other caches' launches stay valid
+    LC_CUDA(cudaFuncSetAttribute(k_probe_tc<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBudget + 1024));
+    pl.smem = kSmemBudget + 1024;
+  }
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)(max_clusters * kCluster));
   cfg.blockDim = dim3(kThreads);
@@ -470,15 +488,16 @@ void launch(lipcache* h, int64_t B, const float* qpad, const float* kappa, unsig
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   // persistent grid: no more clusters than can be resident at once
-  int resident = 0;
-  LC_CUDA(cudaOccupancyMaxActiveClusters(&resident, k_probe_tc<BN>, &cfg));
+  if (pl.resident == 0) LC_CUDA(cudaOccupancyMaxActiveClusters(&pl.resident, k_probe_tc<BN>, &cfg));
+  const int resident = pl.resident;
   LC_REQUIRE(resident >= 1, LIPCACHE_E_CUDA, "no CTA pair of the probe kernel fits on this device");
   int clusters = max_clusters < resident ? max_clusters : resident;
-  if (n_units < clusters) clusters = (int)n_units;
+  if (n_pairs * a.nq < clusters) clusters = (int)(n_pairs * a.nq);  // one item per cluster at least
   cfg.gridDim = dim3((unsigned)(clusters * kCluster));
   h->last_grid = clusters * kCluster;
   h->last_cluster = kCluster;
-  LC_CUDA(cudaLaunchKernelEx(&cfg, k_probe_tc<BN>, tmQ, tmK, a));
+  if (h->launch_event) LC_CUDA(cudaEventRecord(h->launch_event, s));
+  LC_CUDA(cudaLaunchKernelEx(&cfg, k_probe_tc<BN>, pl.tmQ, pl.tmK, a));
   LC_LAUNCH_CHECK("k_probe_tc");
 }
 

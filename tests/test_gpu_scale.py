@@ -77,6 +77,43 @@ def test_scale_probe_all_queries(scale):
     print("scale", stats)
 
 
+def test_scale_probe_hit_rich(scale):
+    """A hit-rich batch against the 4M-entry cache (35 % near-duplicates with
+    noise 0.002 per feature, so that most of them fall inside their entry's
+    radius, as at the paper's operating points where a third to a half of the
+    queries hit): every GPU hit is an exact FP64 hit with the oracle's label
+    and distance, and the near-duplicates of the first 1,024 queries plus 64
+    fresh ones match the oracle's brute force over the whole cache outside
+    the 1e-5 band. The exact kernel gives the same bits."""
+    s = scale
+    w = s["w"].scaled(noise=0.002, dup_frac=0.35)
+    ref = s["ref"]
+    Q, src = synth.queries(w, s["rows"])
+    q = Q[: w.batch]
+    cache = s["cache"]
+    cache.set_probe_path("auto")
+    gi, gl, gd = [t.cpu().numpy() for t in cache.probe(torch.from_numpy(q).to(s["dev"]))]
+    assert cache.info()["device_errors"] == 0 and cache.info()["last_probe_path"] == 3
+    hits = gi >= 0
+    assert hits.mean() > 0.3, hits.mean()
+    D = oracle.pair_dist(q, ref["keys"], np.nonzero(hits)[0], gi[hits])
+    assert np.all(D < ref["radius"][gi[hits]])
+    np.testing.assert_array_equal(gl[hits], ref["label"][gi[hits]])
+    np.testing.assert_allclose(gd[hits].astype(np.float64), D, rtol=1e-5)
+    rng = np.random.default_rng(4)
+    dup = np.nonzero(src[:1024] >= 0)[0]
+    fresh = np.nonzero(src[:1024] < 0)[0]
+    pick = np.sort(np.concatenate([dup, rng.choice(fresh, 64, replace=False)]))
+    orc = oracle.probe(ref["keys"], ref["radius"], ref["label"], q[pick])
+    stats = check_probe(gi[pick], gl[pick], gd[pick], ref, q[pick], orc)
+    record_parity("scale-hit-rich (sample)", "tensor", stats)
+    cache.set_probe_path("exact")
+    ge = [t.cpu().numpy() for t in cache.probe(torch.from_numpy(q).to(s["dev"]))]
+    cache.set_probe_path("auto")
+    assert np.array_equal(ge[0], gi) and np.array_equal(ge[2].view(np.uint32), gd.view(np.uint32))
+    print("scale hit-rich", stats, "batch hit rate", hits.mean())
+
+
 def test_scale_tensor_equals_exact(scale):
     """The same batch through the exact kernel (every pair on CUDA cores) and
     both tensor kernels: bit-identical outputs at full size."""
