@@ -1282,334 +1282,68 @@ int wt_ncg(int C) {
 }
 
 // ---------------------------------------------------------------- FP64 pass
-// Re-certification in FP64 of the rows the compensated FP32 refinement could
-// not pin down (listed by row_finals / tight_write: a margin, or a minimising
-// term of Eq. 29, smaller than 1 / kFixRel times its error bound - rows a hair
-// from a decision boundary, about 0.25 % of the rows of the scale workload).
-// One warp per listed row. FP64 arithmetic on this GPU has a throughput of
-// about 1/64 of FP32 and a dependent latency of ~500 cycles, so it is kept to
-// the few operations that need it: the row's FP32 logits and error bounds
-// (coalesced loads, a warp reduce-scatter) pick the classes that can matter;
-// those are recomputed in FP64 four at a time (products of FP32 values are
-// exact in FP64; each lane chains its slice of the features, a five-level
-// tree sums the lanes: error below gamma_{d/32+6} of sum |W_cj z_j| + |b_c|);
-// comparisons of FP64 values use order-preserving integer keys; y^G, the
-// margin or Eq. 29, the certified lower bound, the thresholds and the skip
-// rules of Algorithm 1 are then taken from the FP64 values and overwrite the
-// row's results. Conservative radius: the candidates are the classes whose
-// FP32 interval reaches the second-largest lower end (they include the true
-// top two). Tight radius: the possible y^G (intervals reaching the largest
-// lower end), then, for the FP64 y^G, the classes whose lower bracket of
-// (s_y - s_j) / ||W_y - W_j|| reaches the smallest upper bracket (they
-// include the minimiser of Eq. 29).
+// The stand-alone FP64 pass (fix_row_warp) over the rows a certify kernel
+// listed, for the kernels that do not run it themselves: a warp per listed
+// row, kFixWarps rows per block; the head is staged once per block into
+// shared memory (rows padded to d + 1 floats, so that a lane per class reads
+// without bank conflicts) when it fits, else read from global memory.
 constexpr int kFixWarps = 8;
 
-// Order-preserving integer key of a double: a larger value has a larger key
-// (-0 and +0 share the key of 0).
-__device__ __forceinline__ long long dkey(double v) {
-  long long b = __double_as_longlong(v);
-  if (b == (long long)0x8000000000000000ull) b = 0;
-  return b >= 0 ? b : (b ^ 0x7fffffffffffffffll);
-}
-// (key, class) of the larger value, the lower class on equal values
-__device__ __forceinline__ void argmax_key(long long& k, int& c, long long k2, int c2) {
-  if (c2 >= 0 && (c < 0 || k2 > k || (k2 == k && c2 < c))) {
-    k = k2;
-    c = c2;
-  }
-}
-__device__ __forceinline__ void warp_argmax_key(long long& k, int& c) {
+// The head's rows in memory, row c at w + c ws.
+struct WRows {
+  const float* w;
+  int ws;
+  __device__ __forceinline__ float operator()(int c, int j) const { return w[(size_t)c * ws + j]; }
+  template <int NP>
+  __device__ __forceinline__ void chains(const int (&cc)[NP], const float* __restrict__ zs, int d,
+                                         float (&acc)[NP]) const {
+    const float* wc[NP];
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) argmax_key(k, c, __shfl_xor_sync(kFull, k, o), __shfl_xor_sync(kFull, c, o));
-}
-
-// FP64 logits of four classes cc[0..3] (warp-uniform; repeats allowed) for
-// the row in shared memory, and FP32 bounds of their errors (rounded up).
-__device__ __forceinline__ void logits_fp64_x4(const CertArgs& a, const float* __restrict__ Wm, int ws,
-                                               const int (&cc)[4], const float* __restrict__ zs, int lane,
-                                               double (&v)[4], float (&e)[4]) {
-  double acc[4] = {0.0, 0.0, 0.0, 0.0};
-  float pa[4] = {0.f, 0.f, 0.f, 0.f};
-  for (int j = lane; j < a.d; j += 32) {
-    const float xf = zs[j];
-    const double x = (double)xf;
-    float w[4];
+    for (int t = 0; t < NP; ++t) {
+      wc[t] = w + (size_t)cc[t] * ws;
+      acc[t] = 0.f;
+    }
+#pragma unroll 4
+    for (int j = 0; j < d; ++j) {
+      const float z = zs[j];
 #pragma unroll
-    for (int u = 0; u < 4; ++u) w[u] = Wm[(size_t)cc[u] * ws + j];
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      acc[u] = fma((double)w[u], x, acc[u]);
-      pa[u] = __fmaf_ru(fabsf(w[u]), fabsf(xf), pa[u]);
+      for (int t = 0; t < NP; ++t) acc[t] = fmaf(wc[t][j], z, acc[t]);
     }
   }
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1)
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      acc[u] += __shfl_xor_sync(kFull, acc[u], o);
-      pa[u] = __fadd_ru(pa[u], __shfl_xor_sync(kFull, pa[u], o));
-    }
-#pragma unroll
-  for (int u = 0; u < 4; ++u) {
-    const float bc = __ldg(a.b + cc[u]);
-    v[u] = acc[u] + (double)bc;
-    e[u] = __fmaf_ru(a.gfix, __fadd_ru(pa[u], fabsf(bc)), kTinyF);
-  }
-}
-
-// Refine the n classes cls[0..n) (shared memory) into cv / ce, four at a time.
-__device__ __forceinline__ void refine_list_fp64(const CertArgs& a, const float* __restrict__ Wm, int ws,
-                                                 const int* cls, int n, const float* zs, int lane, double* cv,
-                                                 float* ce) {
-  for (int k0 = 0; k0 < n; k0 += 4) {
-    int cc[4];
-#pragma unroll
-    for (int u = 0; u < 4; ++u) cc[u] = cls[k0 + u < n ? k0 + u : k0];
-    double v[4];
-    float e[4];
-    logits_fp64_x4(a, Wm, ws, cc, zs, lane, v, e);
-    if (lane == 0)
-#pragma unroll
-      for (int u = 0; u < 4; ++u)
-        if (k0 + u < n) {
-          cv[k0 + u] = v[u];
-          ce[k0 + u] = e[u];
-        }
-  }
-  __syncwarp();
-}
-
-// Append the classes c (c < C) with pred(c) to cls[n...] in ascending order.
-template <typename Pred>
-__device__ __forceinline__ int collect(int C, int lane, int* cls, int n, Pred pred) {
-  for (int cb = 0; cb < C; cb += 32) {
-    const int c = cb + lane;
-    const bool t = c < C && pred(c);
-    const unsigned m = __ballot_sync(kFull, t);
-    if (t) cls[n + __popc(m & ((1u << lane) - 1u))] = c;
-    n += __popc(m);
-  }
-  __syncwarp();
-  return n;
-}
+};
 
 __global__ void __launch_bounds__(kFixWarps * 32) k_certify_fix(const CertArgs a, DevStats* stats, int w_smem) {
-  extern __shared__ __align__(16) float fix_smem[];
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, tid = threadIdx.x;
-  constexpr int kT = kFixWarps * 32;
+  extern __shared__ __align__(16) unsigned char fix_smem[];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int d = a.d, C = a.C;
   const int nfix = *a.fix_count;
-  if (blockIdx.x == 0 && tid == 0 && nfix > 0) atomicAdd(&stats->ins_fp64_rows, (unsigned long long)nfix);
-  if ((int)blockIdx.x >= nfix) return;  // a block per listed row
-  // shared memory: the head (rows padded to d + 1 floats, so that a thread
-  // per class reads without bank conflicts) when it fits, the row, the
-  // refined values, the FP32 logits and bounds, the candidate classes, and
-  // the per-warp partial results of block reductions
-  float* p = fix_smem;
-  const float* Wm = a.W;
-  int ws = d;
+  if (blockIdx.x == 0 && threadIdx.x == 0 && nfix > 0) atomicAdd(&stats->ins_fp64_rows, (unsigned long long)nfix);
+  if ((int)blockIdx.x * kFixWarps >= nfix) return;  // no row for this block
+  unsigned char* p = fix_smem;
+  WRows W{a.W, d};
   if (w_smem) {
     // asynchronous 4-byte copies, all in flight at once
-    float* wsm = p;
-    p += ((size_t)C * (d + 1) + 3) / 4 * 4;
+    float* wsm = reinterpret_cast<float*>(p);
+    p += ((size_t)C * (d + 1) + 3) / 4 * 16;
     for (int c = warp; c < C; c += kFixWarps)
       for (int j = lane; j < d; j += 32) {
         const uint32_t dst = (uint32_t)__cvta_generic_to_shared(wsm + (size_t)c * (d + 1) + j);
         asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(dst), "l"(a.W + (size_t)c * d + j) : "memory");
       }
     asm volatile("cp.async.wait_all;" ::: "memory");
-    Wm = wsm;
-    ws = d + 1;
+    W = WRows{wsm, d + 1};
   }
-  float* zs = p;
-  p += (d + 3) / 4 * 4;
-  double* cv = reinterpret_cast<double*>(p);  // refined values
-  p += 2 * ((C + 1) / 2 * 2);
-  float* sv = p;   // FP32 logits
-  float* ev = sv + C;  // their error bounds
-  float* ce = ev + C;  // bounds of the refined values
-  int* cls = reinterpret_cast<int*>(ce + C);  // candidate classes
-  float* red = reinterpret_cast<float*>(cls + C);  // 2 x kFixWarps partial maxima
-  int* nlist = reinterpret_cast<int*>(red + 2 * kFixWarps);
-  for (int k = blockIdx.x; k < nfix; k += gridDim.x) {
+  __syncthreads();
+  const FixScratch sc = fix_scratch_at(p + (size_t)warp * fix_scratch_bytes(d, C), d, C);
+  for (int k = (int)blockIdx.x * kFixWarps + warp; k < nfix; k += (int)gridDim.x * kFixWarps) {
     const int64_t row = a.fix_list[k];
-    __syncthreads();  // the head is staged; the previous row is done
-    for (int j = tid; j < d; j += kT) zs[j] = __ldg(a.H + (size_t)row * d + j);
-    __syncthreads();
-    const float kn = a.kn[row];
-    const float hn = norm_upper(kn);
-    if (!(hn < INFINITY)) continue;  // no finite bounds: keep the FP32 kernel's result
-    // FP32 logits, a thread per class (a fused multiply-add chain over the
-    // features, within gamma_{d+2}), and the top two lower ends of their
-    // intervals over the block
-    float l1 = -INFINITY, l2 = -INFINITY;
-    bool nan = false;
-    for (int c = tid; c < C; c += kT) {
-      const float* wc = Wm + (size_t)c * ws;
-      float acc = 0.f;
-#pragma unroll 8
-      for (int j = 0; j < d; ++j) acc = fmaf(wc[j], zs[j], acc);
-      const float bc = __ldg(a.b + c);
-      const float sc = __fadd_rn(acc, bc);
-      const float e = logit_err(a.g32f, __ldg(a.Wnorm32 + c), hn, bc, sc);
-      sv[c] = sc;
-      ev[c] = e;
-      nan |= !(sc == sc);
-      const float lo = __fsub_rd(sc, e);
-      l2 = fmaxf(l2, fminf(l1, lo));
-      l1 = fmaxf(l1, lo);
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      const float o1 = __shfl_xor_sync(kFull, l1, o), o2 = __shfl_xor_sync(kFull, l2, o);
-      l2 = fmaxf(l2, fminf(l1, o1));
-      l1 = fmaxf(l1, o1);
-      l2 = fmaxf(l2, fminf(l1, o2));
-      l1 = fmaxf(l1, o2);
-    }
-    if (lane == 0) {
-      red[2 * warp] = l1;
-      red[2 * warp + 1] = l2;
-    }
-    if (__syncthreads_or(nan ? 1 : 0)) continue;  // keep the FP32 kernel's result (a rejected row)
-    l1 = l2 = -INFINITY;
-    for (int w = 0; w < kFixWarps; ++w) {
-      const float o1 = red[2 * w], o2 = red[2 * w + 1];
-      l2 = fmaxf(l2, fminf(l1, o1));
-      l1 = fmaxf(l1, o1);
-      l2 = fmaxf(l2, fminf(l1, o2));
-      l1 = fmaxf(l1, o2);
-    }
-    // the classes that can be y^G (tight) or among the top two
-    // (conservative), refined in FP64 four per warp, the warps in parallel
-    const float Lc = a.tight ? l1 : l2;
-    if (warp == 0) {
-      const int n = collect(C, lane, cls, 0, [&](int c) { return __fadd_ru(sv[c], ev[c]) >= Lc; });
-      if (lane == 0) *nlist = n;
-    }
-    __syncthreads();
-    const int nc = *nlist;
-    for (int k0 = 4 * warp; k0 < nc; k0 += 4 * kFixWarps)
-      refine_list_fp64(a, Wm, ws, cls + k0, nc - k0 < 4 ? nc - k0 : 4, zs, lane, cv + k0, ce + k0);
-    __syncthreads();
-    // y^G: the largest refined value, the lower class on ties
-    long long ky = 0;
-    int y = -1;
-    for (int t = lane; t < nc; t += 32) argmax_key(ky, y, dkey(cv[t]), cls[t]);
-    warp_argmax_key(ky, y);
-    if (y < 0) continue;  // (every thread agrees)
-    int ty = 0;  // y's slot
-    for (int t = lane; t < nc; t += 32)
-      if (cls[t] == y) ty = t;
-    ty = __reduce_max_sync(kFull, ty);
-    const double vy = cv[ty];
-    const float ey = ce[ty];
-    if (!a.tight) {
-      if (warp != 0) continue;
-      // the runner-up value and the largest upper end among the other classes
-      long long k2 = 0, ku = 0;
-      int c2 = -1, cu = -1;
-      for (int t = lane; t < nc; t += 32) {
-        if (cls[t] == y) continue;
-        argmax_key(k2, c2, dkey(cv[t]), cls[t]);
-        argmax_key(ku, cu, dkey(__dadd_ru(cv[t], (double)ce[t])), cls[t]);
-      }
-      warp_argmax_key(k2, c2);
-      warp_argmax_key(ku, cu);
-      if (lane == 0) {
-        double v2 = -INFINITY, up = -INFINITY;
-        for (int t = 0; t < nc; ++t) {
-          if (cls[t] == c2) v2 = cv[t];
-          if (cls[t] == cu) up = __dadd_ru(cv[t], (double)ce[t]);
-        }
-        const double mval = vy - v2;
-        const double mlo = __dsub_rd(__dsub_rd(vy, (double)ey), up);
-        const double r64 = mval * a.inv_denom;
-        const double rs = (mlo > 0.0) ? __dmul_rd(mlo, a.inv_denom_safe) : 0.0;
-        const int32_t lab = a.payload ? a.payload[row] : y;
-        const bool acc =
-            !(a.require_consistency && lab != y) && (r64 > 0.0) && !(a.miss_of && a.miss_of[row] >= 0);
-        float rr, tau;
-        thresholds(__double2float_rd(rs), kn, a.tc, rr, tau);
-        a.accept[row] = acc ? 1 : 0;
-        a.yG[row] = y;
-        a.label[row] = lab;
-        a.radius[row] = __double2float_rz(r64);
-        a.rr[row] = rr;
-        a.tau[row] = tau;
-      }
-    } else {
-      // Eq. 29 for the FP64 y^G: FP32 brackets of every term from the FP32
-      // logits and the FP32 brackets of the reciprocal pair norms, then FP64
-      // for the classes whose lower bracket reaches the smallest upper one
-      const float vyh = __fadd_ru(__double2float_ru(vy), ey), vyl = __fsub_rd(__double2float_rd(vy), ey);
-      const bool brk = a.ipn_up32 != nullptr && a.ipn_dn32 != nullptr;
-      __syncthreads();  // every warp has read the candidates' values
-      if (warp == 0) {
-        float U = INFINITY;
-        if (brk)
-          for (int j = lane; j < C; j += 32) {
-            const float iu = a.ipn_up32[(size_t)y * C + j];
-            if (j == y || !(iu < INFINITY)) continue;  // W_j = W_y: no term
-            U = fminf(U, __fmul_ru(__fsub_ru(vyh, __fsub_rd(sv[j], ev[j])), iu));
-          }
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) U = fminf(U, __shfl_xor_sync(kFull, U, o));
-        const int n = collect(C, lane, cls, 0, [&](int j) {
-          if (j == y) return false;
-          if (!brk) return true;
-          const float iu = a.ipn_up32[(size_t)y * C + j];
-          return iu < INFINITY &&
-                 __fmul_rd(__fsub_rd(vyl, __fadd_ru(sv[j], ev[j])), a.ipn_dn32[(size_t)y * C + j]) <= U;
-        });
-        if (lane == 0) *nlist = n;
-      }
-      __syncthreads();
-      const int nj = *nlist;
-      for (int k0 = 4 * warp; k0 < nj; k0 += 4 * kFixWarps)
-        refine_list_fp64(a, Wm, ws, cls + k0, nj - k0 < 4 ? nj - k0 : 4, zs, lane, cv + k0, ce + k0);
-      __syncthreads();
-      if (warp != 0) continue;
-      // the terms of Eq. 29 and their certified lower bounds (tight_term), one
-      // lane per class, minima by key
-      long long kr = dkey(INFINITY), ks = dkey(INFINITY);  // no term: r* = +inf
-      for (int t = lane; t < nj; t += 32) {
-        double rmin = INFINITY, smin = INFINITY;
-        tight_term(a, y, cls[t], vy, (double)ey, cv[t], (double)ce[t], rmin, smin);
-        kr = min(kr, dkey(rmin));
-        ks = min(ks, dkey(smin));
-      }
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) {
-        kr = min(kr, __shfl_xor_sync(kFull, kr, o));
-        ks = min(ks, __shfl_xor_sync(kFull, ks, o));
-      }
-      if (lane == 0) {
-        // back from the keys (dkey is its own inverse on the bits)
-        const double rmin = kr < 0 ? __longlong_as_double(kr ^ 0x7fffffffffffffffll) : __longlong_as_double(kr);
-        const double smin = ks < 0 ? __longlong_as_double(ks ^ 0x7fffffffffffffffll) : __longlong_as_double(ks);
-        const double r64 = a.kappa * rmin;
-        const double rs = smin > 0.0 ? __dmul_rd(a.kappa, smin) : 0.0;
-        const int32_t lab = a.payload ? a.payload[row] : y;
-        const bool acc =
-            !(a.require_consistency && lab != y) && (r64 > 0.0) && !(a.miss_of && a.miss_of[row] >= 0);
-        float rr, tau;
-        thresholds(__double2float_rd(rs), kn, a.tc, rr, tau);
-        a.accept[row] = acc ? 1 : 0;
-        a.yG[row] = y;
-        a.label[row] = lab;
-        a.radius[row] = __double2float_rz(r64);
-        a.rr[row] = rr;
-        a.tau[row] = tau;
-      }
-    }
+    fix_row_warp(a, row, a.kn[row], W, sc, lane);
   }
 }
 
 size_t fix_smem_bytes(int d, int C, bool w_smem) {
-  const size_t w = w_smem ? ((size_t)C * (d + 1) + 3) / 4 * 4 : 0;
-  return sizeof(float) * (w + (size_t)(d + 3) / 4 * 4 + 2 * (size_t)((C + 1) / 2 * 2) + 4 * (size_t)C +
-                          2 * kFixWarps + 4);
+  const size_t w = w_smem ? ((size_t)C * (d + 1) + 3) / 4 * 16 : 0;
+  return w + (size_t)kFixWarps * fix_scratch_bytes(d, C);
 }
 
 // Exclusive scan of the per-block accepted counts (one block).
@@ -1900,9 +1634,10 @@ void launch_certify(lipcache* h, const float* H, int64_t n, const int32_t* paylo
   const int ncg = wt_ncg(h->C);
   const bool vec16 = h->d % 4 == 0 && ((uintptr_t)H & 15) == 0;
   const WtLayout L = wt_layout(h->d, h->C, ncg > 0 ? ncg : 1);
+  bool fixed_in_kernel = false;
   if (certify_tc_supported(h, H, n)) {
     slot = timing_begin(h, s);
-    certify_tc_launch(h, a, s);
+    fixed_in_kernel = certify_tc_launch(h, a, s);
     h->last_insert_kernel = LIPCACHE_INSERT_TENSOR;
   } else if ((!a.tight || h->ipn_up32) && vec16 && ncg > 0 && L.total <= 227 * 1024 &&
              !(h->debug_flags & LIPCACHE_DEBUG_INSERT_TILE64)) {
@@ -1947,9 +1682,9 @@ void launch_certify(lipcache* h, const float* H, int64_t n, const int32_t* paylo
     LC_LAUNCH_CHECK("k_certify");
     h->last_insert_kernel = LIPCACHE_INSERT_STREAMED;
   }
-  // the FP64 pass over the rows the kernel listed (usually a few per thousand;
-  // none from the kernels that refine in FP64 already)
-  {
+  // the FP64 pass over the rows the kernel listed (a few per 100,000; none
+  // from the kernels that refine in FP64 already), unless the kernel ran it
+  if (!fixed_in_kernel) {
     const bool w_smem = fix_smem_bytes(h->d, h->C, true) <= 200 * 1024;
     const size_t fsm = fix_smem_bytes(h->d, h->C, w_smem);
     if (fsm > 48 * 1024) LC_CUDA(cudaFuncSetAttribute(k_certify_fix, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)fsm));

@@ -34,7 +34,7 @@
 // Each half reduces Eq. 29 over its own candidates in FP64; rows with more
 // candidates than slots take a one-warp path over every class.
 //
-// Schedule. Persistent CTAs, one per SM, 320 threads:
+// Schedule. Persistent CTAs, one per SM, 384 threads:
 //   warp 0     TMA producer: W (resident, 128-byte swizzle, rows past C zero
 //              filled), then each tile's 128 rows (one 16 KB box per 32-feature
 //              chunk, features past d zero filled) into one of nzb buffers,
@@ -54,7 +54,13 @@
 //              in a half, or whose Mb is not below 1e38, has every class of
 //              that half refined; the partners' running selections are merged
 //              and one thread per row runs the FP64 finals. Tight radius: see
-//              above; such rows take the one-warp path.
+//              above; such rows take the one-warp path. Rows the finals list
+//              for the FP64 pass go into a queue in shared memory;
+//   warp 10    the FP64 pass (fix_row_warp) over the queued rows, with the
+//              head read in place, while the epilogue goes on with later
+//              tiles (when its queue and scratch fit in shared memory; else
+//              the rows stay listed for the stand-alone pass);
+//   warp 11    idle.
 // Every mbarrier wait is bounded; a role that gives up raises the CTA's abort
 // flag, the others drain, and the launch counts a device error.
 #include "certify_common.cuh"
@@ -68,7 +74,11 @@ constexpr int kChunkF = 32;                   // features per 128-byte swizzle r
 constexpr int kMaxChunks = 8;                 // d <= 256
 constexpr uint32_t kZChunkBytes = kBM * 128;  // one 32-feature chunk of a tile
 constexpr int kEpiWarps = 8;
-constexpr int kThreads = 32 * (2 + kEpiWarps);
+constexpr int kFixWarp = 2 + kEpiWarps;       // the in-kernel FP64 pass
+// twelve warps (the last one idle): three per SM sub-partition give each
+// thread the same 168 registers as ten, without spills
+constexpr int kThreads = 32 * (4 + kEpiWarps);
+constexpr int kFixQ = 32;                     // slots of the FP64 pass's row queue
 constexpr int kMaxCandTc = 8;                 // candidate slots per row and column half
 constexpr int kListCap = 32 * kMaxCandTc;     // pair list of one epilogue warp
 // per epilogue warp: the pair list, then the refined pairs hi / lo by (row lane, slot)
@@ -123,17 +133,32 @@ __device__ __forceinline__ void top2i_merge(float& a1, int& j1, float& a2, int& 
 }
 
 // Shared-memory layout (offsets from a 1024-byte aligned base).
-struct TcLayout {
-  int nch, Cpad, nzb;
-  uint32_t wbytes, zbytes;
-  uint32_t off_z, off_bias, off_wn, off_list, off_x1, off_x2, off_acc, off_bar, off_misc, total;
+// Queue of the rows listed for the FP64 pass, from the epilogue warps to the
+// fix warp (shared memory): entry k sits in slot k % kFixQ once seq[slot] = k.
+struct FixQueue {
+  int n;      // entries pushed
+  int taken;  // entries the fix warp has finished (their slots are free)
+  int done;   // epilogue warps past their last tile
+  int beat;   // advanced by the epilogue every tile (the fix warp's wait bound)
+  int seq[kFixQ];
+  int row[kFixQ];
+  float kn[kFixQ];
 };
 
-TcLayout tc_layout(int d, int C, int nzb) {
+struct TcLayout {
+  int nch, Cpad, nzb, infix;
+  uint32_t wbytes, zbytes;
+  uint32_t off_z, off_bias, off_wn, off_list, off_x1, off_x2, off_acc, off_bar, off_misc, off_fixq, off_fixs, total;
+};
+
+// infix: the fix warp runs the FP64 pass in the kernel (its queue and scratch
+// in shared memory); else the rows stay listed for the stand-alone pass.
+TcLayout tc_layout(int d, int C, int nzb, int infix) {
   TcLayout L;
   L.nch = (d + kChunkF - 1) / kChunkF;
   L.Cpad = (C + 15) / 16 * 16;
   L.nzb = nzb;
+  L.infix = infix;
   L.wbytes = (uint32_t)L.nch * (uint32_t)L.Cpad * 128u;  // a multiple of 2048
   L.zbytes = (uint32_t)L.nch * kZChunkBytes;
   L.off_z = L.wbytes;
@@ -145,7 +170,9 @@ TcLayout tc_layout(int d, int C, int nzb) {
   L.off_acc = L.off_x2 + kBM * (uint32_t)sizeof(Top2);
   L.off_bar = (L.off_acc + kBM + 32 + 7) / 8 * 8;  // + ok flags of the halves (2 x 4 ints)
   L.off_misc = L.off_bar + (8 + 2 * kMaxChunks) * 8;  // the barrier map is in the kernel
-  L.total = L.off_misc + 16;
+  L.off_fixq = L.off_misc + 16;
+  L.off_fixs = (L.off_fixq + (infix ? (uint32_t)sizeof(FixQueue) : 0u) + 15) / 16 * 16;
+  L.total = L.off_fixs + (infix ? (uint32_t)fix_scratch_bytes(d, C) : 0u);
   return L;
 }
 
@@ -186,6 +213,72 @@ __device__ __forceinline__ float4 lds_f4(uint32_t addr) {
 
 // Named barrier of the two epilogue warps of one lane quarter.
 __device__ __forceinline__ void pair_barrier(int id) { asm volatile("bar.sync %0, 64;" ::"r"(id) : "memory"); }
+
+// The resident head in shared memory (TMA 128-byte swizzle, 32-feature chunks
+// wchunk bytes apart) as the FP64 pass reads it.
+struct WSwz {
+  uint32_t s_w, wchunk;
+  __device__ __forceinline__ float operator()(int c, int j) const {
+    float v;
+    asm volatile("ld.shared.f32 %0, [%1];" : "=f"(v) : "r"(s_w + sw_off(c, j, wchunk)));
+    return v;
+  }
+  // sum_j W_cj zs_j for NP classes, fused multiply-adds in feature order
+  // (d % 16 == 0), four features per 16-byte load
+  template <int NP>
+  __device__ __forceinline__ void chains(const int (&cc)[NP], const float* __restrict__ zs, int d,
+                                         float (&acc)[NP]) const {
+    uint32_t rb[NP], x[NP];
+#pragma unroll
+    for (int t = 0; t < NP; ++t) {
+      rb[t] = s_w + (uint32_t)cc[t] * 128u;
+      x[t] = (uint32_t)cc[t] & 7u;
+      acc[t] = 0.f;
+    }
+    for (int k = 0; k < d; k += kChunkF) {
+      const uint32_t co = (uint32_t)(k / kChunkF) * wchunk;
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        if (k + 4 * u < d) {
+          const float4 z = *reinterpret_cast<const float4*>(zs + k + 4 * u);
+#pragma unroll
+          for (int t = 0; t < NP; ++t) {
+            const float4 w = lds_f4(rb[t] + co + ((((uint32_t)u) ^ x[t]) << 4));
+            acc[t] = fmaf(w.x, z.x, acc[t]);
+            acc[t] = fmaf(w.y, z.y, acc[t]);
+            acc[t] = fmaf(w.z, z.z, acc[t]);
+            acc[t] = fmaf(w.w, z.w, acc[t]);
+          }
+        }
+      }
+    }
+  }
+};
+
+// Hand a listed row to the fix warp (one lane; after the row's results are
+// written). Waits, bounded, for a free slot; false if the kernel aborted.
+__device__ __noinline__ bool fixq_push(FixQueue* q, int row, float kn, volatile int* abort_s, long long limit) {
+  __threadfence_block();  // the row's results before the entry
+  const int k = atomicAdd(&q->n, 1);
+  volatile int* taken = &q->taken;
+  if (*taken <= k - kFixQ) {
+    const long long t0 = clock64();
+    while (*taken <= k - kFixQ) {
+      if (*abort_s) return false;
+      if (clock64() - t0 > limit) {
+        *abort_s = 1;
+        return false;
+      }
+      __nanosleep(128);
+    }
+  }
+  const int sl = k % kFixQ;
+  q->row[sl] = row;
+  q->kn[sl] = kn;
+  __threadfence_block();
+  *(volatile int*)&q->seq[sl] = k;
+  return true;
+}
 
 // Top2 over the union of two disjoint class sets from the two sets' states:
 // the same y^G, runner-up value and bounds as pushing every class into one.
@@ -301,7 +394,8 @@ __device__ __forceinline__ void refine2(uint32_t ws, uint32_t wchunk, uint32_t z
 // features in order, as the wide-tile kernel's fallback), y^G the largest
 // refined logit (lowest class on ties), then Eq. 29 over every other class in
 // FP64. The row's features come from the tile in shared memory (row rz).
-__device__ void tc_tight_row_warp(const CertArgs& a, int64_t row, int rz, uint32_t s_w, uint32_t wchunk, uint32_t zs,
+// Returns (on every lane) whether the row was listed for the FP64 pass.
+__device__ bool tc_tight_row_warp(const CertArgs& a, int64_t row, int rz, uint32_t s_w, uint32_t wchunk, uint32_t zs,
                                   const float* __restrict__ wn_s, const float* __restrict__ b_s, float kn, int lane,
                                   uint8_t* acc_slot) {
   constexpr int kPer = 8;  // classes per lane (C <= 256)
@@ -377,8 +471,9 @@ __device__ void tc_tight_row_warp(const CertArgs& a, int64_t row, int rz, uint32
   }
   rmin = warp_min_d(rmin);
   smin = warp_min_d(smin);
-  if (lane == 0) tight_write(a, row, y, rmin, smin, nan_any, kn, acc_slot);
-  __syncwarp();
+  bool fix = false;
+  if (lane == 0) fix = tight_write(a, row, y, rmin, smin, nan_any, kn, acc_slot);
+  return __shfl_sync(kFull, fix ? 1 : 0, 0) != 0;
 }
 
 template <bool TIGHT>
@@ -406,6 +501,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   volatile int* okf = reinterpret_cast<volatile int*>(smem + L.off_acc + kBM);
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L.off_misc);
   volatile int* abort_s = reinterpret_cast<volatile int*>(smem + L.off_misc + 4);
+  FixQueue* fixq = L.infix ? reinterpret_cast<FixQueue*>(smem + L.off_fixq) : nullptr;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int d = a.d, C = a.C;
@@ -419,6 +515,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     ptx::mbar_init(drain, 1);
     *abort_s = 0;
+    if (fixq) {
+      fixq->n = fixq->taken = fixq->done = fixq->beat = 0;
+      for (int i = 0; i < kFixQ; ++i) fixq->seq[i] = -1;
+    }
     ptx::fence_mbar_init();
     ptx::tma_prefetch_desc(&tmH);
     ptx::tma_prefetch_desc(&tmW);
@@ -509,7 +609,62 @@ __global__ void __launch_bounds__(kThreads, 1)
       ptx::mbar_wait(drain, 0, &never, kWaitLimit);
     }
     __syncwarp();
-  } else {
+  } else if (warp == kFixWarp) {
+    // ------------------------------------------------------------ FP64 pass
+    // the rows the epilogue lists, one at a time, while the epilogue goes on
+    // with later tiles (fix_row_warp); the head is read in place
+    if (fixq) {
+      const WSwz W{s_w, (uint32_t)L.Cpad * 128u};
+      const FixScratch sc = fix_scratch_at(smem + L.off_fixs, d, C);
+      volatile FixQueue* vq = fixq;
+      bool head_ok = false;
+      unsigned long long nfixed = 0;
+      for (int k = 0;; ++k) {
+        // 1: entry k is in its slot; 0: every epilogue warp is done and no
+        // entry k will come, or the kernel aborted. The wait is bounded by
+        // the epilogue's progress (a tile every few microseconds).
+        int st = 0;
+        if (lane == 0) {
+          int beat = vq->beat;
+          long long t0 = clock64();
+          for (;;) {
+            if (vq->seq[k % kFixQ] == k) {
+              st = 1;
+              break;
+            }
+            if (*abort_s) break;
+            if (vq->done == kEpiWarps) {
+              __threadfence_block();
+              if (vq->n <= k) break;  // (else the entry is being written)
+            }
+            const int b = vq->beat;
+            if (b != beat) {
+              beat = b;
+              t0 = clock64();
+            } else if (clock64() - t0 > kWaitLimit) {
+              *abort_s = 1;
+              break;
+            }
+            __nanosleep(256);
+          }
+        }
+        if (__shfl_sync(kFull, st, 0) == 0) break;
+        __threadfence_block();
+        const int row = vq->row[k % kFixQ];
+        const float kn = vq->kn[k % kFixQ];
+        if (!head_ok) head_ok = __all_sync(kFull, ptx::mbar_wait(wfull, 0, abort_s, kWaitLimit));
+        if (!head_ok) break;
+        fix_row_warp(a, (int64_t)row, kn, W, sc, lane);
+        ++nfixed;
+        __syncwarp();
+        if (lane == 0) {
+          __threadfence_block();
+          vq->taken = k + 1;
+        }
+      }
+      if (lane == 0 && nfixed) atomicAdd(&stats->ins_fp64_rows, nfixed);
+    }
+  } else if (warp < 2 + kEpiWarps) {
     // ------------------------------------------------------------ epilogue
     const int ew = warp - 2, quarter = warp & 3, half = ew >> 2;
     const int r = quarter * 32 + lane;  // row of the tile = TMEM lane
@@ -650,6 +805,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     int t = 0;
     for (int tile = blockIdx.x; tile < n_tiles; tile += gridDim.x, ++t) {
       const int buf = t & 1, zb = t % L.nzb;
+      if (fixq && ew == 0 && lane == 0) *(volatile int*)&fixq->beat = t + 1;
       bool ok = ptx::mbar_wait(accfull + 8 * buf, (uint32_t)(t >> 1) & 1u, abort_s, kWaitLimit);
       for (int c = 0; c < L.nch && ok; ++c)  // the features are visible to these threads too
         ok = ptx::mbar_wait(zfull_of(zb, c), (uint32_t)(t / L.nzb) & 1u, abort_s, kWaitLimit);
@@ -904,10 +1060,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         pair_barrier(bar_id);
         if (half == 0) {
           top2_merge(tp, x2[r]);
-          if (live)
-            row_finals(a, grow, tp.result(kn), &acc_s[r]);
-          else
+          if (live) {
+            if (row_finals(a, grow, tp.result(kn), &acc_s[r]) && fixq) fixq_push(fixq, (int)grow, kn, abort_s, kWaitLimit);
+          } else {
             acc_s[r] = 0;
+          }
           const unsigned mb = __ballot_sync(kFull, live && acc_s[r] != 0);
           if (live) a.rank[grow] = __popc(mb & ((1u << lane) - 1u));
           const int64_t blk0 = (int64_t)tile * kBM + quarter * 32;
@@ -985,17 +1142,24 @@ __global__ void __launch_bounds__(kThreads, 1)
         pair_barrier(bar_id);
         if (half == 0) {
           if (!rowfb) acc_s[r] = 0;
-          if (live && !rowfb)
-            tight_write(a, grow, yg, fmin(rmin, tx.rmin[r]), fmin(smin, tx.smin[r]), any_nan || tx.nan[r] != 0, kn,
-                        &acc_s[r]);
+          if (live && !rowfb &&
+              tight_write(a, grow, yg, fmin(rmin, tx.rmin[r]), fmin(smin, tx.smin[r]), any_nan || tx.nan[r] != 0, kn,
+                          &acc_s[r]) &&
+              fixq)
+            fixq_push(fixq, (int)grow, kn, abort_s, kWaitLimit);
         }
         // the rows the screen could not settle, alternately on the two warps
         int k = 0;
         for (unsigned fr = fbm; fr != 0; fr &= fr - 1, ++k) {
           const int ow = __ffs((int)fr) - 1;
-          if ((k & 1) == half)
-            tc_tight_row_warp(a, (int64_t)tile * kBM + rq + ow, rq + ow, s_w, wchunk, zs, wn_s, bias_s,
-                              __shfl_sync(kFull, kn, ow), lane, &acc_s[rq + ow]);
+          if ((k & 1) == half) {
+            const float knw = __shfl_sync(kFull, kn, ow);
+            const int64_t frow = (int64_t)tile * kBM + rq + ow;
+            if (tc_tight_row_warp(a, frow, rq + ow, s_w, wchunk, zs, wn_s, bias_s, knw, lane, &acc_s[rq + ow]) &&
+                fixq && lane == 0)
+              fixq_push(fixq, (int)frow, knw, abort_s, kWaitLimit);
+            __syncwarp();
+          }
         }
         __syncwarp();
         if (lane == 0) ptx::mbar_arrive(zempty + 8 * zb);  // this warp is done with the tile's features
@@ -1011,6 +1175,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0 && (n_pairs | n_full)) {
       atomicAdd(&stats->ins_pairs, n_pairs);
       atomicAdd(&stats->ins_full_rows, n_full);
+    }
+    // every row this warp lists is in the queue: the fix warp may finish
+    __syncwarp();
+    if (fixq && lane == 0) {
+      __threadfence_block();
+      atomicAdd(&fixq->done, 1);
     }
   }
   ptx::tc_fence_before();
@@ -1038,11 +1208,13 @@ void encode_rows(lipcache* h, CUtensorMap* map, const float* base, uint64_t rows
 }
 
 // Two feature buffers when they fit next to the resident head, else one.
+// The FP64 pass in the kernel when its queue and scratch fit as well.
 bool tc_plan(int d, int C, TcLayout& L) {
-  for (int nzb = 2; nzb >= 1; --nzb) {
-    L = tc_layout(d, C, nzb);
-    if (L.total <= (uint32_t)kSmemBudget) return true;
-  }
+  for (int nzb = 2; nzb >= 1; --nzb)
+    for (int infix = 1; infix >= 0; --infix) {
+      L = tc_layout(d, C, nzb, infix);
+      if (L.total <= (uint32_t)kSmemBudget) return true;
+    }
   return false;
 }
 
@@ -1063,7 +1235,7 @@ bool certify_tc_supported(const lipcache* h, const float* H, int64_t n) {
   return tc_plan(h->d, h->C, L);
 }
 
-void certify_tc_launch(lipcache* h, const CertArgs& a, cudaStream_t s) {
+bool certify_tc_launch(lipcache* h, const CertArgs& a, cudaStream_t s) {
   TcLayout L;
   LC_REQUIRE(tc_plan(h->d, h->C, L), LIPCACHE_E_INVALID, "head does not fit the tensor certify kernel");
   CUtensorMap tmH, tmW;
@@ -1079,6 +1251,7 @@ void certify_tc_launch(lipcache* h, const CertArgs& a, cudaStream_t s) {
   kern<<<grid, kThreads, smem, s>>>(tmH, tmW, a, L, n_tiles, h->stats,
                                     (h->debug_flags & LIPCACHE_DEBUG_STALL_INSERT) ? 1 : 0);
   LC_LAUNCH_CHECK("k_certify_tc");
+  return L.infix != 0;
 }
 
 }  // namespace lc
