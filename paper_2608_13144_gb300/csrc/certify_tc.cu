@@ -352,10 +352,35 @@ __device__ __forceinline__ void refine2(uint32_t ws, uint32_t wchunk, uint32_t z
     P = sm;
     CC = add_f32x2(CC, add_f32x2(q, er));
   };
+  // a chunk's sixteen loads are issued together, then its four steps (the
+  // loads are volatile, so their order is the program's)
+  auto ld = [](uint32_t addr) {
+    float v;
+    asm volatile("ld.shared.f32 %0, [%1];" : "=f"(v) : "r"(addr));
+    return v;
+  };
+  auto step_v = [&](float w0, float x0, float w1, float x1) {
+    const uint64_t w = pack2_f32(w0, w1), x = pack2_f32(x0, x1);
+    const uint64_t pr = mul_f32x2(w, x);                // TwoProduct: pr + er = w x
+    const uint64_t er = ptx::fma_f32x2(w, x, pr ^ kSign2);
+    const uint64_t sm = add_f32x2(P, pr);               // TwoSum(P, pr) = sm + q
+    const uint64_t bb = ptx::sub_f32x2(sm, P);
+    const uint64_t q = add_f32x2(ptx::sub_f32x2(P, ptx::sub_f32x2(sm, bb)), ptx::sub_f32x2(pr, bb));
+    P = sm;
+    CC = add_f32x2(CC, add_f32x2(q, er));
+  };
   const int nfull = d >> 5;
   for (int kc = 0; kc < nfull; ++kc) {
+    float w0[4], x0[4], w1[4], x1[4];
 #pragma unroll
-    for (int jj = 0; jj < 4; ++jj) step(wb[0] + ow[0][jj], zb[0] + oz[0][jj], wb[1] + ow[1][jj], zb[1] + oz[1][jj]);
+    for (int jj = 0; jj < 4; ++jj) {
+      w0[jj] = ld(wb[0] + ow[0][jj]);
+      x0[jj] = ld(zb[0] + oz[0][jj]);
+      w1[jj] = ld(wb[1] + ow[1][jj]);
+      x1[jj] = ld(zb[1] + oz[1][jj]);
+    }
+#pragma unroll
+    for (int jj = 0; jj < 4; ++jj) step_v(w0[jj], x0[jj], w1[jj], x1[jj]);
 #pragma unroll
     for (int u = 0; u < 2; ++u) {
       wb[u] += wchunk;
