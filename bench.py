@@ -42,6 +42,7 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 TF32_OVER_BF16 = 1.1 / 2.25  # nominal dense TF32 / BF16 tensor rates of GB300
 # LIPCACHE_DEBUG_INSERT_WIDE_TILE / LIPCACHE_DEBUG_INSERT_TILE64 of the C ABI
 INSERT_KERNEL_FLAGS = {"auto": 0, "wide": 4, "tile64": 2}
+DEBUG_INSERT_FIX_STANDALONE = 16  # LIPCACHE_DEBUG_INSERT_FIX_STANDALONE
 
 
 def parse():
@@ -61,6 +62,9 @@ def parse():
     p.add_argument("--dup", type=float, default=None, help="override the fraction of near-duplicate queries")
     p.add_argument("--insert-kernel", default="auto", choices=sorted(INSERT_KERNEL_FLAGS),
                    help="certify on an FP32 kernel instead of the default choice (profiling)")
+    p.add_argument("--insert-fp64-pass", default="kernel", choices=["kernel", "standalone"],
+                   help="where the tensor certify kernel's listed rows are re-certified in FP64: on its own "
+                        "spare warp (default) or by the stand-alone pass launched after it (profiling)")
     return p.parse_args()
 
 
@@ -364,8 +368,10 @@ def run_ours(args, dist: Dist):
         call; the accepted total comes from the size afterwards), and the
         library's events around each certify kernel."""
         c = LipCache(w.d, w.C, w.N, mode, device=dev)
-        if INSERT_KERNEL_FLAGS[args.insert_kernel]:
-            c.set_debug(INSERT_KERNEL_FLAGS[args.insert_kernel])
+        flags = INSERT_KERNEL_FLAGS[args.insert_kernel] | (
+            DEBUG_INSERT_FIX_STANDALONE if args.insert_fp64_pass == "standalone" else 0)
+        if flags:
+            c.set_debug(flags)
         sig = c.set_head(torch.from_numpy(W).to(dev), torch.from_numpy(b).to(dev))
         torch.cuda.synchronize(dev)
         c.enable_timing(True)
@@ -488,6 +494,8 @@ def run_ours(args, dist: Dist):
                   "device_errors": info["device_errors"], "kernel_ms": kernel_ms,
                   "grid": info["last_grid"], "cluster": info["last_cluster"]},
     }
+    for k in ("insert", "insert_tight"):
+        line[k]["fp64_pass"] = "stand-alone kernel" if args.insert_fp64_pass == "standalone" else "in the kernel"
     return line
 
 

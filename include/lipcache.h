@@ -384,6 +384,11 @@ lipcache_status lipcache_read_head(lipcache_t* h, float* W_host, float* b_host, 
  * appended and lipcache_insert (and the other certifying entry points)
  * return LIPCACHE_E_DEVICE with the cache unchanged. */
 #define LIPCACHE_DEBUG_STALL_INSERT 8
+/* The tensor certify kernel leaves the rows it lists for the FP64 pass to
+ * the stand-alone pass launched after it, instead of re-certifying them on
+ * its own spare warp; both compute the same values (tests compare them bit
+ * for bit; the bench times both). */
+#define LIPCACHE_DEBUG_INSERT_FIX_STANDALONE 16
 lipcache_status lipcache_set_debug(lipcache_t* h, int32_t flags);
 
 /*

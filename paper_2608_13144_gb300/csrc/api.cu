@@ -527,7 +527,8 @@ LC_API lipcache_status lipcache_set_debug(lipcache_t* h, int32_t flags) {
   return guarded([&] {
     check_handle(h);
     LC_REQUIRE((flags & ~(LIPCACHE_DEBUG_STALL_PROBE | LIPCACHE_DEBUG_INSERT_TILE64 |
-                          LIPCACHE_DEBUG_INSERT_WIDE_TILE | LIPCACHE_DEBUG_STALL_INSERT)) == 0,
+                          LIPCACHE_DEBUG_INSERT_WIDE_TILE | LIPCACHE_DEBUG_STALL_INSERT |
+                          LIPCACHE_DEBUG_INSERT_FIX_STANDALONE)) == 0,
                LIPCACHE_E_INVALID,
                "unknown debug flags");
     h->debug_flags = flags;

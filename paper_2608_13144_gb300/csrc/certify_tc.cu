@@ -1233,10 +1233,11 @@ void encode_rows(lipcache* h, CUtensorMap* map, const float* base, uint64_t rows
 }
 
 // Two feature buffers when they fit next to the resident head, else one.
-// The FP64 pass in the kernel when its queue and scratch fit as well.
-bool tc_plan(int d, int C, TcLayout& L) {
+// The FP64 pass in the kernel when its queue and scratch fit as well (and
+// `fix_in_kernel` allows it).
+bool tc_plan(int d, int C, TcLayout& L, bool fix_in_kernel = true) {
   for (int nzb = 2; nzb >= 1; --nzb)
-    for (int infix = 1; infix >= 0; --infix) {
+    for (int infix = fix_in_kernel ? 1 : 0; infix >= 0; --infix) {
       L = tc_layout(d, C, nzb, infix);
       if (L.total <= (uint32_t)kSmemBudget) return true;
     }
@@ -1262,7 +1263,8 @@ bool certify_tc_supported(const lipcache* h, const float* H, int64_t n) {
 
 bool certify_tc_launch(lipcache* h, const CertArgs& a, cudaStream_t s) {
   TcLayout L;
-  LC_REQUIRE(tc_plan(h->d, h->C, L), LIPCACHE_E_INVALID, "head does not fit the tensor certify kernel");
+  LC_REQUIRE(tc_plan(h->d, h->C, L, !(h->debug_flags & LIPCACHE_DEBUG_INSERT_FIX_STANDALONE)), LIPCACHE_E_INVALID,
+             "head does not fit the tensor certify kernel");
   CUtensorMap tmH, tmW;
   encode_rows(h, &tmH, a.H, (uint64_t)a.n, kBM);
   encode_rows(h, &tmW, h->W, (uint64_t)h->C, (uint32_t)L.Cpad);

@@ -80,9 +80,9 @@ def test_debug_flags_validated(dev):
     from paper_2608_13144_gb300.lipcache import LipCache
     c = LipCache(4, 2, 8, device=dev)
     with pytest.raises(LipCacheError) as e:
-        c.set_debug(16)
+        c.set_debug(32)
     assert e.value.status == 1
-    c.set_debug(2 | 4 | 8)  # every known flag together is accepted
+    c.set_debug(2 | 4 | 8 | 16)  # every known flag together is accepted
     c.set_debug(0)
     c.close()
 

@@ -17,7 +17,7 @@ torch = pytest.importorskip("torch")
 pytestmark = pytest.mark.gpu
 
 WIDE_TILE, TILE64, STREAMED, TENSOR = 1, 2, 3, 4
-DEBUG_INSERT_TILE64, DEBUG_INSERT_WIDE_TILE = 2, 4
+DEBUG_INSERT_TILE64, DEBUG_INSERT_WIDE_TILE, DEBUG_INSERT_FIX_STANDALONE = 2, 4, 16
 
 
 @pytest.fixture(scope="module")
@@ -280,6 +280,36 @@ def test_wide_tile_near_ties(dev, d, C, kernel):
           rep["fp64_band"])
     a.close()
     s.close()
+
+
+@pytest.mark.parametrize("mode", ["conservative", "tight"])
+@pytest.mark.parametrize("d,C", [(64, 40), (128, 200), (96, 250)])
+def test_tensor_fp64_pass_in_kernel_and_standalone(dev, mode, d, C):
+    """The tensor kernel's own FP64-pass warp (rows handed over through its
+    shared-memory queue while the epilogue goes on) and the stand-alone pass
+    launched after the kernel re-certify the same listed rows to the same
+    bits: near-tie rows, several per tile, more than the queue's 32 slots per
+    CTA in a launch."""
+    from paper_2608_13144_gb300.lipcache import LipCache
+    rng = np.random.default_rng(7 * d + C)
+    W = (rng.standard_normal((C, d)) / np.sqrt(d)).astype(np.float32)
+    b = (0.1 * rng.standard_normal(C)).astype(np.float32)
+    rows = np.concatenate([_near_ties(W, b, 1500, rng, 2), _near_ties(W, b, 500, rng, 3),
+                           rng.standard_normal((2000, d)).astype(np.float32)])
+    rows = rows[rng.permutation(len(rows))]
+    out = []
+    for flags in (0, DEBUG_INSERT_FIX_STANDALONE):
+        c = LipCache(d, C, len(rows), mode, device=dev)
+        c.set_head(T(W, dev), T(b, dev))
+        c.set_debug(flags)
+        i, r, n = c.insert(T(rows, dev))
+        inf = c.info()
+        assert inf["last_insert_kernel"] == TENSOR
+        out.append((i.cpu().numpy(), r.cpu().numpy(), n, inf["insert_fp64_rows"]))
+        c.close()
+    (ia, ra, na, fa), (ib, rb, nb, fb) = out
+    assert fa == fb and fa > 64, (fa, fb)
+    assert na == nb and same_bits(ia, ib) and same_bits(ra, rb)
 
 
 def build_tight(dev, W, b, rows, tile64, kappa=1.0):
