@@ -56,6 +56,9 @@ def parse():
     p.add_argument("--cpu-seconds", type=float, default=15.0, help="budget of the oracle CPU baseline")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-tf32-peak", action="store_true", help="skip the live cuBLAS TF32 peak measurement")
+    p.add_argument("--sustain-s", type=float, default=3.0,
+                   help="seconds of back-to-back probe steps after the timed region, reported as `sustained` "
+                        "with their clocks (0: skip)")
     p.add_argument("--cache-rows", type=int, default=0, help="override the workload's cache size N (profiling)")
     p.add_argument("--noise", type=float, default=None,
                    help="override the near-duplicate queries' per-feature noise (e.g. 0.002: most of them hit)")
@@ -434,6 +437,34 @@ def run_ours(args, dist: Dist):
 
     value, tmax = aggregate(dist, args.steps * B, step_s)
 
+    # the same step back to back for a few seconds, with its clocks: the
+    # figure under the power cap beside the short timed region's
+    sustained = None
+    if args.sustain_s > 0:
+        cache.reset_stats()
+        cache.enable_timing(True)
+        clk2 = Clocks(dist.local_rank)
+        torch.cuda.synchronize(dev)
+        clk2.mark_start()
+        s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        s0.record(stream)
+        n_sus, t_wall = 0, time.perf_counter()
+        while time.perf_counter() - t_wall < args.sustain_s:
+            for _ in range(16):
+                cache.probe(Qd[n_sus % nb], out=outs[n_sus % nb])
+                n_sus += 1
+            torch.cuda.synchronize(dev)
+        s1.record(stream)
+        torch.cuda.synchronize(dev)
+        clk2.mark_end()
+        sus_s = s0.elapsed_time(s1) * 1e-3
+        inf2 = cache.info()
+        cache.enable_timing(False)
+        k2_ms = inf2["kernel_ms_total"] / max(1, inf2["kernel_launches"])
+        sustained = {"value": n_sus * B / sus_s, "unit": "queries/s", "steps": n_sus, "seconds": sus_s,
+                     "kernel_ms": k2_ms, "kernel_tflops": 2.0 * B * N * w.d / (k2_ms * 1e-3) / 1e12,
+                     "clocks": clk2.stop()}
+
     # end to end through the host-buffer entry point: H2D of the queries,
     # probe, D2H of index/label/distance, every step
     hq = [torch.from_numpy(np.ascontiguousarray(Q[i * B:(i + 1) * B])).pin_memory() for i in range(nb)]
@@ -483,6 +514,7 @@ def run_ours(args, dist: Dist):
         "e2e": {"value": e2e_value, "unit": "queries/s", "h2d_bytes_per_step": B * w.d * 4,
                 "d2h_bytes_per_step": B * (8 + 4 + 4)},
         "gpu_launches": 3 * args.steps,
+        "sustained": sustained,
         "clocks": clocks,
         "insert": insert_summary(w, n_acc, insert_ms, torch.cuda.get_device_properties(dev).multi_processor_count,
                                  clocks, kernel=insert_kernel, tf32_peak=tf32_derived, hbm_peak=pk["hbm_gbs"]),

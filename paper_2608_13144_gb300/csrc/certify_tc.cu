@@ -29,8 +29,9 @@
 // classes whose lower bracket of (s_y - s_j) / ||W_y - W_j|| reaches u_{y2},
 // first with the head row's smallest reciprocal pair norm, then with the
 // class's own (the minimiser of Eq. 29 always passes). Otherwise one test
-// valid for every possible y^G (lower end above lo_1 - 2E, r* below a bound
-// from y1's row) picks the candidates, and y^G is the largest refined one.
+// valid for every possible y^G (its logit above lo_1, since it is at least
+// s_y1; r* below a bound from y1's row) picks the candidates, and y^G is the
+// largest refined one.
 // Each half reduces Eq. 29 over its own candidates in FP64; rows with more
 // candidates than slots take a one-warp path over every class.
 //
@@ -925,10 +926,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       // from above and (lo_1 - hi_j) ipn_min(y1) <= l_j bounds every class's
       // bracket from below, so the minimiser of Eq. 29 passes (lo_1 - hi_j)
       // ipn_min(y1) <= U1 (then also with its own bracket l_j). Otherwise every
-      // possible y^G has its lower end above lo* = lo_1 - 2E (less rounding) and
-      // r*/kappa below U* (below), so one test with lo*, U* and the head's
-      // smallest ipn keeps the minimiser for whichever class is y^G; y^G is
-      // then the largest refined candidate.
+      // possible y^G has s_{y^G} >= s_y1 >= lo_1 and r*/kappa below U* (below),
+      // so one test with lo_1, U* and the head's smallest ipn keeps the
+      // minimiser for whichever class is y^G; y^G is then the largest refined
+      // candidate.
       float lo1 = 0.f, U1 = 0.f, im1 = 0.f;
       bool unc = false;
       if constexpr (TIGHT) {
@@ -949,7 +950,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             // the pair norm ||W_y1 - W_y2||, so the first term bounds it.
             U1 = fmaxf(__fmul_ru(__fsub_ru(hi1, lo2), __ldg(a.ipn_up32 + (size_t)y * C + j2)),
                        __fmul_ru(__fsub_ru(hi2, lo1), __ldg(a.ipn_max32 + y)));
-            lo1 = __fsub_rd(lo1, __fmaf_ru(E, 2.0001f, __fmaf_ru(fabsf(lo1), 9.5367432e-07f /* 2^-20 */, kTinyF)));
+            // lo_1 itself bounds s_{y^G} from below (s_{y^G} >= s_y1 >= lo_1)
             im1 = imA;
           }
         }

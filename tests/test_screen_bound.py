@@ -164,9 +164,9 @@ def screen_tight(st, E, ipn, ipn_min, ipn_max):
             return np.flatnonzero(cand), y1
         second = (hi2 - lo1) * ipn_max[y1]  # NaN (0 x inf) is dropped, as fmaxf does
         U = np.fmax(first, second)
-        lo = lo1 - (2.0001 * E + 2.0 ** -20 * abs(lo1))
+        # any y^G has s >= s_y1 >= lo_1: lo_1 bounds it from below
         imA = ipn_min.min()
-        cand = (lo - h) * imA <= U
+        cand = (lo1 - h) * imA <= U
     return np.flatnonzero(cand), None
 
 
@@ -275,30 +275,27 @@ def test_tight_screen_needs_the_second_term():
     assert certain is None and 3 in cand
     assert refine(s, cand, pn, None) == (y_ref, r_ref)
     # the first term alone would not keep class 3
-    lo = -1.0 - (2.0001 * E + 2.0 ** -20)
+    lo = -1.0
     assert (lo - (st[3] + E)) * ipn_min.min() > (2.0 * E) * ipn[0, 1]
 
 
-def test_tight_screen_lower_end_slack():
-    """lo* = lo_1 - 2E is wider than soundness needs: any y^G has s >= s_y1 >=
-    lo_1, so the union test with lo_1 (less the refinement's rounding) keeps
-    the minimiser too. Checked on the random cases with lo* = lo_1."""
-    rng = np.random.default_rng(5)
-    for trial in range(400):
-        C = int(rng.integers(3, 12))
-        W = rng.standard_normal((C, 3))
-        s = W @ rng.standard_normal(3) + rng.standard_normal(C) * 0.3
-        E = (float(np.ptp(s)) + 1e-3) * float(rng.choice([1e-2, 0.1, 0.5]))
-        st = s + rng.choice([-E, E], C)
-        pn, ipn, ipn_min, ipn_max = pair_tables(W)
-        y1, y2 = top2_lowest(st)
-        lo1, hi1, lo2, hi2 = st[y1] - E, st[y1] + E, st[y2] - E, st[y2] + E
-        if hi2 < lo1:
-            continue
-        with np.errstate(invalid="ignore"):
-            U = np.fmax((hi1 - lo2) * ipn[y1, y2], (hi2 - lo1) * ipn_max[y1])
-            cand = np.flatnonzero((lo1 - (st + E)) * ipn_min.min() <= U)
-        assert refine(s, cand, pn, None) == oracle_tight(s, pn), trial
+def test_tight_screen_lower_end_is_tight():
+    """The union test's lower end lo_1 is the best the screen allows: a true
+    y^G can sit exactly at lo_1 (its logit equal to s_y1 = lo_1), and then a
+    lower end above lo_1 would drop a minimiser the oracle needs. Row: y1 and
+    the true y^G tie at lo_1 (y1 read E too high), the minimiser j far below."""
+    W = np.array([[1.0, 0.0], [0.0, 1.0], [1.0, 1.0], [-3.0, 0.0]])
+    s = np.array([1.0, 1.0, 0.5, -6.0])  # classes 0 and 1 tie on top
+    E = 0.5
+    st = np.array([1.5, 1.0, 0.5, -5.5])  # |s~ - s| <= E; y1 = 0 with lo_1 = 1.0 = s_0
+    assert np.all(np.abs(st - s) <= E)
+    pn, ipn, ipn_min, ipn_max = pair_tables(W)
+    cand, certain = screen_tight(st, E, ipn, ipn_min, ipn_max)
+    y_ref, r_ref = oracle_tight(s, pn)
+    assert y_ref in cand
+    assert refine(s, cand, pn, certain) == (y_ref, r_ref)
+    y1 = top2_lowest(st)[0]
+    assert st[y1] - E == s[y_ref]  # the bound is attained
 
 
 # ---------------------------------------------------------------------------
