@@ -416,17 +416,40 @@ __device__ __forceinline__ void refine2(uint32_t ws, uint32_t wchunk, uint32_t z
 
 // The tight radius (Eq. 29) of one row on one warp, for rows the screen
 // cannot settle (several possible y^G, Mb not below 1e38, more candidates than
-// slots): every class refined with the compensated dot product (lane = class,
-// features in order, as the wide-tile kernel's fallback), y^G the largest
-// refined logit (lowest class on ties), then Eq. 29 over every other class in
-// FP64. The row's features come from the tile in shared memory (row rz).
+// slots): every class refined with the compensated dot product by the four
+// 8-lane groups, two classes per group at a time (refine2, the error factor of
+// 8-lane groups), into the warp's result cells by class; then, lane = class,
+// y^G the largest refined logit (lowest class on ties) and Eq. 29 over every
+// other class in FP64. The row's features come from the tile in shared memory
+// (row rz). res_hi / res_lo: the warp's cells (at least 256 each), free here.
 // Returns (on every lane) whether the row was listed for the FP64 pass.
 __device__ bool tc_tight_row_warp(const CertArgs& a, int64_t row, int rz, uint32_t s_w, uint32_t wchunk, uint32_t zs,
                                   const float* __restrict__ wn_s, const float* __restrict__ b_s, float kn, int lane,
-                                  uint8_t* acc_slot) {
+                                  float* res_hi, float* res_lo, uint8_t* acc_slot) {
   constexpr int kPer = 8;  // classes per lane (C <= 256)
   const int d = a.d, C = a.C;
+  const int g8 = lane / kGroupTc, sub = lane % kGroupTc;
   const float hn = norm_upper(kn);
+  for (int c0 = 0; c0 < C; c0 += 2 * (32 / kGroupTc)) {
+    int cp[2];
+#pragma unroll
+    for (int u = 0; u < 2; ++u) {
+      const int c = c0 + 2 * g8 + u;
+      cp[u] = c < C ? c : C - 1;  // a valid class; the result is not stored
+    }
+    const int rp[2] = {rz, rz};
+    const float bp[2] = {b_s[cp[0]], b_s[cp[1]]};
+    float hi[2], lo[2];
+    refine2(s_w, wchunk, zs, cp, rp, bp, d, sub, hi, lo);
+    if (sub == 0)
+#pragma unroll
+      for (int u = 0; u < 2; ++u)
+        if (c0 + 2 * g8 + u < C) {
+          res_hi[c0 + 2 * g8 + u] = hi[u];
+          res_lo[c0 + 2 * g8 + u] = lo[u];
+        }
+  }
+  __syncwarp();
   float vh[kPer], vl[kPer], ve[kPer];
   float bh = -INFINITY, bl = 0.f;
   int by = -1;
@@ -438,24 +461,10 @@ __device__ bool tc_tight_row_warp(const CertArgs& a, int64_t row, int rz, uint32
     vl[t] = 0.f;
     ve[t] = 0.f;
     if (c < C) {
-      float p = 0.f, cc = 0.f;
-      for (int k = 0; k < d; ++k) {
-        float w, x;
-        asm volatile("ld.shared.f32 %0, [%1];" : "=f"(w) : "r"(s_w + sw_off(c, k, wchunk)));
-        asm volatile("ld.shared.f32 %0, [%1];" : "=f"(x) : "r"(zs + sw_off(rz, k, kZChunkBytes)));
-        const float pr = __fmul_rn(w, x);
-        const float er = __fmaf_rn(w, x, -pr);
-        float s1, q;
-        two_sum(p, pr, s1, q);
-        p = s1;
-        cc = __fadd_rn(cc, __fadd_rn(q, er));
-      }
-      float s1, q, hi, lo;
-      two_sum(p, b_s[c], s1, q);
-      two_sum(s1, __fadd_rn(cc, q), hi, lo);
+      const float hi = res_hi[c], lo = res_lo[c];
       vh[t] = hi;
       vl[t] = lo;
-      ve[t] = refined_err(a.g2f, wn_s[c], hn, b_s[c]);
+      ve[t] = refined_err(a.g2f8, wn_s[c], hn, b_s[c]);
       nan_any |= !(hi == hi && lo == lo);
       if (pair_gt(hi, lo, bh, bl)) {  // ascending classes: ties keep the lowest
         bh = hi;
@@ -464,6 +473,7 @@ __device__ bool tc_tight_row_warp(const CertArgs& a, int64_t row, int rz, uint32
       }
     }
   }
+  __syncwarp();  // the cells are read before the next row's refinement
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
     const float oh = __shfl_xor_sync(kFull, bh, o), ol = __shfl_xor_sync(kFull, bl, o);
@@ -1181,7 +1191,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           if ((k & 1) == half) {
             const float knw = __shfl_sync(kFull, kn, ow);
             const int64_t frow = (int64_t)tile * kBM + rq + ow;
-            if (tc_tight_row_warp(a, frow, rq + ow, s_w, wchunk, zs, wn_s, bias_s, knw, lane, &acc_s[rq + ow]) &&
+            if (tc_tight_row_warp(a, frow, rq + ow, s_w, wchunk, zs, wn_s, bias_s, knw, lane, res_hi, res_lo,
+                                  &acc_s[rq + ow]) &&
                 fixq && lane == 0)
               fixq_push(fixq, (int)frow, knw, abort_s, kWaitLimit);
             __syncwarp();
