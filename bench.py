@@ -214,6 +214,32 @@ def roofline(w: synth.Workload, N: int, B: int, kernel_ms: float, pk: dict, pk_k
             "peak_source": f"{pk_kind} copy bandwidth", "kernel": kernel, "kernel_ms": kernel_ms}
 
 
+def event_floor_ms(dev, reps: int = 50) -> float:
+    """CUDA-event interval of a one-element kernel launched right after
+    another small kernel, bracketed the way the library brackets each probe
+    kernel (event, kernel, event): the fixed cost inside every per-kernel
+    interval on this GPU (kernel launch and completion), median of `reps`."""
+    import torch
+
+    x = torch.zeros(1, device=dev)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    stream = torch.cuda.current_stream(dev)
+    out = []
+    for i in range(reps + 5):
+        # the GPU sleeps while the rest is queued, so the interval holds no
+        # host-side launch time (as in the probe's timed loop, where the host
+        # runs ahead of the GPU)
+        torch.cuda._sleep(1_000_000)
+        x.add_(1.0)
+        e0.record(stream)
+        x.mul_(1.0)
+        e1.record(stream)
+        torch.cuda.synchronize(dev)
+        if i >= 5:
+            out.append(e0.elapsed_time(e1))
+    return statistics.median(out)
+
+
 def measure_tf32_peak(dev, n: int = 8192, reps: int = 10, sustain_s: float = 2.0) -> dict:
     """Dense TF32 tensor throughput of this GPU, measured in this run the way
     the BF16 peak of MEASURED_PEAKS.json was: a cuBLAS (torch.matmul) FP32 GEMM
@@ -497,6 +523,10 @@ def run_ours(args, dist: Dist):
         rf["tf32_measured"] = tf
     if path_id in (3, 4) and w.N == synth.WORKLOADS[w.name].N:
         rf["traffic"] = recorded_traffic(w.name, path_id)
+    # context for short kernels: the part of each per-kernel event interval
+    # that any kernel pays (launch, completion); the fraction above is not
+    # corrected for it
+    rf["event_floor_ms"] = event_floor_ms(dev)
     line = {
         "metric": METRIC, "value": value, "unit": "queries/s", "n_gpus": dist.world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": tmax / args.steps * 1e3, "higher_is_better": True,
