@@ -1355,7 +1355,6 @@ __global__ void __launch_bounds__(1024) k_scan(int32_t* __restrict__ cnt, int32_
                                                int64_t* __restrict__ size_dev, int64_t* __restrict__ size0,
                                                const int32_t* __restrict__ fix_list, const uint8_t* __restrict__ accept,
                                                int32_t* __restrict__ rank, int64_t n) {
-  __shared__ int32_t buf[1024];
   __shared__ int64_t carry;
   const int tid = threadIdx.x;
   if (tid == 0) carry = 0;
@@ -1373,20 +1372,38 @@ __global__ void __launch_bounds__(1024) k_scan(int32_t* __restrict__ cnt, int32_
     cnt[r0 / kRows] = c;
   }
   __syncthreads();
-  for (int base = 0; base < nb; base += 1024) {
-    const int i = base + tid;
-    const int v = (i < nb && st->abort_flag == 0) ? cnt[i] : 0;
-    buf[tid] = v;
-    __syncthreads();
-    for (int s = 1; s < 1024; s <<= 1) {
-      const int t = tid >= s ? buf[tid - s] : 0;
-      __syncthreads();
-      buf[tid] += t;
-      __syncthreads();
+  // exclusive scan, 2,048 counts a pass: two per thread, warp shuffles, then
+  // the 32 warp totals on one warp
+  __shared__ int32_t wsum[32];
+  const int lane = tid & 31, warp = tid >> 5;
+  const bool live = st->abort_flag == 0;
+  for (int base = 0; base < nb; base += 2048) {
+    const int i0 = base + 2 * tid;
+    const int v0 = (i0 < nb && live) ? cnt[i0] : 0;
+    const int v1 = (i0 + 1 < nb && live) ? cnt[i0 + 1] : 0;
+    int x = v0 + v1;  // inclusive scan of the thread pairs within the warp
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, x, o);
+      if (lane >= o) x += y;
     }
-    if (i < nb) off[i] = (int32_t)(carry + buf[tid] - v);
+    if (lane == 31) wsum[warp] = x;
     __syncthreads();
-    if (tid == 1023) carry += buf[1023];
+    if (warp == 0) {
+      int w = wsum[lane];
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, w, o);
+        if (lane >= o) w += y;
+      }
+      wsum[lane] = w;  // inclusive over the warps
+    }
+    __syncthreads();
+    const int64_t before = carry + (warp > 0 ? wsum[warp - 1] : 0) + (x - v0 - v1);
+    if (i0 < nb) off[i0] = (int32_t)before;
+    if (i0 + 1 < nb) off[i0 + 1] = (int32_t)(before + v0);
+    __syncthreads();
+    if (tid == 0) carry += wsum[31];
     __syncthreads();
   }
   if (tid == 0) {
