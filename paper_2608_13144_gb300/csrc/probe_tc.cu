@@ -59,9 +59,12 @@ constexpr int kCluster = 2;
 constexpr uint16_t kClusterMask = 0x3;
 constexpr int kSmemBudget = 227 * 1024 - 1024;  // opt-in limit minus the alignment slack
 constexpr long long kWaitLimit = 1LL << 31;     // ~1 s at GB300 clocks
+constexpr int64_t kPairedReleaseItems = 64;     // items per cluster from which stages are released in pairs
 
 struct TcArgs {
   int nst;       // query ring stages
+  int qgroup;    // stages released together, 1 or 2 (the kernel instantiation; divides nst)
+  int tau_staged;  // screen terms copied to shared memory per run (short runs), else read through L1
   int nch;       // d_pad / 32
   int dpad;
   int nq;        // query tiles
@@ -81,20 +84,20 @@ template <int BN>
 struct Layout {
   static constexpr int kKChunkBytes = BN * 128;
   static constexpr int kTmemCols = 2 * BN;
-  static constexpr int kTauBytes = 4 * BN * 4;  // one private tau slice per epilogue warp (kEpiWarps x 4BN/kEpiWarps)
-  int nch, nst;
+  static constexpr int kTauStaged = 4 * BN * 4;  // one private slice of screen terms per epilogue warp
+  int nch, nst, tau_staged;  // tau_staged: the screen terms copied per run (else read through L1)
   __device__ __host__ int kbytes() const { return nch * kKChunkBytes; }
   __device__ __host__ int qoff() const { return kbytes(); }
   __device__ __host__ int tauoff() const { return qoff() + nst * kQStageBytes; }
-  __device__ __host__ int baroff() const { return tauoff() + kTauBytes; }
+  __device__ __host__ int baroff() const { return tauoff() + (tau_staged ? kTauStaged : 0); }
   // barriers: full_k[nch], empty_k[nch], full_q[nst], empty_q[nst], acc_full[2], acc_empty[2], drain
   __device__ __host__ int nbar() const { return 2 * nch + 2 * nst + 5; }
   __device__ __host__ int miscoff() const { return baroff() + 8 * nbar(); }
   __device__ __host__ int total() const { return miscoff() + 16; }
   // deepest ring that fits the shared-memory budget
-  static __host__ int stages_for(int nch) {
+  static __host__ int stages_for(int nch, int tau_staged) {
     for (int n = kMaxStages; n >= 2; --n) {
-      Layout<BN> L{nch, n};
+      Layout<BN> L{nch, n, tau_staged};
       if (L.total() <= kSmemBudget) return n;
     }
     return 0;
@@ -122,14 +125,19 @@ struct RunCursor {
   }
 };
 
-template <int BN>
+// MODE 0: short ranges (screen terms staged in shared memory, stages released
+// one at a time); 1: long ranges (screen terms through L1), single releases;
+// 2: long ranges, stages released in pairs.
+template <int BN, int MODE>
 __global__ void __launch_bounds__(kThreads, 1)
     k_probe_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK, const TcArgs a) {
+  constexpr int QG = MODE == 2 ? 2 : 1;  // query stages released together
+  constexpr bool kTauStaged = MODE == 0;
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   // 1024-byte alignment of the swizzled tiles
   unsigned char* smem =
       reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
-  const Layout<BN> L{a.nch, a.nst};
+  const Layout<BN> L{a.nch, a.nst, a.tau_staged};
   const uint32_t s_base = ptx::smem_u32(smem);
   const uint32_t s_k = s_base;
   const uint32_t s_q = s_base + L.qoff();
@@ -137,7 +145,6 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t full_k = s_bar, empty_k = s_bar + 8 * a.nch;
   const uint32_t full_q = s_bar + 16 * a.nch, empty_q = full_q + 8 * a.nst;
   const uint32_t acc_full = empty_q + 8 * a.nst, acc_empty = acc_full + 16, drain = acc_empty + 16;
-  float* tau_s = reinterpret_cast<float*>(smem + L.tauoff());
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L.miscoff());
   volatile int* abort_s = reinterpret_cast<volatile int*>(smem + L.miscoff() + 4);
 
@@ -203,9 +210,12 @@ __global__ void __launch_bounds__(kThreads, 1)
               ptx::tma_load_2d(s_k + c * Layout<BN>::kKChunkBytes, &tmK, c * kChunkF, kt * BN, full_k + 8 * c);
               last_k_par[c] = i & 1;
             }
-            // stage qs is free in both CTAs; fetch this CTA's half for both
-            ok = ptx::mbar_wait(empty_q + 8 * qs, qph ^ 1u, abort_s, kWaitLimit);
-            if (!ok) break;
+            // stage qs is free in both CTAs (its group was released); fetch
+            // this CTA's half for both
+            if (QG == 1 || (qs & 1) == 0) {
+              ok = ptx::mbar_wait(empty_q + 8 * (qs >> (QG - 1)), qph ^ 1u, abort_s, kWaitLimit);
+              if (!ok) break;
+            }
             ptx::mbar_expect_tx(full_q + 8 * qs, (uint32_t)kQStageBytes);
             ptx::tma_load_2d_multicast(s_q + qs * kQStageBytes + rank * kQHalfBytes, &tmQ, c * kChunkF,
                                        qt * kBM + (int)rank * (kBM / 2), full_q + 8 * qs, kClusterMask);
@@ -274,8 +284,40 @@ __global__ void __launch_bounds__(kThreads, 1)
               ptx::mma_tf32(d_tmem, qd + 2, kd + 2, idesc, 1u);
               ptx::mma_tf32(d_tmem, qd + 4, kd + 4, idesc, 1u);
               ptx::mma_tf32(d_tmem, qd + 6, kd + 6, idesc, 1u);
-              ptx::mma_commit_multicast(empty_q + 8 * qs, kClusterMask);
+              if (QG == 1 || (qs & 1)) ptx::mma_commit_multicast(empty_q + 8 * (qs >> (QG - 1)), kClusterMask);
               if (last) ptx::mma_commit(empty_k + 8 * c);
+              if (++qs == nst) {
+                qs = 0;
+                qph ^= 1u;
+              }
+            }
+          } else if (QG == 2) {
+            // Steady state, stages released in pairs (nch and nst even, so
+            // a tile starts on the first stage of a pair): the stage waits,
+            // eight MMAs and one release per two stages, no predicated
+            // tensor-pipe instructions.
+            for (int c = 0; c < nch && ok; c += 2, kd += 2 * kKStride) {
+              if (!ptx::mbar_wait(full_q + 8 * qs, qph, abort_s, kWaitLimit)) {
+                ok = false;
+                break;
+              }
+              uint64_t qd = qdesc0 + (uint64_t)qs * kQStride;
+              ptx::mma_tf32(d_tmem, qd, kd, idesc, c != 0);
+              ptx::mma_tf32(d_tmem, qd + 2, kd + 2, idesc, 1u);
+              ptx::mma_tf32(d_tmem, qd + 4, kd + 4, idesc, 1u);
+              ptx::mma_tf32(d_tmem, qd + 6, kd + 6, idesc, 1u);
+              ++qs;  // (even, below nst - 1: no wrap)
+              if (!ptx::mbar_wait(full_q + 8 * qs, qph, abort_s, kWaitLimit)) {
+                ok = false;
+                break;
+              }
+              qd = qdesc0 + (uint64_t)qs * kQStride;
+              const uint64_t kd1 = kd + kKStride;
+              ptx::mma_tf32(d_tmem, qd, kd1, idesc, 1u);
+              ptx::mma_tf32(d_tmem, qd + 2, kd1 + 2, idesc, 1u);
+              ptx::mma_tf32(d_tmem, qd + 4, kd1 + 4, idesc, 1u);
+              ptx::mma_tf32(d_tmem, qd + 6, kd1 + 6, idesc, 1u);
+              ptx::mma_commit_multicast(empty_q + 8 * (qs >> 1), kClusterMask);
               if (++qs == nst) {
                 qs = 0;
                 qph ^= 1u;
@@ -317,8 +359,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int half = ew >> 2;             // column slice
     constexpr int kColsPerWarp = BN * 4 / kEpiWarps;
     constexpr int kChunks = kColsPerWarp / 32;
+    // this warp's private slice of the screen terms when they are staged
+    float* my_tau = reinterpret_cast<float*>(smem + L.tauoff()) + ew * kColsPerWarp;
     const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
-    float* my_tau = tau_s + ew * kColsPerWarp;  // private to this warp
     int t = 0;
     bool ok = true;
     unsigned long long ncand = 0;
@@ -327,17 +370,23 @@ __global__ void __launch_bounds__(kThreads, 1)
     while (ok && rc.next(a, rank, kt, qt0, qt1)) {
       const bool live = kt < a.n_kt;
       const int key0 = kt * BN + half * kColsPerWarp;
-      // this warp's screen terms for the run's key tile, staged once per
-      // run, and their minimum over each 32-key chunk
-      __syncwarp();
-      if (live)
-        for (int v4 = lane; v4 < kColsPerWarp / 4; v4 += 32)
-          reinterpret_cast<float4*>(my_tau)[v4] = __ldg(reinterpret_cast<const float4*>(a.tau + key0) + v4);
-      __syncwarp();
+      // the minimum of this warp's screen terms over each 32-key chunk of
+      // the run's key tile. The per-pair test, which few chunks reach, reads
+      // the terms themselves from a copy in shared memory made here when the
+      // runs are short, else through L1 (the space goes to a deeper query
+      // ring).
+      if (kTauStaged) {
+        __syncwarp();
+        if (live)
+          for (int v4 = lane; v4 < kColsPerWarp / 4; v4 += 32)
+            reinterpret_cast<float4*>(my_tau)[v4] = __ldg(reinterpret_cast<const float4*>(a.tau + key0) + v4);
+        __syncwarp();
+      }
+      const float* __restrict__ tau_g = a.tau + key0;
       float tmin[kChunks];
 #pragma unroll
       for (int ch = 0; ch < kChunks; ++ch) {
-        float m = live ? my_tau[ch * 32 + lane] : INFINITY;
+        float m = !live ? INFINITY : kTauStaged ? my_tau[ch * 32 + lane] : __ldg(tau_g + ch * 32 + lane);
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) m = fminf(m, __shfl_xor_sync(0xffffffffu, m, o));
         tmin[ch] = m;
@@ -373,9 +422,14 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             if (__fsub_rn(fmaxf(m0, m1), tmin[ch]) >= kap) {
               uint32_t mask = 0;
+              if (kTauStaged) {
 #pragma unroll
-              for (int j = 0; j < 32; ++j)
-                mask |= (uint32_t)(__uint_as_float(v[j]) - my_tau[ch * 32 + j] >= kap) << j;
+                for (int j = 0; j < 32; ++j) mask |= (uint32_t)(__uint_as_float(v[j]) - my_tau[ch * 32 + j] >= kap) << j;
+              } else {
+#pragma unroll
+                for (int j = 0; j < 32; ++j)
+                  mask |= (uint32_t)(__uint_as_float(v[j]) - __ldg(tau_g + ch * 32 + j) >= kap) << j;
+              }
               const float* qrow = a.qpad + (size_t)row * a.dpad;
               while (mask) {
                 const int j = __ffs(mask) - 1;
@@ -448,14 +502,23 @@ void launch(lipcache* h, int64_t B, const float* qpad, const float* kappa, unsig
   }
   TcArgs a;
   a.nch = h->dpad / kChunkF;
-  a.nst = Layout<BN>::stages_for(a.nch);
-  LC_REQUIRE(a.nst >= 2, LIPCACHE_E_INVALID, "key tile does not fit shared memory");
+  // (the ring depth depends on whether the screen terms are staged: below)
   a.dpad = h->dpad;
   a.nq = (int)(Bpad / kBM);
   const int64_t n_kt = (h->size + BN - 1) / BN;
   const int64_t n_pairs = (n_kt + kCluster - 1) / kCluster;
   const int max_clusters = h->num_sms / kCluster;
   LC_REQUIRE(max_clusters >= 1, LIPCACHE_E_CUDA, "device has fewer than two SMs");
+  // Long ranges (many items per cluster, the large caches): the screen terms
+  // are read through L1, the shared memory goes to the query ring, and the
+  // stages are released two at a time (one commit per pair) when a tile's
+  // stages pair up and the ring holds whole pairs. Short ranges keep the
+  // staged screen terms and single releases, which measure faster there.
+  const bool long_ranges = n_pairs * a.nq / max_clusters >= kPairedReleaseItems;
+  a.tau_staged = long_ranges ? 0 : 1;
+  a.nst = Layout<BN>::stages_for(a.nch, a.tau_staged);
+  LC_REQUIRE(a.nst >= 2, LIPCACHE_E_INVALID, "key tile does not fit shared memory");
+  a.qgroup = (long_ranges && a.nst % 2 == 0 && a.nch % 2 == 0) ? 2 : 1;
   LC_REQUIRE(n_pairs * a.nq < (1LL << 40), LIPCACHE_E_INVALID, "too many work items");
   a.n_pairs = (int)n_pairs;
   a.n_kt = (int)n_kt;
@@ -467,12 +530,14 @@ void launch(lipcache* h, int64_t B, const float* qpad, const float* kappa, unsig
   a.best = best;
   a.stats = h->stats;
   a.debug_stall = (h->debug_flags & LIPCACHE_DEBUG_STALL_PROBE) ? 1 : 0;
-  const Layout<BN> L{a.nch, a.nst};
+  const Layout<BN> L{a.nch, a.nst, a.tau_staged};
   const int smem = L.total() + 1024;
   if (pl.smem == 0) {
     // the attribute belongs to the kernel, not to this cache: set it to the
     // largest size any shape uses, so other caches' launches stay valid
-    LC_CUDA(cudaFuncSetAttribute(k_probe_tc<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBudget + 1024));
+    LC_CUDA(cudaFuncSetAttribute(k_probe_tc<BN, 0>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBudget + 1024));
+    LC_CUDA(cudaFuncSetAttribute(k_probe_tc<BN, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBudget + 1024));
+    LC_CUDA(cudaFuncSetAttribute(k_probe_tc<BN, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBudget + 1024));
     pl.smem = kSmemBudget + 1024;
   }
   cudaLaunchConfig_t cfg = {};
@@ -488,7 +553,7 @@ void launch(lipcache* h, int64_t B, const float* qpad, const float* kappa, unsig
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   // persistent grid: no more clusters than can be resident at once
-  if (pl.resident == 0) LC_CUDA(cudaOccupancyMaxActiveClusters(&pl.resident, k_probe_tc<BN>, &cfg));
+  if (pl.resident == 0) LC_CUDA(cudaOccupancyMaxActiveClusters(&pl.resident, k_probe_tc<BN, 0>, &cfg));
   const int resident = pl.resident;
   LC_REQUIRE(resident >= 1, LIPCACHE_E_CUDA, "no CTA pair of the probe kernel fits on this device");
   int clusters = max_clusters < resident ? max_clusters : resident;
@@ -497,7 +562,9 @@ void launch(lipcache* h, int64_t B, const float* qpad, const float* kappa, unsig
   h->last_grid = clusters * kCluster;
   h->last_cluster = kCluster;
   if (h->launch_event) LC_CUDA(cudaEventRecord(h->launch_event, s));
-  LC_CUDA(cudaLaunchKernelEx(&cfg, k_probe_tc<BN>, pl.tmQ, pl.tmK, a));
+  void (*kern)(CUtensorMap, CUtensorMap, TcArgs) =
+      a.tau_staged ? k_probe_tc<BN, 0> : a.qgroup == 2 ? k_probe_tc<BN, 2> : k_probe_tc<BN, 1>;
+  LC_CUDA(cudaLaunchKernelEx(&cfg, kern, pl.tmQ, pl.tmK, a));
   LC_LAUNCH_CHECK("k_probe_tc");
 }
 
