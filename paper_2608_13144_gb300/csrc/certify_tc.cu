@@ -414,6 +414,71 @@ __device__ __forceinline__ void refine2(uint32_t ws, uint32_t wchunk, uint32_t z
   }
 }
 
+// The same compensated dot product W_c . z_r + b_c as refine2, for one
+// (row, class) pair on one lane, with the same bits: the eight chains of
+// refine2's group (lane s: features s, s + 8, s + 16, ... in ascending order)
+// run side by side in this lane, then the group's butterfly (xor 4, 2, 1) is
+// taken in the same tree inside the lane, then the bias. TwoSum's error term
+// is the exact rounding error whichever operand comes first and FP32 addition
+// commutes, so after each level every lane of refine2's group holds the pair
+// this lane holds (checked by an FP32 emulation of both layouts on the CPU).
+// Eight independent chains per lane instead of one, and no shuffles. The
+// chains are scalar: packing them two to an FP32x2 register costs a move per
+// operand and a sign flip per product on the integer pipe, which measured
+// slower. The next span's four 16-byte loads are issued before this span's
+// arithmetic.
+__device__ __forceinline__ void refine_lane(uint32_t ws, uint32_t wchunk, uint32_t zs, int c, int r, float bias, int d,
+                                            float& hi, float& lo) {
+  const uint32_t xw = (uint32_t)c & 7u, xz = (uint32_t)r & 7u;
+  const uint32_t wrow = ws + (uint32_t)c * 128u, zrow = zs + (uint32_t)r * 128u;
+  // span i: features 8 i .. 8 i + 7 = units 2 (i % 4) (chains 0-3) and
+  // 2 (i % 4) + 1 (chains 4-7) of chunk i / 4, swizzled with the row mod 8;
+  // the second unit's address is the first's with bit 4 flipped
+  auto aw = [&](int i) { return wrow + (uint32_t)(i >> 2) * wchunk + (((2u * (uint32_t)(i & 3)) ^ xw) << 4); };
+  auto az = [&](int i) { return zrow + (uint32_t)(i >> 2) * kZChunkBytes + (((2u * (uint32_t)(i & 3)) ^ xz) << 4); };
+  float p[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f}, cc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+  auto span = [&](const float4& w0, const float4& w1, const float4& z0, const float4& z1) {
+    const float w[8] = {w0.x, w0.y, w0.z, w0.w, w1.x, w1.y, w1.z, w1.w};
+    const float x[8] = {z0.x, z0.y, z0.z, z0.w, z1.x, z1.y, z1.z, z1.w};
+#pragma unroll
+    for (int s = 0; s < 8; ++s) {
+      const float pr = __fmul_rn(w[s], x[s]);  // TwoProduct: pr + er = w x
+      const float er = __fmaf_rn(w[s], x[s], -pr);
+      const float sm = __fadd_rn(p[s], pr);    // TwoSum(p, pr) = sm + q
+      const float bb = __fsub_rn(sm, p[s]);
+      const float q = __fadd_rn(__fsub_rn(p[s], __fsub_rn(sm, bb)), __fsub_rn(pr, bb));
+      p[s] = sm;
+      cc[s] = __fadd_rn(cc[s], __fadd_rn(q, er));
+    }
+  };
+  const int nsp = d >> 3;  // (d % 16 == 0)
+  float4 w0 = lds_f4(aw(0)), w1 = lds_f4(aw(0) ^ 16u), z0 = lds_f4(az(0)), z1 = lds_f4(az(0) ^ 16u);
+#pragma unroll 2
+  for (int i = 0; i < nsp; ++i) {
+    const int n = i + 1 < nsp ? i + 1 : i;  // (the last span loads itself again)
+    const uint32_t anw = aw(n), anz = az(n);
+    const float4 nw0 = lds_f4(anw), nw1 = lds_f4(anw ^ 16u), nz0 = lds_f4(anz), nz1 = lds_f4(anz ^ 16u);
+    span(w0, w1, z0, z1);
+    w0 = nw0;
+    w1 = nw1;
+    z0 = nz0;
+    z1 = nz1;
+  }
+#pragma unroll
+  for (int o = kGroupTc / 2; o > 0; o >>= 1) {
+#pragma unroll
+    for (int s = 0; s < o; ++s) {
+      float t, q;
+      two_sum(p[s], p[s + o], t, q);
+      p[s] = t;
+      cc[s] = __fadd_rn(__fadd_rn(cc[s], cc[s + o]), q);
+    }
+  }
+  float t, q;
+  two_sum(p[0], bias, t, q);
+  two_sum(t, __fadd_rn(cc[0], q), hi, lo);
+}
+
 // The tight radius (Eq. 29) of one row on one warp, for rows the screen
 // cannot settle (several possible y^G, Mb not below 1e38, more candidates than
 // slots): every class refined with the compensated dot product by the four
@@ -748,6 +813,27 @@ __global__ void __launch_bounds__(kThreads, 1)
     auto pass1_chunk = [&](const uint32_t (&v)[32], int ch, float (&t1)[4], float (&t2)[4]) {
       const int lim = min(32, C - ch * 32);
       const float4* b4 = reinterpret_cast<const float4*>(bias_s + ch * 32);
+      if (lim == 32) {
+        // a full chunk, two values at a time: with hi / lo the larger /
+        // smaller of the two, the new second largest is the largest of t2,
+        // min(t1, hi) and lo (five min / max for two values instead of six,
+        // and no mask)
+#pragma unroll
+        for (int j4 = 0; j4 < 8; ++j4) {
+          const float4 bb = b4[j4];
+          const float bv[4] = {bb.x, bb.y, bb.z, bb.w};
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            const int k = 2 * (j4 & 1) + h;  // tracker
+            const float sa = __fadd_rn(__uint_as_float(v[4 * j4 + 2 * h]), bv[2 * h]);
+            const float sb = __fadd_rn(__uint_as_float(v[4 * j4 + 2 * h + 1]), bv[2 * h + 1]);
+            const float hi2 = fmaxf(sa, sb), lo2 = fminf(sa, sb);
+            t2[k] = ptx::max3_f32(t2[k], fminf(t1[k], hi2), lo2);
+            t1[k] = fmaxf(t1[k], hi2);
+          }
+        }
+        return;
+      }
 #pragma unroll
       for (int j4 = 0; j4 < 8; ++j4) {
         const float4 bb = b4[j4];
@@ -1016,28 +1102,19 @@ __global__ void __launch_bounds__(kThreads, 1)
       __syncwarp();
       if (lane == 0) ptx::mbar_arrive(accempty + 8 * buf);  // the accumulator is free for tile t + 2
 
-      // refinement: the four groups take eight pairs of the list at a time
-      // (balanced over the warp) and store hi / lo at the pair's (row, slot)
+      // refinement: each lane takes one pair of the list at a time
+      // (refine_lane, the bits of refine2) and stores hi / lo at the pair's
+      // (row lane, slot) = e & 0xff: lane + 32 slot
       const int rq = quarter * 32;  // first row of the warp
-      for (int p0 = 0; p0 < P; p0 += 2 * (32 / kGroupTc)) {
-        const int i0 = p0 + 2 * g8, i1 = i0 + 1;
-        const int e0 = list[i0 < P ? i0 : p0], e1 = list[i1 < P ? i1 : p0];
-        const int cp[2] = {e0 >> 8, e1 >> 8};
-        const int rp[2] = {rq + (e0 & 31), rq + (e1 & 31)};
-        const float bp[2] = {bias_s[cp[0]], bias_s[cp[1]]};
-        float hi[2], lo[2];
-        refine2(s_w, wchunk, zs, cp, rp, bp, d, sub, hi, lo);
-        if (sub == 0) {
-          if (i0 < P) {
-            res_hi[(e0 & 0xff)] = hi[0];  // (row lane, slot) = e & 0xff: lane + 32 slot
-            res_lo[(e0 & 0xff)] = lo[0];
-          }
-          if (i1 < P) {
-            res_hi[(e1 & 0xff)] = hi[1];
-            res_lo[(e1 & 0xff)] = lo[1];
-          }
-        }
+      for (int i = lane; i < P; i += 32) {
+        const int e = list[i];
+        const int c = e >> 8;
+        float hi, lo;
+        refine_lane(s_w, wchunk, zs, c, rq + (e & 31), bias_s[c], d, hi, lo);
+        res_hi[e & 0xff] = hi;
+        res_lo[e & 0xff] = lo;
       }
+      __syncwarp();  // every refined pair is visible to its row's lane
       if constexpr (!TIGHT) {
         __syncwarp();
         // each row's lane pushes its own candidates into its running selection

@@ -1,0 +1,153 @@
+"""The certify kernels' compensated refinement (Dot2 of Ogita, Rump and
+Oishi: TwoProduct and TwoSum per feature, then the bias) computed in two
+layouts must give the same bits, emulated here in FP32 on the CPU.
+
+Group layout (every FP32 certify kernel, and the tensor kernel's one-warp
+paths): eight lanes share one (row, class) pair; lane s runs the chain over
+the features k = s, s + 8, s + 16, ... in ascending order, the eight chains
+are combined by a butterfly over the group (xor 4, 2, 1: TwoSum of the two
+partial sums, the compensation terms added, then the TwoSum error), and the
+bias is added last.
+
+Lane layout (the tensor kernel's candidate list): one lane takes the whole
+pair and runs the same eight chains side by side, then combines them in the
+butterfly's tree inside the lane: (0,4) (1,5) (2,6) (3,7), then (0,2)
+(1,3), then (0,1).
+
+The two agree because TwoSum's error term is the exact rounding error of the
+sum whichever operand comes first, and FP32 addition is commutative, so
+every lane of the group holds the same pair after each level. These tests
+check that, and that the group's eight lanes agree, on random, cancelling
+and sign-mixed inputs, with d from 16 to 256.
+"""
+import numpy as np
+import pytest
+
+f32 = np.float32
+
+
+def _add(a, b):
+    return (a + b).astype(f32)
+
+
+def _sub(a, b):
+    return (a - b).astype(f32)
+
+
+def _two_sum(a, b):
+    s = _add(a, b)
+    bb = _sub(s, a)
+    e = _add(_sub(a, _sub(s, bb)), _sub(b, bb))
+    return s, e
+
+
+def _two_prod(w, x):
+    pr = (w * x).astype(f32)
+    # fma(w, x, -pr): the product of two FP32 values is exact in FP64 and its
+    # rounding error is an FP32 value, so one rounding of the FP64 difference
+    # is the fused result
+    er = (w.astype(np.float64) * x.astype(np.float64) - pr.astype(np.float64)).astype(f32)
+    return pr, er
+
+
+def _chains(W, Z):
+    """The eight per-residue chains (P, CC) of every pair: W, Z (n, d) FP32."""
+    n, d = W.shape
+    P = np.zeros((8, n), f32)
+    CC = np.zeros((8, n), f32)
+    for s in range(8):
+        for k in range(s, d, 8):
+            pr, er = _two_prod(W[:, k], Z[:, k])
+            sm = _add(P[s], pr)
+            bb = _sub(sm, P[s])
+            q = _add(_sub(P[s], _sub(sm, bb)), _sub(pr, bb))
+            P[s] = sm
+            CC[s] = _add(CC[s], _add(q, er))
+    return P, CC
+
+
+def _finish(p, cc, bias):
+    t, q = _two_sum(p, bias)
+    return _two_sum(t, _add(cc, q))
+
+
+def refine_group(W, Z, bias):
+    """Eight lanes, butterfly by shuffles: returns every lane's (hi, lo)."""
+    P, CC = _chains(W, Z)
+    p, cc = P.copy(), CC.copy()
+    for o in (4, 2, 1):
+        pn, ccn = np.empty_like(p), np.empty_like(cc)
+        for s in range(8):
+            t, q = _two_sum(p[s], p[s ^ o])        # own value first, then the partner's
+            pn[s] = t
+            ccn[s] = _add(_add(cc[s], cc[s ^ o]), q)
+        p, cc = pn, ccn
+    return [_finish(p[s], cc[s], bias) for s in range(8)]
+
+
+def refine_lane(W, Z, bias):
+    """One lane, the same tree inside the lane."""
+    P, CC = _chains(W, Z)
+    p, cc = list(P), list(CC)
+    for o in (4, 2, 1):
+        for s in range(o):
+            t, q = _two_sum(p[s], p[s + o])
+            cc[s] = _add(_add(cc[s], cc[s + o]), q)
+            p[s] = t
+    return _finish(p[0], cc[0], bias)
+
+
+def _bits(x):
+    return np.asarray(x, f32).view(np.uint32)
+
+
+def _cases(rng, n, d):
+    W = rng.standard_normal((n, d)).astype(f32) / f32(np.sqrt(d))
+    Z = (rng.standard_normal((n, d)) * 3.0).astype(f32)
+    bias = (rng.standard_normal(n) * 0.1).astype(f32)
+    # cancelling pairs: the bias nearly cancels the dot product
+    m = n // 4
+    dots = (W[:m].astype(np.float64) * Z[:m].astype(np.float64)).sum(1)
+    bias[:m] = (-dots).astype(f32)
+    # features spanning many binades, exact zeros and negative zeros
+    Z[m:2 * m] *= (2.0 ** rng.integers(-30, 30, size=(m, d))).astype(f32)
+    Z[2 * m:2 * m + m // 2, ::3] = f32(0.0)
+    Z[2 * m + m // 2:3 * m, ::5] = f32(-0.0)
+    # halves that cancel term by term: exact dot products of zero
+    h = d // 2
+    W[3 * m:3 * m + 8, h:] = W[3 * m:3 * m + 8, :h]
+    Z[3 * m:3 * m + 8, h:] = -Z[3 * m:3 * m + 8, :h]
+    bias[3 * m:3 * m + 8] = f32(0.0)
+    return W, Z, bias
+
+
+@pytest.mark.parametrize("d", [16, 32, 48, 64, 128, 256])
+def test_lane_layout_matches_group_layout(d):
+    rng = np.random.default_rng(1000 + d)
+    W, Z, bias = _cases(rng, 4000, d)
+    group = refine_group(W, Z, bias)
+    hi, lo = refine_lane(W, Z, bias)
+    for s in range(8):  # every lane of the group ends with the same pair
+        assert np.array_equal(_bits(group[s][0]), _bits(group[0][0])), s
+        assert np.array_equal(group[s][1], group[0][1]), s
+    assert np.array_equal(_bits(hi), _bits(group[0][0]))
+    assert np.array_equal(hi, group[0][0]) and np.array_equal(lo, group[0][1])
+
+
+def test_refinement_is_compensated():
+    """The emulation itself is Dot2: hi + lo is within a few units of 2^-48
+    of the scale of the exact dot product plus bias (a dropped error term or
+    a wrong sign in TwoSum would leave FP32-sized errors)."""
+    from fractions import Fraction
+    rng = np.random.default_rng(7)
+    d = 128
+    W, Z, bias = _cases(rng, 400, d)
+    hi, lo = refine_lane(W, Z, bias)
+    worst = 0.0
+    for i in range(0, 400, 7):
+        exact = sum(Fraction(float(W[i, k])) * Fraction(float(Z[i, k])) for k in range(d)) + Fraction(float(bias[i]))
+        got = Fraction(float(hi[i])) + Fraction(float(lo[i]))
+        scale = float(np.abs(W[i].astype(np.float64) * Z[i].astype(np.float64)).sum() + abs(float(bias[i])))
+        if scale > 0:
+            worst = max(worst, abs(float(got - exact)) / scale)
+    assert worst < 2.0 ** -40, worst
