@@ -479,6 +479,77 @@ __device__ __forceinline__ void refine_lane(uint32_t ws, uint32_t wchunk, uint32
   two_sum(t, __fadd_rn(cc[0], q), hi, lo);
 }
 
+// refine_lane with the pair shared by K = 2 or 4 lanes (t = lane % K), for
+// the last pairs of a list, which would leave most lanes of a whole round
+// idle. K = 2: lane t runs chains 4 t .. 4 t + 3 (the 16-byte unit 2 jj + t
+// of each span); the butterfly's first level (chain s with s + 4) is a
+// shuffle with lane t ^ 1, the others stay in the lane. K = 4: lane t runs
+// chains t and t + 4 (word t of both units); the first level is in the lane,
+// the second (s with s + 2) a shuffle with lane t ^ 2, the third with t ^ 1.
+// Every lane of the K returns the same bits as refine_lane. All 32 lanes call
+// it together (the shuffles take the whole warp).
+template <int K>
+__device__ __forceinline__ void refine_lanes(uint32_t ws, uint32_t wchunk, uint32_t zs, int c, int r, float bias, int d,
+                                             int t, float& hi, float& lo) {
+  static_assert(K == 2 || K == 4, "two or four lanes per pair");
+  constexpr int NC = 8 / K;  // chains per lane
+  const uint32_t xw = (uint32_t)c & 7u, xz = (uint32_t)r & 7u;
+  const uint32_t wrow = ws + (uint32_t)c * 128u, zrow = zs + (uint32_t)r * 128u;
+  float p[NC], cc[NC];
+#pragma unroll
+  for (int j = 0; j < NC; ++j) p[j] = cc[j] = 0.f;
+  auto step = [&](int j, float w, float x) {
+    const float pr = __fmul_rn(w, x);
+    const float er = __fmaf_rn(w, x, -pr);
+    const float sm = __fadd_rn(p[j], pr);
+    const float bb = __fsub_rn(sm, p[j]);
+    const float q = __fadd_rn(__fsub_rn(p[j], __fsub_rn(sm, bb)), __fsub_rn(pr, bb));
+    p[j] = sm;
+    cc[j] = __fadd_rn(cc[j], __fadd_rn(q, er));
+  };
+  const int nsp = d >> 3;
+  for (int i = 0; i < nsp; ++i) {
+    const uint32_t u = 2u * (uint32_t)(i & 3);  // first unit of the span
+    const uint32_t ow = (uint32_t)(i >> 2) * wchunk, oz = (uint32_t)(i >> 2) * kZChunkBytes;
+    if constexpr (K == 2) {
+      const float4 w = lds_f4(wrow + ow + (((u + (uint32_t)t) ^ xw) << 4));
+      const float4 z = lds_f4(zrow + oz + (((u + (uint32_t)t) ^ xz) << 4));
+      step(0, w.x, z.x);
+      step(1, w.y, z.y);
+      step(2, w.z, z.z);
+      step(3, w.w, z.w);
+    } else {
+      float w0, w1, z0, z1;
+      asm volatile("ld.shared.f32 %0, [%1];" : "=f"(w0) : "r"(wrow + ow + ((u ^ xw) << 4) + 4u * (uint32_t)t));
+      asm volatile("ld.shared.f32 %0, [%1];" : "=f"(w1) : "r"(wrow + ow + (((u + 1u) ^ xw) << 4) + 4u * (uint32_t)t));
+      asm volatile("ld.shared.f32 %0, [%1];" : "=f"(z0) : "r"(zrow + oz + ((u ^ xz) << 4) + 4u * (uint32_t)t));
+      asm volatile("ld.shared.f32 %0, [%1];" : "=f"(z1) : "r"(zrow + oz + (((u + 1u) ^ xz) << 4) + 4u * (uint32_t)t));
+      step(0, w0, z0);  // chain t
+      step(1, w1, z1);  // chain t + 4
+    }
+  }
+  auto comb = [](float& pa, float& ca, float pb, float cb) {
+    float s, q;
+    two_sum(pa, pb, s, q);
+    pa = s;
+    ca = __fadd_rn(__fadd_rn(ca, cb), q);
+  };
+  if constexpr (K == 2) {
+#pragma unroll
+    for (int j = 0; j < 4; ++j) comb(p[j], cc[j], __shfl_xor_sync(kFull, p[j], 1), __shfl_xor_sync(kFull, cc[j], 1));
+    comb(p[0], cc[0], p[2], cc[2]);
+    comb(p[1], cc[1], p[3], cc[3]);
+    comb(p[0], cc[0], p[1], cc[1]);
+  } else {
+    comb(p[0], cc[0], p[1], cc[1]);
+    comb(p[0], cc[0], __shfl_xor_sync(kFull, p[0], 2), __shfl_xor_sync(kFull, cc[0], 2));
+    comb(p[0], cc[0], __shfl_xor_sync(kFull, p[0], 1), __shfl_xor_sync(kFull, cc[0], 1));
+  }
+  float tt, q;
+  two_sum(p[0], bias, tt, q);
+  two_sum(tt, __fadd_rn(cc[0], q), hi, lo);
+}
+
 // The tight radius (Eq. 29) of one row on one warp, for rows the screen
 // cannot settle (several possible y^G, Mb not below 1e38, more candidates than
 // slots): every class refined with the compensated dot product by the four
@@ -1104,15 +1175,34 @@ __global__ void __launch_bounds__(kThreads, 1)
 
       // refinement: each lane takes one pair of the list at a time
       // (refine_lane, the bits of refine2) and stores hi / lo at the pair's
-      // (row lane, slot) = e & 0xff: lane + 32 slot
+      // (row lane, slot) = e & 0xff: lane + 32 slot. A last round of at most
+      // 16 (8) pairs shares each pair between two (four) lanes
+      // (refine_lanes), so that it takes about half (a quarter) of a whole
+      // round.
       const int rq = quarter * 32;  // first row of the warp
-      for (int i = lane; i < P; i += 32) {
+      const int pfull = (P & 31) > 16 ? P : P & ~31;
+      for (int i = lane; i < pfull; i += 32) {
         const int e = list[i];
         const int c = e >> 8;
         float hi, lo;
         refine_lane(s_w, wchunk, zs, c, rq + (e & 31), bias_s[c], d, hi, lo);
         res_hi[e & 0xff] = hi;
         res_lo[e & 0xff] = lo;
+      }
+      if (pfull < P) {  // (warp-uniform)
+        const int kk = P - pfull > 8 ? 2 : 4;
+        const int i = pfull + lane / kk;
+        const int e = list[i < P ? i : pfull];
+        const int c = e >> 8;
+        float hi, lo;
+        if (kk == 2)
+          refine_lanes<2>(s_w, wchunk, zs, c, rq + (e & 31), bias_s[c], d, lane & 1, hi, lo);
+        else
+          refine_lanes<4>(s_w, wchunk, zs, c, rq + (e & 31), bias_s[c], d, lane & 3, hi, lo);
+        if (i < P && lane % kk == 0) {
+          res_hi[e & 0xff] = hi;
+          res_lo[e & 0xff] = lo;
+        }
       }
       __syncwarp();  // every refined pair is visible to its row's lane
       if constexpr (!TIGHT) {

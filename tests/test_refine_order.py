@@ -12,7 +12,9 @@ bias is added last.
 Lane layout (the tensor kernel's candidate list): one lane takes the whole
 pair and runs the same eight chains side by side, then combines them in the
 butterfly's tree inside the lane: (0,4) (1,5) (2,6) (3,7), then (0,2)
-(1,3), then (0,1).
+(1,3), then (0,1). For the last few pairs of a list, two lanes share a pair
+(lane t: chains 4t..4t+3, the first level across the two lanes) or four do
+(lane t: chains t and t+4, the first level in the lane, the others across).
 
 The two agree because TwoSum's error term is the exact rounding error of the
 sum whichever operand comes first, and FP32 addition is commutative, so
@@ -97,6 +99,40 @@ def refine_lane(W, Z, bias):
     return _finish(p[0], cc[0], bias)
 
 
+def refine_split(W, Z, bias, K):
+    """K lanes per pair: returns every lane's (hi, lo); each lane combines its
+    own value first, as the kernel does."""
+    P, CC = _chains(W, Z)
+    if K == 2:
+        # lane t holds chains 4t..4t+3 as local 0..3
+        lanes = [[list(P[4 * t:4 * t + 4]), list(CC[4 * t:4 * t + 4])] for t in range(2)]
+        new = []
+        for t in range(2):
+            p, cc = [x.copy() for x in lanes[t][0]], [x.copy() for x in lanes[t][1]]
+            for j in range(4):
+                s_, q = _two_sum(p[j], lanes[t ^ 1][0][j])
+                cc[j] = _add(_add(cc[j], lanes[t ^ 1][1][j]), q)
+                p[j] = s_
+            for a, b in ((0, 2), (1, 3), (0, 1)):
+                s_, q = _two_sum(p[a], p[b])
+                cc[a] = _add(_add(cc[a], cc[b]), q)
+                p[a] = s_
+            new.append(_finish(p[0], cc[0], bias))
+        return new
+    # K == 4: lane t holds chains t and t + 4; first level in the lane
+    vals = []
+    for t in range(4):
+        s_, q = _two_sum(P[t], P[t + 4])
+        vals.append((s_, _add(_add(CC[t], CC[t + 4]), q)))
+    for o in (2, 1):
+        nv = []
+        for t in range(4):
+            s_, q = _two_sum(vals[t][0], vals[t ^ o][0])
+            nv.append((s_, _add(_add(vals[t][1], vals[t ^ o][1]), q)))
+        vals = nv
+    return [_finish(v[0], v[1], bias) for v in vals]
+
+
 def _bits(x):
     return np.asarray(x, f32).view(np.uint32)
 
@@ -132,6 +168,17 @@ def test_lane_layout_matches_group_layout(d):
         assert np.array_equal(group[s][1], group[0][1]), s
     assert np.array_equal(_bits(hi), _bits(group[0][0]))
     assert np.array_equal(hi, group[0][0]) and np.array_equal(lo, group[0][1])
+
+
+@pytest.mark.parametrize("K", [2, 4])
+@pytest.mark.parametrize("d", [16, 48, 128])
+def test_split_lanes_match_lane_layout(d, K):
+    rng = np.random.default_rng(2000 + d + K)
+    W, Z, bias = _cases(rng, 3000, d)
+    hi, lo = refine_lane(W, Z, bias)
+    for h, l in refine_split(W, Z, bias, K):  # every lane of the K
+        assert np.array_equal(_bits(h), _bits(hi))
+        assert np.array_equal(_bits(l), _bits(lo))
 
 
 def test_refinement_is_compensated():
