@@ -1439,13 +1439,25 @@ struct ScatterArgs {
 // Append accepted rows in input order. Each warp moves kScatterRows rows:
 // lane u < kScatterRows resolves row u's destination and copies its
 // per-entry fields, then the warp copies the keys of all its rows with every
-// load issued before the stores (float4s for 16-byte rows).
+// load issued before the stores (float4s for 16-byte rows). The first 128
+// floats of every row are loaded before the destinations are known: those
+// loads depend on nothing (the rows were just read by the certify kernel and
+// mostly sit in L2), so they overlap the chain of dependent loads that
+// resolves the destinations; a rejected row is read for nothing.
 constexpr int kScatterRows = 8;
 
 __global__ void __launch_bounds__(256) k_scatter(ScatterArgs a, int vec) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int64_t row0 = ((int64_t)blockIdx.x * 8 + warp) * kScatterRows;
   if (row0 >= a.n) return;
+  const int n4 = a.dpad / 4, d4 = a.d / 4;
+  float4 v0[kScatterRows];
+  if (vec) {
+#pragma unroll
+    for (int u = 0; u < kScatterRows; ++u)
+      v0[u] = (row0 + u < a.n && lane < d4) ? __ldg(reinterpret_cast<const float4*>(a.H + (size_t)(row0 + u) * a.d) + lane)
+                                            : make_float4(0.f, 0.f, 0.f, 0.f);
+  }
   int64_t mydst = -2;  // past the end
   if (lane < kScatterRows && row0 + lane < a.n) {
     const int64_t row = row0 + lane;
@@ -1466,8 +1478,12 @@ __global__ void __launch_bounds__(256) k_scatter(ScatterArgs a, int vec) {
 #pragma unroll
   for (int u = 0; u < kScatterRows; ++u) dst[u] = __shfl_sync(0xffffffffu, mydst, u);
   if (vec) {
-    const int n4 = a.dpad / 4, d4 = a.d / 4;
-    for (int j4 = lane; j4 < n4; j4 += 32) {
+    if (lane < n4) {
+#pragma unroll
+      for (int u = 0; u < kScatterRows; ++u)
+        if (dst[u] >= 0) reinterpret_cast<float4*>(a.t.keys + (size_t)dst[u] * a.dpad)[lane] = v0[u];
+    }
+    for (int j4 = lane + 32; j4 < n4; j4 += 32) {
       float4 v[kScatterRows];
 #pragma unroll
       for (int u = 0; u < kScatterRows; ++u)
