@@ -976,13 +976,34 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       crude &= lim == 32 ? 0xffffffffu : (1u << lim) - 1u;
       uint32_t mask = exact ? 0u : crude;
+      // a full chunk with 16-byte aligned bracket rows: each half's 16
+      // brackets in four 16-byte loads, by the lanes with a class there
+      const bool vec4 = lim == 32 && (C & 3) == 0;
 #pragma unroll
       for (int h16 = 0; h16 < 2; ++h16) {
         float p[16];
+        if (vec4) {
+          const uint32_t hb = (crude >> (16 * h16)) & 0xffffu;
+          if (exact && hb) {
+            const float4* src = reinterpret_cast<const float4*>(irow + ch * 32 + 16 * h16);
 #pragma unroll
-        for (int k = 0; k < 16; ++k) {
-          const int j = 16 * h16 + k;
-          p[k] = (exact && ((crude >> j) & 1u)) ? __ldg(irow + ch * 32 + j) : 0.f;
+            for (int i = 0; i < 4; ++i) {
+              const float4 q = __ldg(src + i);
+              p[4 * i] = q.x;
+              p[4 * i + 1] = q.y;
+              p[4 * i + 2] = q.z;
+              p[4 * i + 3] = q.w;
+            }
+          } else {
+#pragma unroll
+            for (int k = 0; k < 16; ++k) p[k] = 0.f;
+          }
+        } else {
+#pragma unroll
+          for (int k = 0; k < 16; ++k) {
+            const int j = 16 * h16 + k;
+            p[k] = (exact && ((crude >> j) & 1u)) ? __ldg(irow + ch * 32 + j) : 0.f;
+          }
         }
 #pragma unroll
         for (int k = 0; k < 16; ++k) {
