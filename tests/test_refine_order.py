@@ -16,7 +16,10 @@ butterfly's tree inside the lane: (0,4) (1,5) (2,6) (3,7), then (0,2)
 (lane t: chains 4t..4t+3, the first level across the two lanes) or four do
 (lane t: chains t and t+4, the first level in the lane, the others across).
 
-The two agree because TwoSum's error term is the exact rounding error of the
+The last test checks the first screening pass's update of the top two s~ of a
+chunk two values at a time against the one-at-a-time tracker.
+
+The two layouts agree because TwoSum's error term is the exact rounding error of the
 sum whichever operand comes first, and FP32 addition is commutative, so
 every lane of the group holds the same pair after each level. These tests
 check that, and that the group's eight lanes agree, on random, cancelling
@@ -198,3 +201,46 @@ def test_refinement_is_compensated():
         if scale > 0:
             worst = max(worst, abs(float(got - exact)) / scale)
     assert worst < 2.0 ** -40, worst
+
+
+def _top2_sequential(vals):
+    """The first pass's tracker, one value at a time: t2 = max(t2, min(t1, s)),
+    t1 = max(t1, s)."""
+    t1 = t2 = -np.inf
+    for s_ in vals:
+        t2 = max(t2, min(t1, s_))
+        t1 = max(t1, s_)
+    return t1, t2
+
+
+def _top2_pairs(vals):
+    """The tensor kernel's first pass on a full chunk, two values at a time:
+    with hi / lo the larger / smaller of the two, t2 = max(t2, min(t1, hi), lo)
+    and t1 = max(t1, hi)."""
+    t1 = t2 = -np.inf
+    for a, b in zip(vals[0::2], vals[1::2]):
+        hi, lo = max(a, b), min(a, b)
+        t2 = max(t2, min(t1, hi), lo)
+        t1 = max(t1, hi)
+    return t1, t2
+
+
+def test_first_pass_pairs_match_sequential_top_two():
+    """The two-at-a-time update keeps the same largest and second-largest
+    value (ties counted twice) as the one-at-a-time tracker, on random values,
+    heavy ties and infinities."""
+    rng = np.random.default_rng(11)
+    for trial in range(3000):
+        n = 2 * int(rng.integers(1, 17))
+        kind = trial % 3
+        if kind == 0:
+            v = rng.standard_normal(n).astype(np.float32)
+        elif kind == 1:
+            v = rng.integers(-3, 4, size=n).astype(np.float32)  # many exact ties
+        else:
+            v = rng.standard_normal(n).astype(np.float32)
+            v[rng.random(n) < 0.3] = -np.inf
+        vals = [float(x) for x in v]
+        assert _top2_pairs(vals) == _top2_sequential(vals), vals
+        srt = sorted(vals, reverse=True)
+        assert _top2_sequential(vals) == (srt[0], srt[1])
