@@ -16,14 +16,13 @@ butterfly's tree inside the lane: (0,4) (1,5) (2,6) (3,7), then (0,2)
 (lane t: chains 4t..4t+3, the first level across the two lanes) or four do
 (lane t: chains t and t+4, the first level in the lane, the others across).
 
-The last test checks the first screening pass's update of the top two s~ of a
-chunk two values at a time against the one-at-a-time tracker.
-
-The two layouts agree because TwoSum's error term is the exact rounding error of the
-sum whichever operand comes first, and FP32 addition is commutative, so
+The layouts agree because TwoSum's error term is the exact rounding error of
+the sum whichever operand comes first, and FP32 addition is commutative, so
 every lane of the group holds the same pair after each level. These tests
 check that, and that the group's eight lanes agree, on random, cancelling
-and sign-mixed inputs, with d from 16 to 256.
+and sign-mixed inputs, with d from 16 to 256. The last test checks the
+first screening pass's update of the top two s~ of a chunk, two values at a
+time, against the one-at-a-time tracker.
 """
 import numpy as np
 import pytest
